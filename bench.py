@@ -1,0 +1,369 @@
+"""Benchmark of the Flash-BoN draft path on GB300: draft candidates/s at the
+Wan2.1-1.3B shape.
+
+Workload (one "step" = one pass of the whole hot path over one batch):
+  Wan2.1-1.3B-shaped DiT (30 blocks, hidden 1536, 12 x 128 heads, FFN 8960, text
+  512 x 4096 projected to 1536), 480x832 image -> 16 x 60 x 104 latent -> 1560 tokens;
+  N = 32 candidates drafted over the first 10 steps of a 50-step flow-matching schedule
+  (t_i = 1 - i/50) with 1/3 of the blocks skipped per step (seeded) and, on odd steps,
+  half of the remaining blocks proxied from the previous step's cached contribution;
+  then candidate 0 is refined with full computation over the remaining 40 steps.
+  Synthetic bf16 random-init weights N(0, 0.02), latents and text context N(0, 1).
+
+value = candidates per second (N / step time) with inputs resident in HBM; e2e = the
+same through the C-ABI with host (pinned) latents and text, copies inside the timed
+region. The working set (2.6 GB of weights, 0.5-1 GB activations per kernel) is far
+larger than L2, so no L2 flush is done between steps.
+
+--impl reference times the CPU oracle (fp64 numpy) on a bounded sample of the same
+workload and extrapolates the same metric.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+from paper_2607_04461_gb300 import synth  # noqa: E402
+
+METRIC = "draft candidates/sec at Wan2.1-1.3B shape (1 GB300); tensor-pipe % of bf16 peak"
+N_CAND, S_TOTAL, S_DRAFT = 32, 50, 10
+SKIP_FRAC, PROXY_FRAC, PLAN_SEED = 1 / 3, 0.5, 7
+
+
+def workload():
+    cfg = synth.WAN13.with_(max_n=N_CAND)
+    sched = synth.make_schedule(S_TOTAL)
+    skip, proxy = synth.random_plan(S_DRAFT, cfg.depth, SKIP_FRAC, PROXY_FRAC, seed=PLAN_SEED)
+    return cfg, sched, skip, proxy
+
+
+def config_dict(cfg):
+    return {"workload": "wan2.1-1.3B draft pool: N=32, 480x832 (1560 tokens), 10 of 50 "
+                        "steps, 1/3 blocks skipped, half of the rest proxied on odd steps, "
+                        "then a 40-step full refine of candidate 0",
+            "n_candidates": N_CAND, "tokens": cfg.tokens, "dim": cfg.dim, "depth": cfg.depth,
+            "draft_steps": S_DRAFT, "refine_steps": S_TOTAL - S_DRAFT,
+            "l2": "inputs larger than L2 (2.6 GB weights), no flush"}
+
+
+def block_flops(cfg):
+    """Algorithmic FLOPs of one block for one candidate (cross K/V hoisted)."""
+    P, D, F, T = cfg.tokens, cfg.dim, cfg.ffn, cfg.text_len
+    lin = 2 * P * D * (3 * D + D + D + D) + 4 * P * D * F
+    attn = 4 * P * P * D + 4 * P * T * D
+    return lin + attn
+
+
+def computed_blocks(skip, proxy):
+    return int(((skip == 0) & (proxy == -1)).sum())
+
+
+# ---------------------------------------------------------------------------------
+# clocks during the timed region
+# ---------------------------------------------------------------------------------
+class ClockSampler:
+    Q = ("clocks.sm,clocks.max.sm,clocks_event_reasons.hw_slowdown,"
+         "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+         "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index):
+        self.index, self.proc = index, None
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.Q}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except Exception:
+            self.proc = None
+        return self
+
+    def __exit__(self, *exc):
+        self.lines = []
+        if self.proc:
+            self.proc.terminate()
+            try:
+                out, _ = self.proc.communicate(timeout=5)
+            except Exception:
+                self.proc.kill()
+                out = ""
+            self.lines = [l for l in out.splitlines() if l.strip()]
+
+    def summary(self):
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for l in getattr(self, "lines", []):
+            f = [x.strip() for x in l.split(",")]
+            try:
+                sm.append(float(f[0]))
+                mx.append(float(f[1]))
+            except (ValueError, IndexError):
+                continue
+            for n, v in zip(names, f[2:]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"]}
+        return {"sm_mhz": float(np.median(sm)), "sm_max_mhz": max(mx),
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# ---------------------------------------------------------------------------------
+# oracle (CPU) timing: bounded sample, extrapolated
+# ---------------------------------------------------------------------------------
+def oracle_sample(cfg, sched, skip, proxy, budget_s):
+    """Times the oracle's block on candidate 0 at step 0 (blocks in order) until the
+    budget is spent; returns (seconds per computed block, blocks timed)."""
+    from oracle import OracleModel
+    n_blocks = max(1, min(cfg.depth, int(budget_s // 2) or 1))
+    w = synth.make_weights(cfg, layers=range(n_blocks))
+    sub = cfg.with_(depth=n_blocks)
+    ref = OracleModel(sub, {k: v for k, v in w.items()})
+    ctx = synth.make_text(cfg)
+    kv = ref.encode_text(ctx)
+    z = synth.make_latents(cfg, 1)[0]
+    temb, mod = ref.time_embed(sched[0])
+    h = ref.patch_embed(z)
+    t0 = time.perf_counter()
+    done = 0
+    for l in range(n_blocks):
+        h = ref.block(l, h, mod, kv[l])
+        done += 1
+        if time.perf_counter() - t0 > budget_s:
+            break
+    return (time.perf_counter() - t0) / done, done
+
+
+def oracle_cands_per_s(per_block_s, cfg, skip, proxy):
+    blocks = N_CAND * computed_blocks(skip, proxy) + (S_TOTAL - S_DRAFT) * cfg.depth
+    return N_CAND / (blocks * per_block_s)
+
+
+# ---------------------------------------------------------------------------------
+def read_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as fh:
+            d = json.load(fh)
+        return d, "measured"
+    return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}, "fallback"
+
+
+def gemm_traffic_per_launch():
+    """DRAM bytes per tcgen05 GEMM launch from the committed ncu summary, if it was taken
+    on the current kernel source (else None)."""
+    src = os.path.join(ROOT, "paper_2607_04461_gb300", "csrc", "gemm_tc.cu")
+    summ = os.path.join(ROOT, "profiles", "gemm_tc_wan13.md")
+    if not os.path.exists(summ):
+        return None
+    sha = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
+    vals = {}
+    for line in open(summ):
+        if line.startswith("bench-key "):
+            k, _, v = line[len("bench-key "):].partition(":")
+            vals[k.strip()] = v.strip()
+    if vals.get("kernel_sha") != sha or "traffic_bytes_per_launch" not in vals:
+        return None
+    return float(vals["traffic_bytes_per_launch"])
+
+
+def dist_env():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return ws, rank, local
+
+
+def run_reference(args):
+    ws, rank, _ = dist_env()
+    if rank != 0:
+        return 0
+    cfg, sched, skip, proxy = workload()
+    per_step = max(2.0, min(20.0, 120.0 / max(1, args.steps + args.warmup)))
+    times = []
+    for i in range(args.warmup + args.steps):
+        pb, nb = oracle_sample(cfg, sched, skip, proxy, per_step)
+        if i >= args.warmup:
+            times.append(pb)
+    pb = float(np.median(times))
+    v = oracle_cands_per_s(pb, cfg, skip, proxy)
+    cores = os.cpu_count()
+    sample = (f"fp64 numpy oracle: Wan2.1-1.3B block forward of candidate 0 at step 0, "
+              f"{nb} block(s) per step ({pb:.2f} s per block), extrapolated to the "
+              f"workload's {N_CAND * computed_blocks(skip, proxy)} draft + "
+              f"{(S_TOTAL - S_DRAFT) * cfg.depth} refine block evaluations")
+    line = {"impl": "reference", "metric": METRIC, "value": v, "unit": "candidates/s",
+            "n_gpus": ws, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": 1e3 * N_CAND / v, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": config_dict(cfg),
+            "cpu_baseline": {"value": v, "unit": "candidates/s", "cores": cores,
+                             "kind": "oracle", "sample": sample},
+            "e2e": {"value": v, "unit": "candidates/s", "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+    print(json.dumps(line))
+    return 0
+
+
+def run_gb300(args):
+    import torch
+    from paper_2607_04461_gb300 import flashbon as fb
+
+    ws, rank, local = dist_env()
+    torch.cuda.set_device(local)
+    pg = None
+    if ws > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+        pg = dist
+    cfg, sched, skip, proxy = workload()
+    t_setup = time.time()
+    w = synth.make_weights(cfg)
+    model = fb.Model(cfg, w)
+    del w
+    stream = torch.cuda.Stream()
+    model.set_stream(stream)
+    # each rank drafts its own 32 candidates (weak scaling, no collective on the path)
+    z0 = torch.from_numpy(synth.make_latents(cfg, N_CAND, first=rank * N_CAND)).cuda()
+    ctx_h = synth.make_text(cfg)
+    ctx = torch.from_numpy(ctx_h).cuda()
+    z = torch.empty_like(z0)
+    zr = torch.empty_like(z0[0])
+    draft_sched, tail = sched[: S_DRAFT + 1], sched[S_DRAFT:]
+    setup_s = time.time() - t_setup
+
+    def dev_step():
+        with torch.cuda.stream(stream):
+            z.copy_(z0)
+        model.draft(z, ctx, draft_sched, skip, proxy)
+        with torch.cuda.stream(stream):
+            zr.copy_(z[0])
+        model.refine(zr, ctx, tail)
+
+    for _ in range(args.warmup):
+        dev_step()
+    torch.cuda.synchronize()
+    model.reset_stats()
+    model.set_timing(1 << fb.K["gemm_tc"])
+    if pg:
+        pg.barrier()
+    torch.cuda.synchronize()
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(local) as clk:
+        ev0.record(stream)
+        for _ in range(args.steps):
+            dev_step()
+        ev1.record(stream)
+        torch.cuda.synchronize()
+    ms = ev0.elapsed_time(ev1)
+    stats = model.stats()
+    model.set_timing(0)
+    if pg:
+        t = torch.tensor([ms], device="cuda")
+        pg.all_reduce(t, op=pg.ReduceOp.MAX)
+        ms = float(t.item())
+        pg.barrier()
+    ms_step = ms / args.steps
+    value = ws * N_CAND / (ms_step / 1e3)
+
+    # end to end through the C-ABI with host buffers (pinned), copies inside the region
+    zh = torch.empty(z0.shape, dtype=torch.float32, pin_memory=True)
+    zrh = torch.empty(z0.shape[1:], dtype=torch.float32, pin_memory=True)
+    ctxh = torch.from_numpy(ctx_h).pin_memory()
+    z0h = z0.cpu()
+    model.set_stream(None)
+
+    def host_step():
+        zh.copy_(z0h)
+        model.draft(zh, ctxh, draft_sched, skip, proxy)
+        zrh.copy_(zh[0])
+        model.refine(zrh, ctxh, tail)
+
+    host_step()
+    torch.cuda.synchronize()
+    if pg:
+        pg.barrier()
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        host_step()
+    e2e_s = (time.perf_counter() - t0) / args.steps
+    if pg:
+        t = torch.tensor([e2e_s], device="cuda")
+        pg.all_reduce(t, op=pg.ReduceOp.MAX)
+        e2e_s = float(t.item())
+    zbytes = z0.numel() * 4
+    h2d = zbytes + 2 * ctx_h.nbytes + zbytes // N_CAND
+    d2h = zbytes + zbytes // N_CAND
+
+    peaks, peak_kind = read_peaks()
+    g = stats["gemm_tc"]
+    achieved = g["flops"] / (g["ms"] / 1e3) / 1e12 if g["ms"] > 0 else None
+    peak = peaks["bf16_tflops_sustained"]
+    traffic = gemm_traffic_per_launch()
+    launches = sum(s["launches"] for s in stats.values())
+    algo_flops = N_CAND * computed_blocks(skip, proxy) * block_flops(cfg) + \
+        (S_TOTAL - S_DRAFT) * cfg.depth * block_flops(cfg)
+    out = {"metric": METRIC, "value": value, "unit": "candidates/s", "n_gpus": ws,
+           "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_step,
+           "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+           "data": "synthetic", "config": config_dict(cfg),
+           "roofline": {"bound": "tensor", "kernel": "gemm_tc (tcgen05/TMEM GEMM, all "
+                        "projections)", "achieved": achieved, "peak": peak,
+                        "unit": "TFLOP/s", "frac": (achieved / peak) if achieved else None,
+                        "peak_kind": f"bf16 sustained, {peak_kind}",
+                        "traffic": traffic,
+                        "launches": g["launches"], "ms": g["ms"] / args.steps},
+           "step_tflops": algo_flops / (ms_step / 1e3) / 1e12,
+           "step_frac_of_peak": algo_flops / (ms_step / 1e3) / 1e12 / peak,
+           "e2e": {"value": ws * N_CAND / e2e_s, "unit": "candidates/s",
+                   "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h)},
+           "gpu_launches": int(launches),
+           "clocks": clk.summary(),
+           "kernels": {k: {"launches": v["launches"] // args.steps,
+                           "gflop": v["flops"] / args.steps / 1e9}
+                       for k, v in stats.items() if v["launches"]},
+           "setup_s": setup_s}
+    if rank == 0 and ws == 1 and not args.no_cpu_baseline:
+        pb, nb = oracle_sample(cfg, sched, skip, proxy, args.cpu_budget)
+        v = oracle_cands_per_s(pb, cfg, skip, proxy)
+        out["cpu_baseline"] = {
+            "value": v, "unit": "candidates/s", "cores": os.cpu_count(), "kind": "oracle",
+            "sample": f"fp64 numpy oracle, {nb} Wan2.1-1.3B block forward(s) of one candidate "
+                      f"({pb:.2f} s each), extrapolated to the step's "
+                      f"{N_CAND * computed_blocks(skip, proxy)} draft + "
+                      f"{(S_TOTAL - S_DRAFT) * cfg.depth} refine block evaluations"}
+    if rank == 0:
+        print(json.dumps(out))
+    model.close()
+    if pg:
+        pg.destroy_process_group()
+    return 0
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=3)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
+    ap.add_argument("--cpu-budget", type=float, default=15.0)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.impl == "reference":
+        return run_reference(args)
+    return run_gb300(args)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

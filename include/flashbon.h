@@ -1,0 +1,189 @@
+/* flashbon.h -- C-ABI of the GB300 (sm_103a) Flash-BoN draft-generation library.
+ *
+ * The library runs the hot path of Flash-BoN ("Instant Drafts for Inference-Time
+ * Scaling in Diffusion Models"): a pool of N seed-varied candidates is denoised by a
+ * DiT flow-matching model under the paper's three acceleration knobs (§4.1):
+ * a truncated timestep schedule (early stopping), a per-step layer-skip set (Eq. 6)
+ * and activation proxies (Eqs. 3-5) that stand in for a block's computation; then one
+ * selected latent is refined with full computation (§4.2, Stage 3).
+ *
+ * Conventions for every entry point:
+ *  - Return an fb_status; they never abort. fb_last_error() gives a message for the
+ *    last failing call on the calling thread.
+ *  - The caller owns every input and output buffer. The model owns its device weights,
+ *    activation buffers and the proxy cache.
+ *  - All work is enqueued on the model's stream (fb_set_stream, default: a stream the
+ *    model creates) and the call returns after that stream has finished the work.
+ *  - "host or device" pointers are classified with cudaPointerGetAttributes: device
+ *    (or managed) memory is used in place; host memory is staged through device
+ *    buffers inside the call.
+ *  - A device-side wait that exceeds its time limit (about two seconds) makes the
+ *    kernel give up, and the call returns FB_ECUDA with "device wait timed out".
+ */
+#ifndef FLASHBON_H
+#define FLASHBON_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum fb_status {
+  FB_OK = 0,
+  FB_EINVAL = 1,  /* bad argument: null pointer, size out of range, bad schedule */
+  FB_ENOMEM = 2,  /* device or host allocation failed */
+  FB_ECUDA = 3,   /* a CUDA call or a kernel failed, or a device wait timed out */
+  FB_EPLAN = 4,   /* malformed skip_mask / proxy_plan */
+  FB_ESTATE = 5   /* call out of order, e.g. block forward before fb_encode_text */
+} fb_status;
+
+/* Model shape. Linear weights are [out][in]. dim = heads * head_dim; head_dim is 64
+ * or 128; latent_h and latent_w are multiples of patch; patch_dim =
+ * latent_c * patch * patch <= 64. max_n bounds the candidates per call (buffers are
+ * sized for max_n * tokens rows). eps_ln: LayerNorm epsilon; eps_rms: RMSNorm epsilon;
+ * rope_theta: RoPE base; freq_dim: sinusoidal timestep-embedding width (even). */
+typedef struct fb_cfg {
+  int depth, dim, heads, head_dim, ffn, text_len, text_dim;
+  int latent_c, latent_h, latent_w, patch, max_n, freq_dim;
+  float eps_ln, eps_rms, rope_theta;
+} fb_cfg;
+
+typedef struct fb_model fb_model;
+
+/* ---- weight layout -------------------------------------------------------------
+ * The packed host weight buffer is fp32, tensors back to back in entry order
+ * 0..count-1. Entry order and names:
+ *   patch.w [D][C p p], patch.b [D], time.w1 [D][freq_dim], time.b1 [D],
+ *   time.w2 [D][D], time.b2 [D], mod.w [6D][D], mod.b [6D], text.w1 [D][text_dim],
+ *   text.b1 [D], text.w2 [D][D], text.b2 [D], head.table [2][D], head.w [C p p][D],
+ *   head.b [C p p], then for each block l = 0..depth-1 with prefix "blocks.<l>.":
+ *   table [6][D], attn.wqkv [3D][D], attn.bqkv [3D], attn.norm_q [D],
+ *   attn.norm_k [D], attn.wo [D][D], attn.bo [D], norm3.w [D], norm3.b [D],
+ *   cross.wq [D][D], cross.bq [D], cross.wkv [2D][D], cross.bkv [2D],
+ *   cross.norm_q [D], cross.norm_k [D], cross.wo [D][D], cross.bo [D],
+ *   ffn.w1 [F][D], ffn.b1 [F], ffn.w2 [D][F], ffn.b2 [D].
+ * fb_weights_entry: name (static string), element offset into the packed buffer and
+ * element count of entry idx. FB_EINVAL for idx out of range or a bad cfg. */
+fb_status fb_weights_count(const fb_cfg* cfg, int* count, size_t* total_elems);
+fb_status fb_weights_entry(const fb_cfg* cfg, int idx, const char** name,
+                           size_t* offset, size_t* numel);
+
+/* ---- model --------------------------------------------------------------------
+ * fb_init_model: validates cfg, copies the packed fp32 host weights to the device as
+ * bf16 (matrices) and fp32 (biases, norm scales, modulation tables), allocates the
+ * activation buffers for max_n candidates. *out is NULL on failure. The denoiser is
+ * the black-box f_theta of §3 (a DiT); the block follows Eq. 7. */
+fb_status fb_init_model(const fb_cfg* cfg, const float* weights_host, fb_model** out);
+void fb_free(fb_model* m);
+/* stream: a cudaStream_t (NULL = the model's own stream). */
+fb_status fb_set_stream(fb_model* m, void* stream);
+
+/* fb_encode_text: text projection of the prompt embedding x (§3) and, per block, the
+ * cross-attention keys and values; they do not change across steps or candidates and
+ * are kept in the model. text_ctx: [text_len][text_dim] fp32, host or device. */
+fb_status fb_encode_text(fb_model* m, const float* text_ctx);
+
+/* ---- the draft and refine calls (§4.2 Stages 1 and 3) -------------------------
+ * fb_draft: Stage 1 (Eq. 8) for n candidates (0 <= n <= max_n; n == 0 is a no-op).
+ *  latents:  [n][latent_c][latent_h][latent_w] fp32, host or device; in: z_T per
+ *            candidate; out: the latent after n_steps steps (the cached draft state).
+ *  text_ctx: as fb_encode_text (encoded once per call).
+ *  schedule: n_steps + 1 fp32 host values, strictly decreasing, in [0, 1]; step i goes
+ *            from t = schedule[i] to t' = schedule[i+1] with the Euler update
+ *            z <- z + (t' - t) v of the flow-matching ODE (App. A.1). Early stopping
+ *            (§4.1, knob 1) is a schedule that ends before t = 0.
+ *  skip_mask:  [n_steps][depth] uint8 host; 1 = skip the block (Eq. 6).
+ *  proxy_plan: [n_steps][depth] int32 host; -1 = compute the block (Eq. 7); otherwise
+ *            src_step | (order << 16), 0 <= order <= 2: the block's contribution
+ *            Delta = B(h) - h is forecast by the Taylor expansion of Eqs. 3-5 from the
+ *            contributions cached at the layer's most recent computed steps at or before
+ *            src_step (most recent first; the order drops while fewer than order + 1
+ *            exist) and added to h. The layer must have been computed at src_step,
+ *            src_step < the current step, and the entry's skip bit must be 0.
+ *            NULL skip_mask / proxy_plan mean "no skip" / "compute everything".
+ *  Errors: FB_EINVAL (sizes, schedule), FB_EPLAN (plan rules above), FB_ENOMEM (proxy
+ *  cache growth), FB_ECUDA. Latents are unchanged unless FB_OK is returned for a
+ *  device pointer... (a device buffer may be partially updated on FB_ECUDA). */
+fb_status fb_draft(fb_model* m, float* latents, int n, const float* text_ctx,
+                   const float* schedule, int n_steps, const uint8_t* skip_mask,
+                   const int32_t* proxy_plan);
+
+/* fb_refine: Stage 3 (§4.2): resumes one latent [latent_c][latent_h][latent_w]
+ * (host or device, in/out) with full computation (no skip, no proxy) over
+ * full_schedule (n_steps + 1 values, as fb_draft). Valid because sampling is
+ * Markovian: the result depends only on the latent it starts from. */
+fb_status fb_refine(fb_model* m, float* latent, const float* text_ctx,
+                    const float* full_schedule, int n_steps);
+
+/* fb_plan_from_phi: expands phi = (S', n_skip, l_start, l_end, f_full) (§4.1,
+ * "Configuration Space") into skip_mask [S'][depth] and proxy_plan [S'][depth]
+ * (caller-allocated host arrays). Layers l_start..l_end are 1-indexed as in the paper
+ * and are skipped at draft steps k >= n_skip; step k is a full step iff
+ * k mod f_full == 0; on other steps every non-skipped layer is proxied with the given
+ * order from the last full step. FB_EINVAL if 1 <= S' <= S, 1 <= l_start <= l_end <=
+ * depth, f_full >= 1, n_skip >= 0, 0 <= order <= 2 do not all hold. */
+fb_status fb_plan_from_phi(int S, int S_prime, int n_skip, int l_start, int l_end,
+                           int f_full, int order, int depth, uint8_t* skip_mask,
+                           int32_t* proxy_plan);
+
+/* fb_block_forward: one block B_layer (Eq. 7) in place on h [n * tokens][dim] fp32
+ * DEVICE memory (candidate-major rows), with the modulation of timestep t and the
+ * text context of the last fb_encode_text (FB_ESTATE without one). */
+fb_status fb_block_forward(fb_model* m, int layer, float* h, int n, float t);
+
+const char* fb_last_error(void);
+
+/* ---- statistics ----------------------------------------------------------------
+ * Per kernel class: launches, summed device time (ms; measured with CUDA events on the
+ * model's stream while timing is on) and algorithmic FLOPs and bytes of the launches. */
+enum {
+  FB_K_GEMM_TC = 0,   /* tcgen05/TMEM GEMM (all epilogues) */
+  FB_K_GEMM_SIMT,     /* CUDA-core GEMM for shapes the tcgen05 kernel does not tile */
+  FB_K_ATTN_SELF,     /* self-attention */
+  FB_K_ATTN_CROSS,    /* cross-attention */
+  FB_K_NORM,          /* LayerNorm + modulation */
+  FB_K_QKNORM,        /* q/k RMSNorm + RoPE */
+  FB_K_PROXY,         /* activation-proxy residual add */
+  FB_K_EMBED,         /* patch embedding */
+  FB_K_HEAD,          /* head + Euler update */
+  FB_K_SMALL,         /* timestep embedding, modulation, conversions */
+  FB_K_COUNT
+};
+typedef struct fb_kstat {
+  uint64_t launches;
+  double ms, flops, bytes;
+} fb_kstat;
+fb_status fb_set_timing(fb_model* m, int on);
+fb_status fb_get_stats(fb_model* m, fb_kstat* out /* [FB_K_COUNT] */);
+fb_status fb_reset_stats(fb_model* m);
+const char* fb_kernel_name(int kind);
+
+/* ---- single-op entry points (DEVICE pointers; enqueued on the model's stream) ---
+ * They run one kernel of the path on caller buffers, for kernel-level parity tests.
+ *
+ * fb_op_gemm: D[M][N] = A[M][K] * W[N][K]^T + bias[N] with epilogue `epi`:
+ *   0: out bf16 = acc + bias
+ *   1: out bf16 = gelu_tanh(acc + bias)
+ *   2: out fp32 = resid[M][N] + gate[N] * (acc + bias)  (gate may be NULL = 1; resid may
+ *      equal out)
+ *   3: as 2, and also delta bf16 = out - base[M][N] (fp32), base may equal out
+ * A, W bf16 row-major, leading dimensions K; out / resid / base / delta leading
+ * dimension N. impl: 0 = automatic (tcgen05 when N % 128 == 0 and K % 64 == 0),
+ * 1 = force the CUDA-core kernel. */
+fb_status fb_op_gemm(fb_model* m, int M, int N, int K, const void* A, const void* W,
+                     const float* bias, int epi, void* out, const float* resid,
+                     const float* gate, const float* base, void* delta, int impl);
+/* fb_op_attention: O = softmax(Q K^T / sqrt(head_dim)) V per (batch, head), bf16 row
+ * major; Q rows b*Lq..b*Lq+Lq-1 with row stride ldq elements, head h at column
+ * h*head_dim; likewise K, V (kv_batch_rows = 0 shares one K/V across the batch,
+ * otherwise the row offset between batches); O row stride ldo. */
+fb_status fb_op_attention(fb_model* m, const void* Q, int ldq, const void* K, int ldk,
+                          const void* V, int ldv, void* O, int ldo, int batch, int Lq,
+                          int Lkv, int kv_batch_rows, int heads, int head_dim);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* FLASHBON_H */

@@ -1,0 +1,905 @@
+// C-ABI of libflashbon.so: model set-up, the host dispatcher of the draft path and the
+// single-op entry points. See include/flashbon.h for the contract of each call.
+//
+// The dispatcher turns (schedule, skip_mask, proxy_plan) into one launch list per step:
+// a computed block is its chain of kernels (norms, tcgen05 GEMMs, attention), a run of
+// proxied blocks (skipped blocks between them are no-ops, Eq. 6) is ONE proxy_add
+// launch, a skipped block launches nothing. Cached contributions Delta_l are written by
+// the epilogue of the block's last GEMM into a ring of anchor slots; slots are assigned
+// on the host from the plan, so only contributions some later proxy reads are stored.
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <map>
+#include <string>
+#include <vector>
+
+#include "../../include/flashbon.h"
+#include "kernels.h"
+
+namespace {
+
+thread_local std::string g_last_error;
+
+fb_status fail(fb_status s, const char* fmt, ...) {
+  char buf[512];
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(buf, sizeof buf, fmt, ap);
+  va_end(ap);
+  g_last_error = buf;
+  return s;
+}
+
+#define CK(call)                                                                    \
+  do {                                                                              \
+    cudaError_t e_ = (call);                                                        \
+    if (e_ != cudaSuccess)                                                          \
+      return fail(FB_ECUDA, "%s failed: %s (%s:%d)", #call, cudaGetErrorString(e_), \
+                  __FILE__, __LINE__);                                              \
+  } while (0)
+#define CKS(call)                  \
+  do {                             \
+    fb_status s_ = (call);         \
+    if (s_ != FB_OK) return s_;    \
+  } while (0)
+
+enum WKind { W_MAT, W_VEC };
+struct WEntry {
+  std::string name;
+  size_t numel;
+  WKind kind;
+};
+
+std::vector<WEntry> weight_table(const fb_cfg& c) {
+  const size_t D = c.dim, F = c.ffn, PD = (size_t)c.latent_c * c.patch * c.patch;
+  std::vector<WEntry> t = {
+      {"patch.w", D * PD, W_MAT}, {"patch.b", D, W_VEC},
+      {"time.w1", D * c.freq_dim, W_MAT}, {"time.b1", D, W_VEC},
+      {"time.w2", D * D, W_MAT}, {"time.b2", D, W_VEC},
+      {"mod.w", 6 * D * D, W_MAT}, {"mod.b", 6 * D, W_VEC},
+      {"text.w1", D * c.text_dim, W_MAT}, {"text.b1", D, W_VEC},
+      {"text.w2", D * D, W_MAT}, {"text.b2", D, W_VEC},
+      {"head.table", 2 * D, W_VEC}, {"head.w", PD * D, W_MAT}, {"head.b", PD, W_VEC},
+  };
+  for (int l = 0; l < c.depth; ++l) {
+    const std::string p = "blocks." + std::to_string(l) + ".";
+    std::vector<WEntry> b = {
+        {p + "table", 6 * D, W_VEC},
+        {p + "attn.wqkv", 3 * D * D, W_MAT}, {p + "attn.bqkv", 3 * D, W_VEC},
+        {p + "attn.norm_q", D, W_VEC}, {p + "attn.norm_k", D, W_VEC},
+        {p + "attn.wo", D * D, W_MAT}, {p + "attn.bo", D, W_VEC},
+        {p + "norm3.w", D, W_VEC}, {p + "norm3.b", D, W_VEC},
+        {p + "cross.wq", D * D, W_MAT}, {p + "cross.bq", D, W_VEC},
+        {p + "cross.wkv", 2 * D * D, W_MAT}, {p + "cross.bkv", 2 * D, W_VEC},
+        {p + "cross.norm_q", D, W_VEC}, {p + "cross.norm_k", D, W_VEC},
+        {p + "cross.wo", D * D, W_MAT}, {p + "cross.bo", D, W_VEC},
+        {p + "ffn.w1", F * D, W_MAT}, {p + "ffn.b1", F, W_VEC},
+        {p + "ffn.w2", D * F, W_MAT}, {p + "ffn.b2", D, W_VEC},
+    };
+    t.insert(t.end(), b.begin(), b.end());
+  }
+  return t;
+}
+
+bool ln_width_ok(int D) {
+  switch (D) {
+    case 128: case 256: case 512: case 1024: case 1536: case 2048: case 3072: case 4096:
+    case 5120:
+      return true;
+  }
+  return false;
+}
+
+fb_status check_cfg(const fb_cfg* c) {
+  if (!c) return fail(FB_EINVAL, "cfg is NULL");
+  if (c->depth < 1 || c->dim < 1 || c->heads < 1 || c->ffn < 1 || c->text_len < 1 ||
+      c->text_dim < 1 || c->latent_c < 1 || c->patch < 1 || c->max_n < 1 || c->freq_dim < 2)
+    return fail(FB_EINVAL, "cfg: sizes must be positive");
+  if (c->head_dim != 64 && c->head_dim != 128)
+    return fail(FB_EINVAL, "cfg: head_dim must be 64 or 128");
+  if (c->heads * c->head_dim != c->dim) return fail(FB_EINVAL, "cfg: dim != heads * head_dim");
+  if (!ln_width_ok(c->dim)) return fail(FB_EINVAL, "cfg: unsupported dim %d", c->dim);
+  if (c->latent_h % c->patch || c->latent_w % c->patch || c->latent_h < c->patch ||
+      c->latent_w < c->patch)
+    return fail(FB_EINVAL, "cfg: latent size must be a positive multiple of patch");
+  const int pd = c->latent_c * c->patch * c->patch;
+  if (pd % 8 || pd > 64 || 256 % pd) return fail(FB_EINVAL, "cfg: C*p*p must be 8, 16, 32 or 64");
+  if (c->ffn % 8 || c->text_dim % 8 || c->freq_dim % 16)
+    return fail(FB_EINVAL, "cfg: ffn, text_dim multiple of 8; freq_dim multiple of 16");
+  if (!(c->eps_ln > 0) || !(c->eps_rms > 0) || !(c->rope_theta > 1))
+    return fail(FB_EINVAL, "cfg: eps must be > 0 and rope_theta > 1");
+  return FB_OK;
+}
+
+struct Layer {
+  bf16 *wqkv, *wo, *cq, *ckv, *co, *w1, *w2;
+  float *table, *bqkv, *nq, *nk, *bo, *n3w, *n3b, *cbq, *cbkv, *cnq, *cnk, *cbo, *b1, *b2;
+};
+
+struct Pending {
+  int kind;
+  cudaEvent_t a, b;
+};
+
+}  // namespace
+
+struct fb_model {
+  fb_cfg c;
+  int P, PD, gh, gw;
+  size_t Mmax;
+  int num_sms;
+  cudaStream_t own = nullptr, st = nullptr;
+  // weights
+  void* wmat = nullptr;  // bf16 matrices
+  void* wvec = nullptr;  // fp32 vectors (tables contiguous: per-layer tables first)
+  bf16 *patch_w, *time_w1, *time_w2, *mod_w, *text_w1, *text_w2, *head_w;
+  float *patch_b, *time_b1, *time_b2, *mod_b, *text_b1, *text_b2, *head_table, *head_b;
+  float* tables;  // [depth][6][D]
+  std::vector<Layer> L;
+  // activations
+  float *hA = nullptr, *hB = nullptr;
+  bf16 *act = nullptr, *qkv = nullptr, *ao = nullptr, *cqb = nullptr, *ffh = nullptr;
+  float* ctx_f = nullptr;
+  bf16 *ctx_b = nullptr, *ctx_h = nullptr, *ctx_p = nullptr, *kvctx = nullptr;
+  bool text_ready = false;
+  float *emb = nullptr, *th1 = nullptr, *temb = nullptr, *mod = nullptr, *modl = nullptr,
+        *hmod = nullptr;
+  float2* rope = nullptr;
+  float* zbuf = nullptr;
+  bf16* anchors = nullptr;
+  size_t anchor_elems = 0;
+  int* derr = nullptr;
+  int* herr = nullptr;  // pinned
+  // statistics
+  unsigned timing_mask = 0;
+  fb_kstat stats[FB_K_COUNT];
+  std::vector<Pending> pending;
+  std::vector<cudaEvent_t> ev_pool;
+  std::vector<void*> allocs;
+};
+
+namespace {
+
+// ---- allocation helpers -------------------------------------------------------------
+fb_status dalloc(fb_model* m, void** p, size_t bytes) {
+  *p = nullptr;
+  if (bytes == 0) bytes = 16;
+  cudaError_t e = cudaMalloc(p, bytes);
+  if (e != cudaSuccess) {
+    cudaGetLastError();
+    return fail(FB_ENOMEM, "cudaMalloc(%zu bytes) failed: %s", bytes, cudaGetErrorString(e));
+  }
+  m->allocs.push_back(*p);
+  return FB_OK;
+}
+template <typename T>
+fb_status dalloc_t(fb_model* m, T** p, size_t n) {
+  return dalloc(m, reinterpret_cast<void**>(p), n * sizeof(T));
+}
+
+// ---- statistics ---------------------------------------------------------------------
+struct KTimer {
+  fb_model* m;
+  int kind;
+  cudaEvent_t a = nullptr, b = nullptr;
+  KTimer(fb_model* mm, int k, double flops, double bytes, int nlaunch = 1) : m(mm), kind(k) {
+    m->stats[k].launches += nlaunch;
+    m->stats[k].flops += flops;
+    m->stats[k].bytes += bytes;
+    if (m->timing_mask & (1u << k)) {
+      a = get();
+      b = get();
+      if (a && b) cudaEventRecord(a, m->st);
+    }
+  }
+  cudaEvent_t get() {
+    if (!m->ev_pool.empty()) {
+      cudaEvent_t e = m->ev_pool.back();
+      m->ev_pool.pop_back();
+      return e;
+    }
+    cudaEvent_t e = nullptr;
+    if (cudaEventCreate(&e) != cudaSuccess) {
+      cudaGetLastError();
+      return nullptr;
+    }
+    return e;
+  }
+  ~KTimer() {
+    if (a && b) {
+      cudaEventRecord(b, m->st);
+      m->pending.push_back({kind, a, b});
+    } else {
+      if (a) m->ev_pool.push_back(a);
+      if (b) m->ev_pool.push_back(b);
+    }
+  }
+};
+
+void collect_timings(fb_model* m) {
+  for (auto& p : m->pending) {
+    float ms = 0.f;
+    if (cudaEventElapsedTime(&ms, p.a, p.b) == cudaSuccess) m->stats[p.kind].ms += ms;
+    else cudaGetLastError();
+    m->ev_pool.push_back(p.a);
+    m->ev_pool.push_back(p.b);
+  }
+  m->pending.clear();
+}
+
+// Starts an API call: clears the device error word.
+fb_status begin_call(fb_model* m) {
+  CK(cudaMemsetAsync(m->derr, 0, sizeof(int), m->st));
+  return FB_OK;
+}
+// Ends an API call: waits for the stream, checks the device error word.
+fb_status end_call(fb_model* m) {
+  CK(cudaMemcpyAsync(m->herr, m->derr, sizeof(int), cudaMemcpyDeviceToHost, m->st));
+  CK(cudaStreamSynchronize(m->st));
+  collect_timings(m);
+  if (*m->herr == FB_DEVERR_WAIT_TIMEOUT)
+    return fail(FB_ECUDA, "device wait timed out (a kernel gave up after its time limit)");
+  if (*m->herr != 0) return fail(FB_ECUDA, "device error %d", *m->herr);
+  return FB_OK;
+}
+
+// ---- kernel wrappers with statistics ------------------------------------------------
+fb_status run_gemm(fb_model* m, const GemmArgs& g, int force_simt = 0) {
+  const double flops = 2.0 * g.M * (double)g.N * g.K;
+  double bytes = 2.0 * ((double)g.M * g.K + (double)g.N * g.K);
+  bytes += (g.kind <= EPI_GELU_BF16) ? 2.0 * g.M * g.N : 8.0 * g.M * g.N;
+  if (g.kind == EPI_RESID_DELTA) bytes += 6.0 * g.M * g.N;
+  if (!force_simt && gemm_tc_supported(g)) {
+    KTimer t(m, FB_K_GEMM_TC, flops, bytes);
+    CK(gemm_tc(g, m->derr, m->num_sms, m->st));
+  } else {
+    KTimer t(m, FB_K_GEMM_SIMT, flops, bytes);
+    CK(gemm_simt(g, m->st));
+  }
+  return FB_OK;
+}
+
+GemmArgs gemm_args(int M, int N, int K, const bf16* A, const bf16* W, const float* bias,
+                   int kind, void* out) {
+  GemmArgs g{};
+  g.M = M; g.N = N; g.K = K;
+  g.A = A; g.lda = K;
+  g.W = W; g.ldw = K;
+  g.kind = kind;
+  g.epi.bias = bias;
+  g.epi.out = out;
+  g.epi.ldo = N;
+  return g;
+}
+
+fb_status run_attn(fb_model* m, const AttnArgs& a, int kind) {
+  const double flops = 4.0 * a.batch * a.heads * (double)a.Lq * a.Lkv * a.head_dim;
+  const double kvb = (a.kv_batch_rows ? a.batch : 1) * 2.0 * a.Lkv * a.heads * a.head_dim * 2;
+  const double bytes = 2.0 * a.batch * a.Lq * (double)a.heads * a.head_dim * 2 + kvb;
+  KTimer t(m, kind, flops, bytes);
+  CK(attention(a, m->st));
+  return FB_OK;
+}
+
+fb_status run_ln(fb_model* m, const float* x, bf16* out, int rows, float mb, const float* mul,
+                 const float* add) {
+  KTimer t(m, FB_K_NORM, 8.0 * rows * m->c.dim, 6.0 * rows * m->c.dim);
+  CK(ln_mod(x, out, rows, m->c.dim, m->c.eps_ln, mb, mul, add, m->st));
+  return FB_OK;
+}
+
+fb_status run_qkn(fb_model* m, bf16* x, int rows, int ld, int nseg, int col0, const float* w0,
+                  int col1, const float* w1, const float2* rope) {
+  KTimer t(m, FB_K_QKNORM, 6.0 * rows * nseg * m->c.dim, 4.0 * rows * nseg * m->c.dim);
+  CK(qk_norm_rope(x, rows, ld, m->c.dim, nseg, col0, w0, col1, w1, m->c.eps_rms, rope, m->P,
+                  m->c.head_dim, m->st));
+  return FB_OK;
+}
+
+// ---- text encoding (once per call) --------------------------------------------------
+fb_status encode_text(fb_model* m, const float* ctx) {
+  const fb_cfg& c = m->c;
+  const size_t nctx = (size_t)c.text_len * c.text_dim;
+  cudaPointerAttributes at{};
+  const float* src = ctx;
+  if (cudaPointerGetAttributes(&at, ctx) != cudaSuccess) cudaGetLastError();
+  if (at.type != cudaMemoryTypeDevice && at.type != cudaMemoryTypeManaged) {
+    CK(cudaMemcpyAsync(m->ctx_f, ctx, nctx * sizeof(float), cudaMemcpyHostToDevice, m->st));
+    src = m->ctx_f;
+  }
+  {
+    KTimer t(m, FB_K_SMALL, 0, 6.0 * nctx);
+    CK(f32_to_bf16(src, m->ctx_b, nctx, m->st));
+  }
+  const int T = c.text_len, D = c.dim;
+  CKS(run_gemm(m, gemm_args(T, D, c.text_dim, m->ctx_b, m->text_w1, m->text_b1, EPI_GELU_BF16,
+                            m->ctx_h)));
+  CKS(run_gemm(m, gemm_args(T, D, D, m->ctx_h, m->text_w2, m->text_b2, EPI_BF16, m->ctx_p)));
+  for (int l = 0; l < c.depth; ++l) {
+    bf16* kv = m->kvctx + (size_t)l * T * 2 * D;
+    CKS(run_gemm(m, gemm_args(T, 2 * D, D, m->ctx_p, m->L[l].ckv, m->L[l].cbkv, EPI_BF16, kv)));
+    CKS(run_qkn(m, kv, T, 2 * D, 1, 0, m->L[l].cnk, 0, m->L[l].cnk, nullptr));
+  }
+  m->text_ready = true;
+  return FB_OK;
+}
+
+// ---- per-step conditioning: temb, mod, per-layer modulation, head modulation ---------
+fb_status time_embed(fb_model* m, float t) {
+  const fb_cfg& c = m->c;
+  const int D = c.dim;
+  KTimer k(m, FB_K_SMALL, 2.0 * D * (c.freq_dim + D + 6.0 * D),
+           2.0 * D * (c.freq_dim + D + 6.0 * D), 5);
+  CK(timestep_sincos(t, c.freq_dim, m->emb, m->st));
+  CK(gemv(m->time_w1, m->time_b1, m->emb, m->th1, D, c.freq_dim, 0, 1, m->st));
+  CK(gemv(m->time_w2, m->time_b2, m->th1, m->temb, D, D, 0, 0, m->st));
+  CK(gemv(m->mod_w, m->mod_b, m->temb, m->mod, 6 * D, D, 1, 0, m->st));
+  CK(mod_prepare(m->mod, m->tables, c.depth, D, m->modl, m->head_table, m->temb, m->hmod, m->st));
+  return FB_OK;
+}
+
+// ---- one block B_l (Eq. 7) on h = hA (rows M), optional contribution write ----------
+fb_status block_forward(fb_model* m, int l, float* h, int n, bf16* delta) {
+  const fb_cfg& c = m->c;
+  const int D = c.dim, M = n * m->P;
+  const Layer& w = m->L[l];
+  const float* md = m->modl + (size_t)l * 6 * D;
+  const float *s1 = md, *c1 = md + D, *g1 = md + 2 * D, *s2 = md + 3 * D, *c2 = md + 4 * D,
+              *g2 = md + 5 * D;
+  float* hB = m->hB;
+  // self-attention branch
+  CKS(run_ln(m, h, m->act, M, 1.f, c1, s1));
+  CKS(run_gemm(m, gemm_args(M, 3 * D, D, m->act, w.wqkv, w.bqkv, EPI_BF16, m->qkv)));
+  CKS(run_qkn(m, m->qkv, M, 3 * D, 2, 0, w.nq, D, w.nk, m->rope));
+  {
+    AttnArgs a{};
+    a.Q = m->qkv; a.K = m->qkv + D; a.V = m->qkv + 2 * D; a.O = m->ao;
+    a.ldq = a.ldk = a.ldv = 3 * D; a.ldo = D;
+    a.batch = n; a.Lq = m->P; a.Lkv = m->P; a.kv_batch_rows = m->P;
+    a.heads = c.heads; a.head_dim = c.head_dim;
+    CKS(run_attn(m, a, FB_K_ATTN_SELF));
+  }
+  {
+    GemmArgs g = gemm_args(M, D, D, m->ao, w.wo, w.bo, EPI_RESID, hB);
+    g.epi.resid = h;
+    g.epi.gate = g1;
+    CKS(run_gemm(m, g));
+  }
+  // cross-attention branch
+  CKS(run_ln(m, hB, m->act, M, 0.f, w.n3w, w.n3b));
+  CKS(run_gemm(m, gemm_args(M, D, D, m->act, w.cq, w.cbq, EPI_BF16, m->cqb)));
+  CKS(run_qkn(m, m->cqb, M, D, 1, 0, w.cnq, 0, w.cnq, nullptr));
+  {
+    const bf16* kv = m->kvctx + (size_t)l * c.text_len * 2 * D;
+    AttnArgs a{};
+    a.Q = m->cqb; a.K = kv; a.V = kv + D; a.O = m->ao;
+    a.ldq = D; a.ldk = a.ldv = 2 * D; a.ldo = D;
+    a.batch = n; a.Lq = m->P; a.Lkv = c.text_len; a.kv_batch_rows = 0;
+    a.heads = c.heads; a.head_dim = c.head_dim;
+    CKS(run_attn(m, a, FB_K_ATTN_CROSS));
+  }
+  {
+    GemmArgs g = gemm_args(M, D, D, m->ao, w.co, w.cbo, EPI_RESID, hB);
+    g.epi.resid = hB;
+    CKS(run_gemm(m, g));
+  }
+  // feed-forward branch; the last epilogue writes h and, if asked, Delta = h_new - h_old
+  CKS(run_ln(m, hB, m->act, M, 1.f, c2, s2));
+  CKS(run_gemm(m, gemm_args(M, c.ffn, D, m->act, w.w1, w.b1, EPI_GELU_BF16, m->ffh)));
+  {
+    GemmArgs g = gemm_args(M, D, c.ffn, m->ffh, w.w2, w.b2, delta ? EPI_RESID_DELTA : EPI_RESID, h);
+    g.epi.resid = hB;
+    g.epi.gate = g2;
+    g.epi.base = h;
+    g.epi.delta = delta;
+    CKS(run_gemm(m, g));
+  }
+  return FB_OK;
+}
+
+// ---- plan analysis ------------------------------------------------------------------
+struct Action {
+  int type;   // 0 compute, 1 proxy run
+  int layer;  // compute: layer
+  int slot;   // compute: anchor slot for Delta, -1 = none
+  std::vector<std::pair<int, double>> terms;  // proxy: (slot, coefficient)
+};
+struct Plan {
+  std::vector<std::vector<Action>> steps;
+  int n_slots = 0;
+};
+
+fb_status analyse_plan(const fb_cfg& c, const float* sched, int S, const uint8_t* skip,
+                       const int32_t* proxy, Plan* out) {
+  const int L = c.depth;
+  auto is_skip = [&](int k, int l) { return skip && skip[(size_t)k * L + l] != 0; };
+  auto code = [&](int k, int l) { return proxy ? proxy[(size_t)k * L + l] : -1; };
+  // computed steps per layer; anchors per proxy; last use per (step, layer)
+  std::vector<std::vector<int>> computed(L);
+  std::map<std::pair<int, int>, std::vector<int>> anchors;
+  std::map<std::pair<int, int>, int> last_use;  // (step, layer) -> last proxy step using it
+  for (int k = 0; k < S; ++k)
+    for (int l = 0; l < L; ++l) {
+      const int32_t cd = code(k, l);
+      if (cd == -1) {
+        if (!is_skip(k, l)) computed[l].push_back(k);
+        continue;
+      }
+      if (is_skip(k, l)) return fail(FB_EPLAN, "step %d layer %d: skipped and proxied", k, l);
+      if (cd < 0) return fail(FB_EPLAN, "step %d layer %d: bad proxy code %d", k, l, cd);
+      const int src = cd & 0xFFFF, order = cd >> 16;
+      if (order > 2) return fail(FB_EPLAN, "step %d layer %d: order %d > 2", k, l, order);
+      if (src >= k) return fail(FB_EPLAN, "step %d layer %d: source step %d not earlier", k, l, src);
+      const auto& cl = computed[l];
+      if (std::find(cl.begin(), cl.end(), src) == cl.end())
+        return fail(FB_EPLAN, "step %d layer %d: not computed at source step %d", k, l, src);
+      std::vector<int> an;
+      for (auto it = cl.rbegin(); it != cl.rend() && (int)an.size() < order + 1; ++it)
+        if (*it <= src) an.push_back(*it);
+      for (int s : an) last_use[{s, l}] = k;
+      anchors[{k, l}] = an;
+    }
+  // slot assignment: per layer a pool; a slot is free once its last user has run
+  std::vector<std::vector<int>> free_at(L);  // per layer: for each slot, step after which it is free
+  std::vector<int> slot_base(L, 0);
+  std::map<std::pair<int, int>, int> slot_of;  // (step, layer) -> local slot
+  for (int k = 0; k < S; ++k)
+    for (int l = 0; l < L; ++l) {
+      auto lu = last_use.find({k, l});
+      if (lu == last_use.end()) continue;
+      auto& pool = free_at[l];
+      int s = -1;
+      for (size_t i = 0; i < pool.size(); ++i)
+        if (pool[i] < k) { s = (int)i; break; }
+      if (s < 0) { s = (int)pool.size(); pool.push_back(0); }
+      pool[s] = lu->second;
+      slot_of[{k, l}] = s;
+    }
+  int total = 0;
+  for (int l = 0; l < L; ++l) { slot_base[l] = total; total += (int)free_at[l].size(); }
+  out->n_slots = total;
+  out->steps.assign(S, {});
+  for (int k = 0; k < S; ++k) {
+    auto& acts = out->steps[k];
+    for (int l = 0; l < L; ++l) {
+      if (is_skip(k, l)) continue;  // Eq. 6: identity, no launch
+      const int32_t cd = code(k, l);
+      if (cd == -1) {
+        Action a{0, l, -1, {}};
+        auto so = slot_of.find({k, l});
+        if (so != slot_of.end()) a.slot = slot_base[l] + so->second;
+        acts.push_back(a);
+        continue;
+      }
+      // Eqs. 3-5 as weights of the anchors h1, h2, h3 (most recent first):
+      // h~ = h1 + a (h1 - h2) + a^2/2 (h1 - 2 h2 + h3), a = (t - tau1) / (tau1 - tau2)
+      const auto& an = anchors[{k, l}];
+      const double t = sched[k];
+      std::vector<double> w;
+      if (an.size() == 1) {
+        w = {1.0};
+      } else {
+        const double tau1 = sched[an[0]], tau2 = sched[an[1]];
+        const double a = (t - tau1) / (tau1 - tau2);
+        if (an.size() == 2) w = {1.0 + a, -a};
+        else w = {1.0 + a + 0.5 * a * a, -a - a * a, 0.5 * a * a};
+      }
+      if (acts.empty() || acts.back().type != 1) acts.push_back(Action{1, -1, -1, {}});
+      for (size_t i = 0; i < an.size(); ++i)
+        acts.back().terms.push_back({slot_base[l] + slot_of[{an[i], l}], w[i]});
+    }
+  }
+  return FB_OK;
+}
+
+fb_status check_schedule(const float* s, int n_steps) {
+  if (!s) return fail(FB_EINVAL, "schedule is NULL");
+  for (int i = 0; i <= n_steps; ++i)
+    if (!(s[i] >= 0.f && s[i] <= 1.f)) return fail(FB_EINVAL, "schedule[%d] outside [0, 1]", i);
+  for (int i = 0; i < n_steps; ++i)
+    if (!(s[i + 1] < s[i])) return fail(FB_EINVAL, "schedule not strictly decreasing at %d", i);
+  return FB_OK;
+}
+
+bool is_device_ptr(const void* p) {
+  cudaPointerAttributes at{};
+  if (cudaPointerGetAttributes(&at, p) != cudaSuccess) {
+    cudaGetLastError();
+    return false;
+  }
+  return at.type == cudaMemoryTypeDevice || at.type == cudaMemoryTypeManaged;
+}
+
+// The sampler loop shared by fb_draft and fb_refine (latents z on the device).
+fb_status sample(fb_model* m, float* z, int n, const float* sched, int S, const Plan& plan) {
+  const fb_cfg& c = m->c;
+  const size_t slot_elems = (size_t)n * m->P * c.dim;
+  const size_t need = slot_elems * plan.n_slots;
+  if (need > m->anchor_elems) {
+    CK(cudaStreamSynchronize(m->st));
+    if (m->anchors) {
+      cudaFree(m->anchors);
+      m->allocs.erase(std::find(m->allocs.begin(), m->allocs.end(), (void*)m->anchors));
+      m->anchors = nullptr;
+      m->anchor_elems = 0;
+    }
+    CKS(dalloc_t(m, &m->anchors, need));
+    m->anchor_elems = need;
+  }
+  const int M = n * m->P;
+  for (int k = 0; k < S; ++k) {
+    const float t = sched[k], t1 = sched[k + 1];
+    CKS(time_embed(m, t));
+    {
+      KTimer kt(m, FB_K_EMBED, 2.0 * M * (double)c.dim * m->PD,
+                4.0 * M * (double)(c.dim + m->PD));
+      CK(patch_embed(z, n, c.latent_c, c.latent_h, c.latent_w, c.patch, m->patch_w, m->patch_b,
+                     c.dim, m->hA, m->st));
+    }
+    for (const Action& a : plan.steps[k]) {
+      if (a.type == 0) {
+        bf16* d = a.slot >= 0 ? m->anchors + (size_t)a.slot * slot_elems : nullptr;
+        CKS(block_forward(m, a.layer, m->hA, n, d));
+      } else {
+        for (size_t i0 = 0; i0 < a.terms.size(); i0 += FB_PROXY_MAX_TERMS) {
+          ProxyTerms pt{};
+          pt.n = (int)std::min(a.terms.size() - i0, (size_t)FB_PROXY_MAX_TERMS);
+          for (int i = 0; i < pt.n; ++i) {
+            pt.ptr[i] = m->anchors + (size_t)a.terms[i0 + i].first * slot_elems;
+            pt.coef[i] = (float)a.terms[i0 + i].second;
+          }
+          KTimer kt(m, FB_K_PROXY, 2.0 * pt.n * (double)M * c.dim,
+                    (double)M * c.dim * (8.0 + 2.0 * pt.n));
+          CK(proxy_add(m->hA, (size_t)M * c.dim, pt, m->st));
+        }
+      }
+    }
+    CKS(run_ln(m, m->hA, m->act, M, 1.f, m->hmod + c.dim, m->hmod));
+    {
+      KTimer kt(m, FB_K_HEAD, 2.0 * M * (double)c.dim * m->PD,
+                2.0 * M * (double)c.dim + 8.0 * M * m->PD);
+      CK(head_euler(m->act, n, c.latent_c, c.latent_h, c.latent_w, c.patch, m->head_w, m->head_b,
+                    c.dim, t1 - t, z, m->st));
+    }
+  }
+  return FB_OK;
+}
+
+fb_status run_sampler(fb_model* m, float* latents, int n, const float* text_ctx,
+                      const float* sched, int S, const Plan& plan) {
+  const fb_cfg& c = m->c;
+  const size_t zn = (size_t)n * c.latent_c * c.latent_h * c.latent_w;
+  CKS(begin_call(m));
+  CKS(encode_text(m, text_ctx));
+  const bool dev = is_device_ptr(latents);
+  float* z = dev ? latents : m->zbuf;
+  if (!dev) CK(cudaMemcpyAsync(z, latents, zn * sizeof(float), cudaMemcpyHostToDevice, m->st));
+  CKS(sample(m, z, n, sched, S, plan));
+  if (!dev) CK(cudaMemcpyAsync(latents, z, zn * sizeof(float), cudaMemcpyDeviceToHost, m->st));
+  return end_call(m);
+}
+
+}  // namespace
+
+// =====================================================================================
+// C-ABI
+// =====================================================================================
+extern "C" {
+
+const char* fb_last_error(void) { return g_last_error.c_str(); }
+
+fb_status fb_weights_count(const fb_cfg* cfg, int* count, size_t* total) {
+  CKS(check_cfg(cfg));
+  if (!count || !total) return fail(FB_EINVAL, "null output pointer");
+  auto t = weight_table(*cfg);
+  *count = (int)t.size();
+  size_t s = 0;
+  for (auto& e : t) s += e.numel;
+  *total = s;
+  return FB_OK;
+}
+
+fb_status fb_weights_entry(const fb_cfg* cfg, int idx, const char** name, size_t* offset,
+                           size_t* numel) {
+  CKS(check_cfg(cfg));
+  static thread_local std::vector<WEntry> cache;
+  cache = weight_table(*cfg);
+  if (idx < 0 || idx >= (int)cache.size()) return fail(FB_EINVAL, "entry %d out of range", idx);
+  size_t off = 0;
+  for (int i = 0; i < idx; ++i) off += cache[i].numel;
+  if (name) *name = cache[idx].name.c_str();
+  if (offset) *offset = off;
+  if (numel) *numel = cache[idx].numel;
+  return FB_OK;
+}
+
+void fb_free(fb_model* m) {
+  if (!m) return;
+  if (m->st) cudaStreamSynchronize(m->st);
+  for (auto& p : m->pending) { cudaEventDestroy(p.a); cudaEventDestroy(p.b); }
+  for (auto e : m->ev_pool) cudaEventDestroy(e);
+  for (void* p : m->allocs) cudaFree(p);
+  if (m->herr) cudaFreeHost(m->herr);
+  if (m->own) cudaStreamDestroy(m->own);
+  delete m;
+}
+
+fb_status fb_init_model(const fb_cfg* cfg, const float* weights_host, fb_model** out) {
+  if (!out) return fail(FB_EINVAL, "out is NULL");
+  *out = nullptr;
+  CKS(check_cfg(cfg));
+  if (!weights_host) return fail(FB_EINVAL, "weights_host is NULL");
+  fb_model* m = new fb_model();
+  m->c = *cfg;
+  const fb_cfg& c = m->c;
+  m->gh = c.latent_h / c.patch;
+  m->gw = c.latent_w / c.patch;
+  m->P = m->gh * m->gw;
+  m->PD = c.latent_c * c.patch * c.patch;
+  m->Mmax = (size_t)c.max_n * m->P;
+  memset(m->stats, 0, sizeof m->stats);
+  auto bail = [&](fb_status s) { fb_free(m); return s; };
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&m->num_sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) {
+    cudaGetLastError();
+    return bail(fail(FB_ECUDA, "no CUDA device"));
+  }
+  if (cudaStreamCreateWithFlags(&m->own, cudaStreamNonBlocking) != cudaSuccess)
+    return bail(fail(FB_ECUDA, "cudaStreamCreate failed"));
+  m->st = m->own;
+  if (cudaMallocHost(&m->herr, sizeof(int)) != cudaSuccess)
+    return bail(fail(FB_ENOMEM, "cudaMallocHost failed"));
+
+  // weights: matrices bf16, vectors fp32 (all per-layer tables first, contiguous)
+  auto table = weight_table(c);
+  size_t nmat = 0, nvec = (size_t)c.depth * 6 * c.dim;
+  for (auto& e : table)
+    if (e.kind == W_MAT) nmat += e.numel;
+    else if (e.name.find(".table") == std::string::npos || e.name == "head.table") nvec += e.numel;
+  fb_status s;
+  if ((s = dalloc(m, &m->wmat, nmat * 2)) != FB_OK) return bail(s);
+  if ((s = dalloc(m, &m->wvec, nvec * 4)) != FB_OK) return bail(s);
+  float* stage = nullptr;
+  size_t max_mat = 0;
+  for (auto& e : table) if (e.kind == W_MAT) max_mat = std::max(max_mat, e.numel);
+  if ((s = dalloc_t(m, &stage, max_mat)) != FB_OK) return bail(s);
+  m->tables = reinterpret_cast<float*>(m->wvec);
+  std::map<std::string, void*> ptr;
+  size_t off = 0, mo = 0, vo = (size_t)c.depth * 6 * c.dim;
+  for (auto& e : table) {
+    const float* src = weights_host + off;
+    off += e.numel;
+    void* dst;
+    if (e.kind == W_MAT) {
+      dst = reinterpret_cast<bf16*>(m->wmat) + mo;
+      mo += e.numel;
+      if (cudaMemcpyAsync(stage, src, e.numel * 4, cudaMemcpyHostToDevice, m->st) != cudaSuccess ||
+          f32_to_bf16(stage, reinterpret_cast<bf16*>(dst), e.numel, m->st) != cudaSuccess ||
+          cudaStreamSynchronize(m->st) != cudaSuccess)
+        return bail(fail(FB_ECUDA, "weight upload failed (%s)", e.name.c_str()));
+    } else {
+      if (e.name.size() > 6 && e.name.compare(0, 7, "blocks.") == 0 &&
+          e.name.find(".table") != std::string::npos) {
+        const int l = atoi(e.name.c_str() + 7);
+        dst = m->tables + (size_t)l * 6 * c.dim;
+      } else {
+        dst = reinterpret_cast<float*>(m->wvec) + vo;
+        vo += e.numel;
+      }
+      if (cudaMemcpyAsync(dst, src, e.numel * 4, cudaMemcpyHostToDevice, m->st) != cudaSuccess)
+        return bail(fail(FB_ECUDA, "weight upload failed (%s)", e.name.c_str()));
+    }
+    ptr[e.name] = dst;
+  }
+  if (cudaStreamSynchronize(m->st) != cudaSuccess) return bail(fail(FB_ECUDA, "weight upload"));
+  cudaFree(stage);
+  m->allocs.erase(std::find(m->allocs.begin(), m->allocs.end(), (void*)stage));
+  auto B = [&](const std::string& n) { return reinterpret_cast<bf16*>(ptr[n]); };
+  auto Fp = [&](const std::string& n) { return reinterpret_cast<float*>(ptr[n]); };
+  m->patch_w = B("patch.w"); m->patch_b = Fp("patch.b");
+  m->time_w1 = B("time.w1"); m->time_b1 = Fp("time.b1");
+  m->time_w2 = B("time.w2"); m->time_b2 = Fp("time.b2");
+  m->mod_w = B("mod.w"); m->mod_b = Fp("mod.b");
+  m->text_w1 = B("text.w1"); m->text_b1 = Fp("text.b1");
+  m->text_w2 = B("text.w2"); m->text_b2 = Fp("text.b2");
+  m->head_table = Fp("head.table"); m->head_w = B("head.w"); m->head_b = Fp("head.b");
+  m->L.resize(c.depth);
+  for (int l = 0; l < c.depth; ++l) {
+    const std::string p = "blocks." + std::to_string(l) + ".";
+    Layer& w = m->L[l];
+    w.table = Fp(p + "table");
+    w.wqkv = B(p + "attn.wqkv"); w.bqkv = Fp(p + "attn.bqkv");
+    w.nq = Fp(p + "attn.norm_q"); w.nk = Fp(p + "attn.norm_k");
+    w.wo = B(p + "attn.wo"); w.bo = Fp(p + "attn.bo");
+    w.n3w = Fp(p + "norm3.w"); w.n3b = Fp(p + "norm3.b");
+    w.cq = B(p + "cross.wq"); w.cbq = Fp(p + "cross.bq");
+    w.ckv = B(p + "cross.wkv"); w.cbkv = Fp(p + "cross.bkv");
+    w.cnq = Fp(p + "cross.norm_q"); w.cnk = Fp(p + "cross.norm_k");
+    w.co = B(p + "cross.wo"); w.cbo = Fp(p + "cross.bo");
+    w.w1 = B(p + "ffn.w1"); w.b1 = Fp(p + "ffn.b1");
+    w.w2 = B(p + "ffn.w2"); w.b2 = Fp(p + "ffn.b2");
+  }
+
+  // activation buffers
+  const size_t M = m->Mmax, D = c.dim;
+  const size_t zn = (size_t)c.max_n * c.latent_c * c.latent_h * c.latent_w;
+  if ((s = dalloc_t(m, &m->hA, M * D)) || (s = dalloc_t(m, &m->hB, M * D)) ||
+      (s = dalloc_t(m, &m->act, M * D)) || (s = dalloc_t(m, &m->qkv, M * 3 * D)) ||
+      (s = dalloc_t(m, &m->ao, M * D)) || (s = dalloc_t(m, &m->cqb, M * D)) ||
+      (s = dalloc_t(m, &m->ffh, M * c.ffn)) ||
+      (s = dalloc_t(m, &m->ctx_f, (size_t)c.text_len * c.text_dim)) ||
+      (s = dalloc_t(m, &m->ctx_b, (size_t)c.text_len * c.text_dim)) ||
+      (s = dalloc_t(m, &m->ctx_h, (size_t)c.text_len * D)) ||
+      (s = dalloc_t(m, &m->ctx_p, (size_t)c.text_len * D)) ||
+      (s = dalloc_t(m, &m->kvctx, (size_t)c.depth * c.text_len * 2 * D)) ||
+      (s = dalloc_t(m, &m->emb, (size_t)c.freq_dim)) || (s = dalloc_t(m, &m->th1, D)) ||
+      (s = dalloc_t(m, &m->temb, D)) || (s = dalloc_t(m, &m->mod, 6 * D)) ||
+      (s = dalloc_t(m, &m->modl, (size_t)c.depth * 6 * D)) || (s = dalloc_t(m, &m->hmod, 2 * D)) ||
+      (s = dalloc_t(m, &m->rope, (size_t)m->P * c.head_dim / 2)) ||
+      (s = dalloc_t(m, &m->zbuf, zn)) || (s = dalloc_t(m, &m->derr, 1)))
+    return bail(s);
+  // RoPE table: pair j of a head rotates by the token's row (j < head_dim/4) or column,
+  // with frequency theta^(-2 j' / (head_dim/2)), j' = j mod head_dim/4.
+  {
+    const int half = c.head_dim / 2, npair = half / 2;
+    std::vector<float2> tab((size_t)m->P * half);
+    for (int tok = 0; tok < m->P; ++tok) {
+      const int r = tok / m->gw, col = tok % m->gw;
+      for (int j = 0; j < half; ++j) {
+        const int jj = j % npair;
+        const double pos = j < npair ? r : col;
+        const double ang = pos * std::pow((double)c.rope_theta, -2.0 * jj / half);
+        tab[(size_t)tok * half + j] = make_float2((float)std::cos(ang), (float)std::sin(ang));
+      }
+    }
+    if (cudaMemcpy(m->rope, tab.data(), tab.size() * sizeof(float2), cudaMemcpyHostToDevice) !=
+        cudaSuccess)
+      return bail(fail(FB_ECUDA, "rope table upload failed"));
+  }
+  if (cudaMemset(m->derr, 0, sizeof(int)) != cudaSuccess)
+    return bail(fail(FB_ECUDA, "cudaMemset failed"));
+  *out = m;
+  return FB_OK;
+}
+
+fb_status fb_set_stream(fb_model* m, void* stream) {
+  if (!m) return fail(FB_EINVAL, "model is NULL");
+  CK(cudaStreamSynchronize(m->st));
+  m->st = stream ? reinterpret_cast<cudaStream_t>(stream) : m->own;
+  return FB_OK;
+}
+
+fb_status fb_encode_text(fb_model* m, const float* text_ctx) {
+  if (!m || !text_ctx) return fail(FB_EINVAL, "null argument");
+  CKS(begin_call(m));
+  CKS(encode_text(m, text_ctx));
+  return end_call(m);
+}
+
+fb_status fb_draft(fb_model* m, float* latents, int n, const float* text_ctx,
+                   const float* schedule, int n_steps, const uint8_t* skip_mask,
+                   const int32_t* proxy_plan) {
+  if (!m) return fail(FB_EINVAL, "model is NULL");
+  if (n < 0 || n > m->c.max_n) return fail(FB_EINVAL, "n=%d outside [0, max_n=%d]", n, m->c.max_n);
+  if (n_steps < 0) return fail(FB_EINVAL, "n_steps < 0");
+  if (n == 0 || n_steps == 0) return FB_OK;
+  if (!latents || !text_ctx) return fail(FB_EINVAL, "null latents or text_ctx");
+  CKS(check_schedule(schedule, n_steps));
+  Plan plan;
+  CKS(analyse_plan(m->c, schedule, n_steps, skip_mask, proxy_plan, &plan));
+  return run_sampler(m, latents, n, text_ctx, schedule, n_steps, plan);
+}
+
+fb_status fb_refine(fb_model* m, float* latent, const float* text_ctx,
+                    const float* full_schedule, int n_steps) {
+  if (!m) return fail(FB_EINVAL, "model is NULL");
+  if (n_steps < 0) return fail(FB_EINVAL, "n_steps < 0");
+  if (n_steps == 0) return FB_OK;
+  if (!latent || !text_ctx) return fail(FB_EINVAL, "null latent or text_ctx");
+  CKS(check_schedule(full_schedule, n_steps));
+  Plan plan;
+  CKS(analyse_plan(m->c, full_schedule, n_steps, nullptr, nullptr, &plan));
+  return run_sampler(m, latent, 1, text_ctx, full_schedule, n_steps, plan);
+}
+
+fb_status fb_plan_from_phi(int S, int S_prime, int n_skip, int l_start, int l_end, int f_full,
+                           int order, int depth, uint8_t* skip_mask, int32_t* proxy_plan) {
+  if (!skip_mask || !proxy_plan) return fail(FB_EINVAL, "null output arrays");
+  if (depth < 1 || S_prime < 1 || S_prime > S || f_full < 1 || n_skip < 0 || l_start < 1 ||
+      l_start > l_end || l_end > depth || order < 0 || order > 2 || S_prime > 0xFFFF)
+    return fail(FB_EINVAL, "invalid phi");
+  for (int k = 0; k < S_prime; ++k) {
+    const bool full = (k % f_full) == 0;
+    const int last_full = k - k % f_full;
+    for (int l = 0; l < depth; ++l) {
+      const bool sk = k >= n_skip && l >= l_start - 1 && l <= l_end - 1;
+      skip_mask[(size_t)k * depth + l] = sk ? 1 : 0;
+      proxy_plan[(size_t)k * depth + l] = (sk || full) ? -1 : (last_full | (order << 16));
+    }
+  }
+  return FB_OK;
+}
+
+fb_status fb_block_forward(fb_model* m, int layer, float* h, int n, float t) {
+  if (!m || !h) return fail(FB_EINVAL, "null argument");
+  if (layer < 0 || layer >= m->c.depth) return fail(FB_EINVAL, "layer %d out of range", layer);
+  if (n < 0 || n > m->c.max_n) return fail(FB_EINVAL, "n=%d outside [0, max_n]", n);
+  if (!m->text_ready) return fail(FB_ESTATE, "fb_encode_text has not been called");
+  if (n == 0) return FB_OK;
+  if (!is_device_ptr(h)) return fail(FB_EINVAL, "h must be device memory");
+  CKS(begin_call(m));
+  CKS(time_embed(m, t));
+  CKS(block_forward(m, layer, h, n, nullptr));
+  return end_call(m);
+}
+
+fb_status fb_set_timing(fb_model* m, int mask) {
+  if (!m) return fail(FB_EINVAL, "model is NULL");
+  m->timing_mask = (unsigned)mask;
+  return FB_OK;
+}
+
+fb_status fb_get_stats(fb_model* m, fb_kstat* out) {
+  if (!m || !out) return fail(FB_EINVAL, "null argument");
+  CK(cudaStreamSynchronize(m->st));
+  collect_timings(m);
+  memcpy(out, m->stats, sizeof m->stats);
+  return FB_OK;
+}
+
+fb_status fb_reset_stats(fb_model* m) {
+  if (!m) return fail(FB_EINVAL, "model is NULL");
+  CK(cudaStreamSynchronize(m->st));
+  collect_timings(m);
+  memset(m->stats, 0, sizeof m->stats);
+  return FB_OK;
+}
+
+const char* fb_kernel_name(int kind) {
+  static const char* names[FB_K_COUNT] = {"gemm_tc", "gemm_simt", "attn_self", "attn_cross",
+                                          "ln_mod", "qk_norm_rope", "proxy_add", "patch_embed",
+                                          "head_euler", "small"};
+  return (kind >= 0 && kind < FB_K_COUNT) ? names[kind] : "?";
+}
+
+fb_status fb_op_gemm(fb_model* m, int M, int N, int K, const void* A, const void* W,
+                     const float* bias, int epi, void* out, const float* resid,
+                     const float* gate, const float* base, void* delta, int impl) {
+  if (!m || !A || !W || !out) return fail(FB_EINVAL, "null argument");
+  if (M < 1 || N < 1 || K < 1 || epi < 0 || epi > 3) return fail(FB_EINVAL, "bad sizes / epi");
+  if (epi >= EPI_RESID && !resid) return fail(FB_EINVAL, "resid required");
+  if (epi == EPI_RESID_DELTA && (!base || !delta)) return fail(FB_EINVAL, "base/delta required");
+  if (N % 8) return fail(FB_EINVAL, "N must be a multiple of 8");
+  GemmArgs g = gemm_args(M, N, K, (const bf16*)A, (const bf16*)W, bias, epi, out);
+  g.epi.resid = resid;
+  g.epi.gate = gate;
+  g.epi.base = base;
+  g.epi.delta = (bf16*)delta;
+  CKS(begin_call(m));
+  CKS(run_gemm(m, g, impl == 1));
+  return end_call(m);
+}
+
+fb_status fb_op_attention(fb_model* m, const void* Q, int ldq, const void* K, int ldk,
+                          const void* V, int ldv, void* O, int ldo, int batch, int Lq, int Lkv,
+                          int kv_batch_rows, int heads, int head_dim) {
+  if (!m || !Q || !K || !V || !O) return fail(FB_EINVAL, "null argument");
+  if (batch < 1 || Lq < 1 || Lkv < 1 || heads < 1 || (head_dim != 64 && head_dim != 128))
+    return fail(FB_EINVAL, "bad sizes");
+  AttnArgs a{};
+  a.Q = (const bf16*)Q; a.K = (const bf16*)K; a.V = (const bf16*)V; a.O = (bf16*)O;
+  a.ldq = ldq; a.ldk = ldk; a.ldv = ldv; a.ldo = ldo;
+  a.batch = batch; a.Lq = Lq; a.Lkv = Lkv; a.kv_batch_rows = kv_batch_rows;
+  a.heads = heads; a.head_dim = head_dim;
+  CKS(begin_call(m));
+  CKS(run_attn(m, a, FB_K_ATTN_SELF));
+  return end_call(m);
+}
+
+}  // extern "C"

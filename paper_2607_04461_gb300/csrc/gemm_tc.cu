@@ -1,0 +1,273 @@
+// tcgen05 / TMEM GEMM for sm_103a: out[M][N] = epilogue(A[M][K] * W[N][K]^T).
+//
+// The dense projections of the DiT block (Eq. 7's B_l: QKV, attention output, cross
+// query, cross output, FFN up and down) and the text projection run here.
+//
+// Design (one CTA per SM, persistent over output tiles of 128 x BN):
+//  * warp 0, one thread: TMA producer. Loads 128x64 tiles of A and BNx64 tiles of W
+//    (bf16, 128-byte swizzle) into a ring of STAGES shared-memory stages; each stage
+//    has a "full" mbarrier (TMA transaction bytes) and an "empty" one (MMA done).
+//  * warp 1: allocates 2*BN TMEM columns (two fp32 accumulators of 128 lanes x BN);
+//    one thread issues tcgen05.mma (M=128, N=BN, K=16, bf16 -> fp32), commits each
+//    stage back to its "empty" barrier and each finished tile to "tmem_full".
+//  * warps 2-5: epilogue. Warp w reads TMEM lanes 32*(w%4).. (its lane quarter) with
+//    tcgen05.ld, applies bias / GELU / gated residual / contribution write, stores to
+//    global, and releases the accumulator ("tmem_empty") so that the MMA of the tile
+//    after next can start while this epilogue runs.
+// Every mbarrier wait is bounded (mbar_wait): on timeout the kernel records the error,
+// stops issuing work, waits (bounded) for its own TMA loads, frees TMEM and returns.
+#include <cudaTypedefs.h>
+
+#include "kernels.h"
+
+namespace {
+
+constexpr int BM = 128;
+constexpr int BK = 64;  // 64 bf16 = 128 bytes: one swizzle row
+constexpr int NUM_THREADS = 192;
+
+template <int BN>
+struct TcCfg {
+  static constexpr int STAGES = (BN == 256) ? 4 : 6;
+  static constexpr int A_BYTES = BM * BK * 2;
+  static constexpr int B_BYTES = BN * BK * 2;
+  static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
+  static constexpr int TMEM_COLS = 2 * BN;  // 256 or 512 (power of two >= 32)
+  static constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + 1024 /*align*/ + 256 /*barriers*/;
+};
+
+// Shared-memory matrix descriptor: K-major, 128-byte swizzle; 8-row core-matrix groups
+// are 1024 bytes apart (stride byte offset); leading byte offset unused for this layout.
+__device__ __forceinline__ uint64_t sdesc_sw128(uint32_t saddr) {
+  uint64_t d = 0;
+  d |= (uint64_t)((saddr & 0x3FFFFu) >> 4);
+  d |= (uint64_t)1 << 16;                 // leading byte offset (16 B, ignored)
+  d |= (uint64_t)(1024 >> 4) << 32;       // stride byte offset
+  d |= (uint64_t)1 << 46;                 // descriptor version (tcgen05)
+  d |= (uint64_t)2 << 61;                 // layout: 128-byte swizzle
+  return d;
+}
+
+// Instruction descriptor, kind::f16: D fp32, A and B bf16, both K-major, M=128, N=BN.
+template <int BN>
+__device__ __forceinline__ uint32_t idesc_bf16() {
+  return (1u << 4)                     // D format: f32
+         | (1u << 7)                   // A format: bf16
+         | (1u << 10)                  // B format: bf16
+         | ((uint32_t)(BN >> 3) << 17) // N >> 3
+         | ((uint32_t)(BM >> 4) << 24);// M >> 4
+}
+
+template <int BN, int KIND>
+__global__ void __launch_bounds__(NUM_THREADS, 1)
+    gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmW,
+                   int M, int N, int K, GemmEpi epi, int* err) {
+  using C = TcCfg<BN>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + C::STAGES * C::STAGE_BYTES);
+  uint64_t* empty = full + C::STAGES;
+  uint64_t* tmem_full = empty + C::STAGES;
+  uint64_t* tmem_empty = tmem_full + 2;
+  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(tmem_empty + 2);
+
+  const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+  const int n_mt = (M + BM - 1) / BM, n_nt = N / BN, n_tiles = n_mt * n_nt;
+  const int nk = K / BK;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < C::STAGES; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(&tmem_full[a], 1);
+      mbar_init(&tmem_empty[a], 128);
+    }
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    tma_prefetch_desc(&tmA);
+    tma_prefetch_desc(&tmW);
+  }
+  if (warp == 1) tmem_alloc(tmem_holder, C::TMEM_COLS);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_holder;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ---------------- TMA producer ----------------
+      int stage = 0;
+      uint32_t phase = 0;
+      uint32_t issued[C::STAGES];
+#pragma unroll
+      for (int s = 0; s < C::STAGES; ++s) issued[s] = 0;
+      bool ok = true;
+      for (int tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x) {
+        const int m0 = (tile / n_nt) * BM, n0 = (tile % n_nt) * BN;
+        for (int kb = 0; kb < nk; ++kb) {
+          if (!mbar_wait(&empty[stage], phase ^ 1u, err)) { ok = false; break; }
+          uint8_t* sa = smem + stage * C::STAGE_BYTES;
+          mbar_expect_tx(&full[stage], C::STAGE_BYTES);
+          tma_load_2d(sa, &tmA, &full[stage], kb * BK, m0);
+          tma_load_2d(sa + C::A_BYTES, &tmW, &full[stage], kb * BK, n0);
+          ++issued[stage];
+          if (++stage == C::STAGES) { stage = 0; phase ^= 1u; }
+        }
+      }
+      if (!ok) {
+        // Let this CTA's loads in flight land before the CTA exits.
+        for (int s = 0; s < C::STAGES; ++s)
+          if (issued[s]) {
+            const uint32_t a = smem_u32(&full[s]);
+            const uint64_t t0 = fb_globaltimer();
+            while (!mbar_try(a, (issued[s] - 1) & 1u) &&
+                   fb_globaltimer() - t0 < FB_WAIT_LIMIT_NS) {
+            }
+          }
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      // ---------------- MMA issuer ----------------
+      const uint32_t idesc = idesc_bf16<BN>();
+      int stage = 0;
+      uint32_t phase = 0;
+      bool ok = true;
+      int it = 0;
+      for (int tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x, ++it) {
+        const int acc = it & 1;
+        const uint32_t acc_phase = (it >> 1) & 1;
+        if (!mbar_wait(&tmem_empty[acc], acc_phase ^ 1u, err)) break;
+        tc_fence_after();
+        const uint32_t d_tmem = tmem_base + acc * BN;
+        for (int kb = 0; kb < nk; ++kb) {
+          if (!mbar_wait(&full[stage], phase, err)) { ok = false; break; }
+          tc_fence_after();
+          const uint32_t sa = smem_u32(smem + stage * C::STAGE_BYTES);
+          const uint64_t adesc = sdesc_sw128(sa), bdesc = sdesc_sw128(sa + C::A_BYTES);
+#pragma unroll
+          for (int k = 0; k < BK / 16; ++k) {
+            // +32 bytes per K=16 step inside the swizzle row (encoded >> 4 -> +2)
+            tc_mma_f16(d_tmem, adesc + 2 * k, bdesc + 2 * k, idesc, (kb | k) ? 1u : 0u);
+          }
+          tc_commit(&empty[stage]);
+          if (++stage == C::STAGES) { stage = 0; phase ^= 1u; }
+        }
+        if (ok) tc_commit(&tmem_full[acc]);
+      }
+    }
+  } else {
+    // ---------------- epilogue (warps 2..5) ----------------
+    const int quarter = warp & 3;
+    int it = 0;
+    for (int tile = blockIdx.x; tile < n_tiles; tile += gridDim.x, ++it) {
+      const int acc = it & 1;
+      const uint32_t acc_phase = (it >> 1) & 1;
+      const int m0 = (tile / n_nt) * BM, n0 = (tile % n_nt) * BN;
+      // every lane waits; the warp leaves together if any lane gave up, so the
+      // .sync.aligned tcgen05.ld below is always executed by the whole warp
+      const bool ok = mbar_wait(&tmem_full[acc], acc_phase, err);
+      if (!__all_sync(0xffffffffu, ok)) break;
+      tc_fence_after();
+      const int row = m0 + quarter * 32 + lane;
+      const uint32_t taddr = tmem_base + ((uint32_t)(quarter * 32) << 16) + acc * BN;
+#pragma unroll 1
+      for (int c = 0; c < BN / 32; ++c) {
+        uint32_t r[32];
+        tmem_ld32(taddr + c * 32, r);
+        tmem_ld_wait();
+        if (row < M) {
+#pragma unroll
+          for (int g = 0; g < 4; ++g) {
+            float v[8];
+#pragma unroll
+            for (int j = 0; j < 8; ++j) v[j] = __uint_as_float(r[g * 8 + j]);
+            epi_apply8<KIND>(epi, row, n0 + c * 32 + g * 8, v);
+          }
+        }
+      }
+      tc_fence_before();
+      mbar_arrive(&tmem_empty[acc]);
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem_base, C::TMEM_COLS);
+  }
+}
+
+PFN_cuTensorMapEncodeTiled_v12000 get_encode() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  if (!fn) {
+    cudaDriverEntryPointQueryResult q;
+    void* p = nullptr;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  }
+  return fn;
+}
+
+// 2-D bf16 tensor map over rows x cols (row stride ld elements), box box_rows x 64.
+bool make_map(CUtensorMap* map, const bf16* ptr, int rows, int cols, int ld, int box_rows) {
+  auto enc = get_encode();
+  if (!enc) return false;
+  cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
+  cuuint64_t strides[1] = {(cuuint64_t)ld * sizeof(bf16)};
+  cuuint32_t box[2] = {(cuuint32_t)BK, (cuuint32_t)box_rows};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<bf16*>(ptr), dims,
+                   strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                   CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
+template <int BN, int KIND>
+cudaError_t launch(const GemmArgs& g, int* err, int num_sms, cudaStream_t st) {
+  using C = TcCfg<BN>;
+  CUtensorMap ma, mw;
+  if (!make_map(&ma, g.A, g.M, g.K, g.lda, BM) || !make_map(&mw, g.W, g.N, g.K, g.ldw, BN))
+    return cudaErrorInvalidValue;
+  cudaError_t e = cudaFuncSetAttribute(gemm_tc_kernel<BN, KIND>,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM_BYTES);
+  if (e != cudaSuccess) return e;
+  const int tiles = ((g.M + BM - 1) / BM) * (g.N / BN);
+  const int grid = tiles < num_sms ? tiles : num_sms;
+  gemm_tc_kernel<BN, KIND><<<grid, NUM_THREADS, C::SMEM_BYTES, st>>>(ma, mw, g.M, g.N, g.K,
+                                                                      g.epi, err);
+  return cudaGetLastError();
+}
+
+template <int BN>
+cudaError_t dispatch_kind(const GemmArgs& g, int* err, int num_sms, cudaStream_t st) {
+  switch (g.kind) {
+    case EPI_BF16: return launch<BN, EPI_BF16>(g, err, num_sms, st);
+    case EPI_GELU_BF16: return launch<BN, EPI_GELU_BF16>(g, err, num_sms, st);
+    case EPI_RESID: return launch<BN, EPI_RESID>(g, err, num_sms, st);
+    case EPI_RESID_DELTA: return launch<BN, EPI_RESID_DELTA>(g, err, num_sms, st);
+  }
+  return cudaErrorInvalidValue;
+}
+
+}  // namespace
+
+bool gemm_tc_supported(const GemmArgs& g) {
+  auto al16 = [](const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15) == 0; };
+  return g.M >= 1 && g.N % 128 == 0 && g.K % BK == 0 && g.K >= BK && g.lda % 8 == 0 &&
+         g.ldw % 8 == 0 && g.epi.ldo % 8 == 0 && al16(g.A) && al16(g.W) && al16(g.epi.out);
+}
+
+cudaError_t gemm_tc(const GemmArgs& g, int* err, int num_sms, cudaStream_t st) {
+  if (!gemm_tc_supported(g)) return cudaErrorInvalidValue;
+  // BN = 256 halves the A re-reads; use it when it still gives every SM a tile.
+  const int mt = (g.M + BM - 1) / BM;
+  if (g.N % 256 == 0 && mt * (g.N / 256) >= num_sms) return dispatch_kind<256>(g, err, num_sms, st);
+  return dispatch_kind<128>(g, err, num_sms, st);
+}

@@ -1,0 +1,70 @@
+// Host-side launchers of the sm_103a kernels (internal to libflashbon.so).
+// Every launcher enqueues on `st` and returns the cudaError_t of the launch.
+#pragma once
+#include <cuda_runtime.h>
+#include <stddef.h>
+#include <stdint.h>
+
+#include "common.cuh"
+
+// ---- GEMM: out[M][N] = epilogue(A[M][K] * W[N][K]^T) --------------------------------
+struct GemmArgs {
+  int M, N, K;
+  const bf16* A;  // row-major, leading dimension lda
+  int lda;
+  const bf16* W;  // row-major [N][K], leading dimension ldw
+  int ldw;
+  int kind;       // EPI_*
+  GemmEpi epi;
+};
+// tcgen05 path: requires N % 128 == 0, K % 64 == 0, 16-byte aligned rows.
+bool gemm_tc_supported(const GemmArgs& g);
+cudaError_t gemm_tc(const GemmArgs& g, int* err, int num_sms, cudaStream_t st);
+// CUDA-core path: requires N % 8 == 0.
+cudaError_t gemm_simt(const GemmArgs& g, cudaStream_t st);
+
+// ---- attention: O = softmax(Q K^T / sqrt(dh)) V ----------------------------------
+struct AttnArgs {
+  const bf16 *Q, *K, *V;
+  bf16* O;
+  int ldq, ldk, ldv, ldo;  // row strides (elements)
+  int batch, Lq, Lkv;
+  int kv_batch_rows;       // row offset of batch b's K/V (0 = shared)
+  int heads, head_dim;
+};
+cudaError_t attention(const AttnArgs& a, cudaStream_t st);
+
+// ---- pointwise / small kernels ------------------------------------------------------
+// out[r][:] = bf16(LN(x[r][:]) * (mul_base + mul[:]) + add[:]), x fp32 [rows][D].
+cudaError_t ln_mod(const float* x, bf16* out, int rows, int D, float eps, float mul_base,
+                   const float* mul, const float* add, cudaStream_t st);
+// In place on bf16 rows: x[r][col0 + :D] = RMSNorm(.) * w, then (if rope != null) RoPE
+// with table rope[(r % tokens)][head_dim/2] of (cos, sin) per adjacent pair.
+// Two segments (col0, w0) and (col1, w1) when nseg == 2.
+cudaError_t qk_norm_rope(bf16* x, int rows, int ld, int D, int nseg, int col0, const float* w0,
+                         int col1, const float* w1, float eps, const float2* rope,
+                         int tokens, int head_dim, cudaStream_t st);
+// h[i] += sum_t coef[t] * anchor_t[i] over n_elems fp32 elements (bf16 anchors).
+#define FB_PROXY_MAX_TERMS 64
+struct ProxyTerms {
+  const bf16* ptr[FB_PROXY_MAX_TERMS];
+  float coef[FB_PROXY_MAX_TERMS];
+  int n;
+};
+cudaError_t proxy_add(float* h, size_t n_elems, const ProxyTerms& t, cudaStream_t st);
+// h[(b*P + tok)][:] = W_p * patch(z_b, tok) + b_p.
+cudaError_t patch_embed(const float* z, int n, int C, int H, int W, int p, const bf16* Wp,
+                        const float* bp, int D, float* h, cudaStream_t st);
+// z[b] += dt * unpatchify(a * Wh^T + bh), a bf16 [n*P][D].
+cudaError_t head_euler(const bf16* a, int n, int C, int H, int W, int p, const bf16* Wh,
+                       const float* bh, int D, float dt, float* z, cudaStream_t st);
+// y[o] = act_out(b[o] + sum_k W[o][k] act_in(x[k])), act: 0 none, 1 SiLU.
+cudaError_t gemv(const bf16* W, const float* b, const float* x, float* y, int O, int K,
+                 int act_in, int act_out, cudaStream_t st);
+// emb = [cos(1000 t f_k), sin(1000 t f_k)], f_k = 10000^(-k/half).
+cudaError_t timestep_sincos(float t, int dim, float* emb, cudaStream_t st);
+// modl[l][j][:] = mod[j][:] + table_l[j][:] (6 rows, all layers); head[j] = htab[j] + temb.
+cudaError_t mod_prepare(const float* mod, const float* tables, int L, int D,
+                        float* modl, const float* htab, const float* temb, float* head_mod,
+                        cudaStream_t st);
+cudaError_t f32_to_bf16(const float* x, bf16* y, size_t n, cudaStream_t st);

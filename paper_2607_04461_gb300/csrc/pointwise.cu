@@ -1,0 +1,411 @@
+// Memory-bound and small kernels of the draft path:
+//  ln_mod       adaLN: LayerNorm (no affine) * (1 + scale) + shift, or affine LN; fp32 in,
+//               bf16 out (feeds the next GEMM). Row held in registers: one HBM read.
+//  qk_norm_rope RMSNorm of q / k over the model width, then 2-D axial RoPE, in place.
+//  proxy_add    activation proxy (Eqs. 3-5 as a linear combination of cached block
+//               contributions): h += sum_t c_t Delta_t, one read and write of h per run.
+//  patch_embed  2x2 patchify + linear (D x C p p), writes the fp32 residual stream.
+//  head_euler   output projection D -> C p p, unpatchify and the Euler step
+//               z += (t' - t) v of dx = v dt, fused.
+//  gemv, timestep_sincos, mod_prepare, f32_to_bf16: per-step conditioning, conversions.
+#include "kernels.h"
+
+namespace {
+
+template <int THREADS>
+__device__ __forceinline__ float block_sum(float v, float* red) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  if (THREADS > 32) {
+    const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+    __syncthreads();
+    if (lane == 0) red[warp] = v;
+    __syncthreads();
+    v = 0.f;
+#pragma unroll
+    for (int w = 0; w < THREADS / 32; ++w) v += red[w];
+  }
+  return v;
+}
+
+// ---------------------------------------------------------------------------------
+// ln_mod: THREADS threads per row, VPT float4 per thread (D = 4 * VPT * THREADS).
+template <int THREADS, int VPT>
+__global__ void __launch_bounds__(THREADS) ln_mod_kernel(const float* __restrict__ x,
+                                                         bf16* __restrict__ out, int D,
+                                                         float eps, float mul_base,
+                                                         const float* __restrict__ mul,
+                                                         const float* __restrict__ add) {
+  __shared__ float red[THREADS / 32 > 0 ? THREADS / 32 : 1];
+  const size_t row = blockIdx.x;
+  const float* xr = x + row * D;
+  float4 v[VPT];
+  float s = 0.f;
+#pragma unroll
+  for (int i = 0; i < VPT; ++i) {
+    v[i] = *reinterpret_cast<const float4*>(xr + (i * THREADS + threadIdx.x) * 4);
+    s += v[i].x + v[i].y + v[i].z + v[i].w;
+  }
+  const float mean = block_sum<THREADS>(s, red) / D;
+  float q = 0.f;
+#pragma unroll
+  for (int i = 0; i < VPT; ++i) {
+    const float a = v[i].x - mean, b = v[i].y - mean, c = v[i].z - mean, d = v[i].w - mean;
+    q += a * a + b * b + c * c + d * d;
+  }
+  const float rstd = rsqrtf(block_sum<THREADS>(q, red) / D + eps);
+#pragma unroll
+  for (int i = 0; i < VPT; ++i) {
+    const int col = (i * THREADS + threadIdx.x) * 4;
+    const float4 m = *reinterpret_cast<const float4*>(mul + col);
+    const float4 ad = *reinterpret_cast<const float4*>(add + col);
+    const float y0 = (v[i].x - mean) * rstd * (mul_base + m.x) + ad.x;
+    const float y1 = (v[i].y - mean) * rstd * (mul_base + m.y) + ad.y;
+    const float y2 = (v[i].z - mean) * rstd * (mul_base + m.z) + ad.z;
+    const float y3 = (v[i].w - mean) * rstd * (mul_base + m.w) + ad.w;
+    uint2 u;
+    u.x = pack_bf16x2(y0, y1);
+    u.y = pack_bf16x2(y2, y3);
+    *reinterpret_cast<uint2*>(out + row * D + col) = u;
+  }
+}
+
+template <int THREADS, int VPT>
+cudaError_t ln_mod_launch(const float* x, bf16* out, int rows, int D, float eps, float mb,
+                          const float* mul, const float* add, cudaStream_t st) {
+  ln_mod_kernel<THREADS, VPT><<<rows, THREADS, 0, st>>>(x, out, D, eps, mb, mul, add);
+  return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------------------------
+// qk_norm_rope: THREADS threads per (row, segment), VPT chunks of 4 bf16 per thread.
+__device__ __forceinline__ void load_bf16x4(const bf16* p, float* v) {
+  uint2 u = *reinterpret_cast<const uint2*>(p);
+  float2 a = unpack_bf16x2(u.x), b = unpack_bf16x2(u.y);
+  v[0] = a.x; v[1] = a.y; v[2] = b.x; v[3] = b.y;
+}
+__device__ __forceinline__ void store_bf16x4(bf16* p, const float* v) {
+  uint2 u;
+  u.x = pack_bf16x2(v[0], v[1]);
+  u.y = pack_bf16x2(v[2], v[3]);
+  *reinterpret_cast<uint2*>(p) = u;
+}
+
+template <int THREADS, int VPT>
+__global__ void __launch_bounds__(THREADS) qk_norm_rope_kernel(
+    bf16* __restrict__ x, int ld, int D, int col0, const float* __restrict__ w0, int col1,
+    const float* __restrict__ w1, float eps, const float2* __restrict__ rope, int tokens,
+    int head_dim) {
+  __shared__ float red[THREADS / 32 > 0 ? THREADS / 32 : 1];
+  const size_t row = blockIdx.x;
+  const int seg = blockIdx.y;
+  const int col0s = seg ? col1 : col0;
+  const float* w = seg ? w1 : w0;
+  bf16* xr = x + row * ld + col0s;
+  float v[VPT][4];
+  float ss = 0.f;
+#pragma unroll
+  for (int i = 0; i < VPT; ++i) {
+    load_bf16x4(xr + (i * THREADS + threadIdx.x) * 4, v[i]);
+#pragma unroll
+    for (int j = 0; j < 4; ++j) ss += v[i][j] * v[i][j];
+  }
+  const float r = rsqrtf(block_sum<THREADS>(ss, red) / D + eps);
+  const float2* rp = rope ? rope + (size_t)(row % tokens) * (head_dim / 2) : nullptr;
+#pragma unroll
+  for (int i = 0; i < VPT; ++i) {
+    const int col = (i * THREADS + threadIdx.x) * 4;
+    const float4 wv = *reinterpret_cast<const float4*>(w + col);
+    v[i][0] *= r * wv.x; v[i][1] *= r * wv.y; v[i][2] *= r * wv.z; v[i][3] *= r * wv.w;
+    if (rp) {
+      const int d0 = col % head_dim;  // a chunk never straddles a head (head_dim % 4 == 0)
+#pragma unroll
+      for (int j = 0; j < 4; j += 2) {
+        const float2 cs = rp[(d0 + j) >> 1];
+        const float a = v[i][j], b = v[i][j + 1];
+        v[i][j] = a * cs.x - b * cs.y;
+        v[i][j + 1] = a * cs.y + b * cs.x;
+      }
+    }
+    store_bf16x4(xr + col, v[i]);
+  }
+}
+
+template <int THREADS, int VPT>
+cudaError_t qkn_launch(bf16* x, int rows, int ld, int D, int nseg, int col0, const float* w0,
+                       int col1, const float* w1, float eps, const float2* rope, int tokens,
+                       int head_dim, cudaStream_t st) {
+  dim3 grid(rows, nseg);
+  qk_norm_rope_kernel<THREADS, VPT><<<grid, THREADS, 0, st>>>(x, ld, D, col0, w0, col1, w1,
+                                                             eps, rope, tokens, head_dim);
+  return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------------------------
+__global__ void __launch_bounds__(256) proxy_add_kernel(float* __restrict__ h, size_t n8,
+                                                        ProxyTerms t) {
+  for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < n8;
+       i += (size_t)gridDim.x * blockDim.x) {
+    float acc[8];
+    load_f32x8(h + i * 8, acc);
+    for (int k = 0; k < t.n; ++k) {
+      float a[8];
+      load_bf16x8(t.ptr[k] + i * 8, a);
+      const float c = t.coef[k];
+#pragma unroll
+      for (int j = 0; j < 8; ++j) acc[j] += c * a[j];
+    }
+    store_f32x8(h + i * 8, acc);
+  }
+}
+
+// ---------------------------------------------------------------------------------
+// patch_embed: 32 tokens per CTA, 256 threads; thread owns output columns n = tid + 256 k.
+constexpr int PE_TOK = 32;
+__global__ void __launch_bounds__(256) patch_embed_kernel(const float* __restrict__ z, int n,
+                                                          int C, int H, int W, int p,
+                                                          const bf16* __restrict__ Wp,
+                                                          const float* __restrict__ bp, int D,
+                                                          float* __restrict__ h) {
+  extern __shared__ float xs[];  // [PE_TOK][PD]
+  const int PD = C * p * p, gw = W / p, P = (H / p) * gw;
+  const int M = n * P;
+  const int tok0 = blockIdx.x * PE_TOK;
+  for (int i = threadIdx.x; i < PE_TOK * PD; i += blockDim.x) {
+    const int t = i / PD, k = i % PD;
+    const int tok = tok0 + t;
+    float val = 0.f;
+    if (tok < M) {
+      const int b = tok / P, pt = tok % P, r = pt / gw, cc = pt % gw;
+      const int ch = k / (p * p), dy = (k / p) % p, dx = k % p;
+      val = z[(((size_t)b * C + ch) * H + r * p + dy) * W + cc * p + dx];
+    }
+    xs[i] = val;
+  }
+  __syncthreads();
+  for (int col = threadIdx.x; col < D; col += blockDim.x) {
+    float acc[PE_TOK];
+    const float bias = bp[col];
+#pragma unroll
+    for (int t = 0; t < PE_TOK; ++t) acc[t] = bias;
+    for (int k0 = 0; k0 < PD; k0 += 8) {
+      float wv[8];
+      load_bf16x8(Wp + (size_t)col * PD + k0, wv);
+#pragma unroll
+      for (int t = 0; t < PE_TOK; ++t)
+#pragma unroll
+        for (int j = 0; j < 8; ++j) acc[t] += wv[j] * xs[t * PD + k0 + j];
+    }
+#pragma unroll
+    for (int t = 0; t < PE_TOK; ++t)
+      if (tok0 + t < M) h[(size_t)(tok0 + t) * D + col] = acc[t];
+  }
+}
+
+// ---------------------------------------------------------------------------------
+// head_euler: 32 tokens per CTA, 256 threads; K staged through shared memory in
+// chunks of 128. Thread -> output o = tid % PD, tokens (tid / PD) * TPT .. + TPT - 1.
+constexpr int HE_TOK = 32, HE_KC = 128;
+__global__ void __launch_bounds__(256) head_euler_kernel(const bf16* __restrict__ a, int n,
+                                                         int C, int H, int W, int p,
+                                                         const bf16* __restrict__ Wh,
+                                                         const float* __restrict__ bh, int D,
+                                                         float dt, float* __restrict__ z) {
+  __shared__ float as[HE_TOK][HE_KC + 1];
+  __shared__ float ws[64][HE_KC + 1];
+  const int PD = C * p * p, gw = W / p, P = (H / p) * gw, M = n * P;
+  const int tok0 = blockIdx.x * HE_TOK;
+  const int o = threadIdx.x % PD, grp = threadIdx.x / PD;
+  const int TPT = HE_TOK * PD / 256;  // tokens per thread (PD in {8,...,64}, PD | 256)
+  float acc[32];
+#pragma unroll
+  for (int i = 0; i < 32; ++i) acc[i] = 0.f;
+  for (int k0 = 0; k0 < D; k0 += HE_KC) {
+    __syncthreads();
+    for (int i = threadIdx.x; i < HE_TOK * HE_KC / 8; i += 256) {
+      const int t = i / (HE_KC / 8), kc = (i % (HE_KC / 8)) * 8;
+      float v[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+      if (tok0 + t < M && k0 + kc < D) load_bf16x8(a + (size_t)(tok0 + t) * D + k0 + kc, v);
+#pragma unroll
+      for (int j = 0; j < 8; ++j) as[t][kc + j] = v[j];
+    }
+    for (int i = threadIdx.x; i < PD * HE_KC / 8; i += 256) {
+      const int r = i / (HE_KC / 8), kc = (i % (HE_KC / 8)) * 8;
+      float v[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+      if (k0 + kc < D) load_bf16x8(Wh + (size_t)r * D + k0 + kc, v);
+#pragma unroll
+      for (int j = 0; j < 8; ++j) ws[r][kc + j] = v[j];
+    }
+    __syncthreads();
+    if (grp * TPT < HE_TOK) {
+      for (int k = 0; k < HE_KC; ++k) {
+        const float wv = ws[o][k];
+        for (int i = 0; i < TPT; ++i) acc[i] += wv * as[grp * TPT + i][k];
+      }
+    }
+  }
+  if (grp * TPT >= HE_TOK) return;
+  const float bias = bh[o];
+  const int ch = o / (p * p), dy = (o / p) % p, dx = o % p;
+  for (int i = 0; i < TPT; ++i) {
+    const int tok = tok0 + grp * TPT + i;
+    if (tok >= M) break;
+    const int b = tok / P, pt = tok % P, r = pt / gw, cc = pt % gw;
+    float* zp = z + (((size_t)b * C + ch) * H + r * p + dy) * W + cc * p + dx;
+    *zp += dt * (acc[i] + bias);
+  }
+}
+
+// ---------------------------------------------------------------------------------
+// gemv: one warp per output row.
+__global__ void __launch_bounds__(256) gemv_kernel(const bf16* __restrict__ W,
+                                                   const float* __restrict__ b,
+                                                   const float* __restrict__ x,
+                                                   float* __restrict__ y, int O, int K,
+                                                   int act_in, int act_out) {
+  const int warp = (blockIdx.x * blockDim.x + threadIdx.x) / 32, lane = threadIdx.x % 32;
+  if (warp >= O) return;
+  const bf16* wr = W + (size_t)warp * K;
+  float acc = 0.f;
+  for (int k = lane * 8; k < K; k += 32 * 8) {
+    float wv[8], xv[8];
+    load_bf16x8(wr + k, wv);
+    load_f32x8(x + k, xv);
+#pragma unroll
+    for (int j = 0; j < 8; ++j) acc += wv[j] * (act_in ? silu_f(xv[j]) : xv[j]);
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+  if (lane == 0) {
+    float v = acc + (b ? b[warp] : 0.f);
+    y[warp] = act_out ? silu_f(v) : v;
+  }
+}
+
+__global__ void timestep_sincos_kernel(float t, int dim, float* emb) {
+  const int half = dim / 2;
+  for (int k = threadIdx.x; k < half; k += blockDim.x) {
+    // f_k = 10000^(-k/half); the argument is formed in double for accuracy at 1000 t
+    const double f = exp(-9.210340371976184 * (double)k / (double)half);
+    const double arg = 1000.0 * (double)t * f;
+    emb[k] = (float)cos(arg);
+    emb[half + k] = (float)sin(arg);
+  }
+}
+
+__global__ void mod_prepare_kernel(const float* __restrict__ mod,
+                                   const float* __restrict__ tables, int L, int D,
+                                   float* __restrict__ modl, const float* __restrict__ htab,
+                                   const float* __restrict__ temb, float* __restrict__ head_mod) {
+  const size_t n6 = 6 * (size_t)D;
+  for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < (size_t)L * n6;
+       i += (size_t)gridDim.x * blockDim.x)
+    modl[i] = mod[i % n6] + tables[i];
+  if (blockIdx.x == 0)
+    for (int i = threadIdx.x; i < 2 * D; i += blockDim.x) head_mod[i] = htab[i] + temb[i % D];
+}
+
+__global__ void f32_to_bf16_kernel(const float* __restrict__ x, bf16* __restrict__ y, size_t n) {
+  for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < n;
+       i += (size_t)gridDim.x * blockDim.x)
+    y[i] = __float2bfloat16_rn(x[i]);
+}
+
+int grid_for(size_t work, int threads) {
+  size_t g = (work + threads - 1) / threads;
+  const size_t cap = 152 * 16;
+  return (int)(g < 1 ? 1 : (g > cap ? cap : g));
+}
+
+}  // namespace
+
+// ---- launchers --------------------------------------------------------------------
+
+cudaError_t ln_mod(const float* x, bf16* out, int rows, int D, float eps, float mul_base,
+                   const float* mul, const float* add, cudaStream_t st) {
+  if (rows == 0) return cudaSuccess;
+  switch (D) {  // threads * 4 * VPT == D
+    case 128: return ln_mod_launch<32, 1>(x, out, rows, D, eps, mul_base, mul, add, st);
+    case 256: return ln_mod_launch<64, 1>(x, out, rows, D, eps, mul_base, mul, add, st);
+    case 512: return ln_mod_launch<128, 1>(x, out, rows, D, eps, mul_base, mul, add, st);
+    case 1024: return ln_mod_launch<128, 2>(x, out, rows, D, eps, mul_base, mul, add, st);
+    case 1536: return ln_mod_launch<128, 3>(x, out, rows, D, eps, mul_base, mul, add, st);
+    case 2048: return ln_mod_launch<128, 4>(x, out, rows, D, eps, mul_base, mul, add, st);
+    case 3072: return ln_mod_launch<256, 3>(x, out, rows, D, eps, mul_base, mul, add, st);
+    case 4096: return ln_mod_launch<256, 4>(x, out, rows, D, eps, mul_base, mul, add, st);
+    case 5120: return ln_mod_launch<256, 5>(x, out, rows, D, eps, mul_base, mul, add, st);
+  }
+  return cudaErrorInvalidValue;
+}
+
+cudaError_t qk_norm_rope(bf16* x, int rows, int ld, int D, int nseg, int col0, const float* w0,
+                         int col1, const float* w1, float eps, const float2* rope, int tokens,
+                         int head_dim, cudaStream_t st) {
+  if (rows == 0) return cudaSuccess;
+#define QKN(T, V) qkn_launch<T, V>(x, rows, ld, D, nseg, col0, w0, col1, w1, eps, rope, tokens, head_dim, st)
+  switch (D) {  // threads * 4 * VPT == D
+    case 128: return QKN(32, 1);
+    case 256: return QKN(64, 1);
+    case 512: return QKN(128, 1);
+    case 1024: return QKN(128, 2);
+    case 1536: return QKN(128, 3);
+    case 2048: return QKN(128, 4);
+    case 3072: return QKN(256, 3);
+    case 4096: return QKN(256, 4);
+    case 5120: return QKN(256, 5);
+  }
+#undef QKN
+  return cudaErrorInvalidValue;
+}
+
+cudaError_t proxy_add(float* h, size_t n_elems, const ProxyTerms& t, cudaStream_t st) {
+  if (n_elems == 0 || t.n == 0) return cudaSuccess;
+  if (n_elems % 8) return cudaErrorInvalidValue;
+  const size_t n8 = n_elems / 8;
+  proxy_add_kernel<<<grid_for(n8, 256), 256, 0, st>>>(h, n8, t);
+  return cudaGetLastError();
+}
+
+cudaError_t patch_embed(const float* z, int n, int C, int H, int W, int p, const bf16* Wp,
+                        const float* bp, int D, float* h, cudaStream_t st) {
+  const int PD = C * p * p, M = n * (H / p) * (W / p);
+  if (M == 0) return cudaSuccess;
+  if (PD % 8 || PD > 64) return cudaErrorInvalidValue;
+  patch_embed_kernel<<<(M + PE_TOK - 1) / PE_TOK, 256, PE_TOK * PD * sizeof(float), st>>>(
+      z, n, C, H, W, p, Wp, bp, D, h);
+  return cudaGetLastError();
+}
+
+cudaError_t head_euler(const bf16* a, int n, int C, int H, int W, int p, const bf16* Wh,
+                       const float* bh, int D, float dt, float* z, cudaStream_t st) {
+  const int PD = C * p * p, M = n * (H / p) * (W / p);
+  if (M == 0) return cudaSuccess;
+  if (PD % 8 || PD > 64 || 256 % PD || D % 8) return cudaErrorInvalidValue;
+  head_euler_kernel<<<(M + HE_TOK - 1) / HE_TOK, 256, 0, st>>>(a, n, C, H, W, p, Wh, bh, D, dt, z);
+  return cudaGetLastError();
+}
+
+cudaError_t gemv(const bf16* W, const float* b, const float* x, float* y, int O, int K,
+                 int act_in, int act_out, cudaStream_t st) {
+  if (K % 8) return cudaErrorInvalidValue;
+  gemv_kernel<<<(O * 32 + 255) / 256, 256, 0, st>>>(W, b, x, y, O, K, act_in, act_out);
+  return cudaGetLastError();
+}
+
+cudaError_t timestep_sincos(float t, int dim, float* emb, cudaStream_t st) {
+  timestep_sincos_kernel<<<1, 128, 0, st>>>(t, dim, emb);
+  return cudaGetLastError();
+}
+
+cudaError_t mod_prepare(const float* mod, const float* tables, int L, int D, float* modl,
+                        const float* htab, const float* temb, float* head_mod, cudaStream_t st) {
+  mod_prepare_kernel<<<grid_for((size_t)L * 6 * D, 256), 256, 0, st>>>(mod, tables, L, D, modl,
+                                                                       htab, temb, head_mod);
+  return cudaGetLastError();
+}
+
+cudaError_t f32_to_bf16(const float* x, bf16* y, size_t n, cudaStream_t st) {
+  if (n == 0) return cudaSuccess;
+  f32_to_bf16_kernel<<<grid_for(n, 256), 256, 0, st>>>(x, y, n);
+  return cudaGetLastError();
+}

@@ -1,0 +1,272 @@
+"""ctypes binding of libflashbon.so (include/flashbon.h). Argument marshalling only:
+every step of the draft path runs in the library's CUDA kernels. There is no CPU
+fallback: if the library is missing, loading raises.
+
+Buffers may be numpy arrays (host memory) or torch tensors (host or CUDA); they are
+passed to the library as raw pointers and must be contiguous float32 / uint8 / int32.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+import numpy as np
+
+from . import synth
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libflashbon.so")
+
+FB_OK, FB_EINVAL, FB_ENOMEM, FB_ECUDA, FB_EPLAN, FB_ESTATE = range(6)
+KERNEL_KINDS = ["gemm_tc", "gemm_simt", "attn_self", "attn_cross", "ln_mod", "qk_norm_rope",
+                "proxy_add", "patch_embed", "head_euler", "small"]
+K = {name: i for i, name in enumerate(KERNEL_KINDS)}
+
+
+class FlashBonError(RuntimeError):
+    def __init__(self, status, msg):
+        super().__init__(f"flashbon status {status}: {msg}")
+        self.status = status
+
+
+class fb_cfg(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_int) for n in (
+        "depth", "dim", "heads", "head_dim", "ffn", "text_len", "text_dim", "latent_c",
+        "latent_h", "latent_w", "patch", "max_n", "freq_dim")] + [
+        ("eps_ln", ctypes.c_float), ("eps_rms", ctypes.c_float), ("rope_theta", ctypes.c_float)]
+
+
+class fb_kstat(ctypes.Structure):
+    _fields_ = [("launches", ctypes.c_uint64), ("ms", ctypes.c_double),
+                ("flops", ctypes.c_double), ("bytes", ctypes.c_double)]
+
+
+EXPORTS = ["fb_weights_count", "fb_weights_entry", "fb_init_model", "fb_free", "fb_set_stream",
+           "fb_encode_text", "fb_draft", "fb_refine", "fb_plan_from_phi", "fb_block_forward",
+           "fb_last_error", "fb_set_timing", "fb_get_stats", "fb_reset_stats", "fb_kernel_name",
+           "fb_op_gemm", "fb_op_attention"]
+
+_lib = None
+
+
+def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
+    """Loads libflashbon.so (raises FileNotFoundError if it was not built)."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(path):
+        raise FileNotFoundError(f"{path} not built: run paper_2607_04461_gb300.build.build()")
+    L = ctypes.CDLL(path)
+    P, I, S, F = ctypes.c_void_p, ctypes.c_int, ctypes.c_size_t, ctypes.c_float
+    sig = {
+        "fb_weights_count": (I, [ctypes.POINTER(fb_cfg), ctypes.POINTER(I), ctypes.POINTER(S)]),
+        "fb_weights_entry": (I, [ctypes.POINTER(fb_cfg), I, ctypes.POINTER(ctypes.c_char_p),
+                                 ctypes.POINTER(S), ctypes.POINTER(S)]),
+        "fb_init_model": (I, [ctypes.POINTER(fb_cfg), P, ctypes.POINTER(P)]),
+        "fb_free": (None, [P]),
+        "fb_set_stream": (I, [P, P]),
+        "fb_encode_text": (I, [P, P]),
+        "fb_draft": (I, [P, P, I, P, P, I, P, P]),
+        "fb_refine": (I, [P, P, P, P, I]),
+        "fb_plan_from_phi": (I, [I, I, I, I, I, I, I, I, P, P]),
+        "fb_block_forward": (I, [P, I, P, I, F]),
+        "fb_last_error": (ctypes.c_char_p, []),
+        "fb_set_timing": (I, [P, I]),
+        "fb_get_stats": (I, [P, P]),
+        "fb_reset_stats": (I, [P]),
+        "fb_kernel_name": (ctypes.c_char_p, [I]),
+        "fb_op_gemm": (I, [P, I, I, I, P, P, P, I, P, P, P, P, P, I]),
+        "fb_op_attention": (I, [P, P, I, P, I, P, I, P, I, I, I, I, I, I, I]),
+    }
+    for name, (res, args) in sig.items():
+        fn = getattr(L, name)
+        fn.restype, fn.argtypes = res, args
+    _lib = L
+    return L
+
+
+def _check(status):
+    if status != FB_OK:
+        raise FlashBonError(status, load_library().fb_last_error().decode())
+
+
+def _ptr(x, dtype=None):
+    """Raw pointer of a numpy array or torch tensor (must be contiguous)."""
+    if x is None:
+        return None
+    if isinstance(x, np.ndarray):
+        if dtype is not None and x.dtype != dtype:
+            raise TypeError(f"expected {dtype}, got {x.dtype}")
+        if not x.flags["C_CONTIGUOUS"]:
+            raise ValueError("array must be C-contiguous")
+        return x.ctypes.data
+    if hasattr(x, "data_ptr"):
+        if not x.is_contiguous():
+            raise ValueError("tensor must be contiguous")
+        return x.data_ptr()
+    if isinstance(x, int):
+        return x
+    raise TypeError(f"unsupported buffer type {type(x)}")
+
+
+def make_cfg(cfg: synth.Cfg) -> fb_cfg:
+    c = fb_cfg()
+    for f, _ in fb_cfg._fields_:
+        setattr(c, f, getattr(cfg, f))
+    return c
+
+
+def pack_weights(cfg: synth.Cfg, weights: dict) -> np.ndarray:
+    """Packs named weights into the library's fp32 layout (fb_weights_entry order)."""
+    L = load_library()
+    c = make_cfg(cfg)
+    count, total = ctypes.c_int(), ctypes.c_size_t()
+    _check(L.fb_weights_count(ctypes.byref(c), ctypes.byref(count), ctypes.byref(total)))
+    buf = np.empty(total.value, np.float32)
+    name, off, numel = ctypes.c_char_p(), ctypes.c_size_t(), ctypes.c_size_t()
+    for i in range(count.value):
+        _check(L.fb_weights_entry(ctypes.byref(c), i, ctypes.byref(name), ctypes.byref(off),
+                                  ctypes.byref(numel)))
+        w = np.asarray(weights[name.value.decode()], np.float32).ravel()
+        if w.size != numel.value:
+            raise ValueError(f"{name.value.decode()}: {w.size} elements, expected {numel.value}")
+        buf[off.value: off.value + numel.value] = w
+    return buf
+
+
+# ---- functions with the C-ABI names -------------------------------------------------
+
+def fb_init_model(cfg: synth.Cfg, weights) -> int:
+    """weights: dict of named arrays, or an already packed fp32 buffer."""
+    L = load_library()
+    packed = weights if isinstance(weights, np.ndarray) else pack_weights(cfg, weights)
+    c = make_cfg(cfg)
+    h = ctypes.c_void_p()
+    _check(L.fb_init_model(ctypes.byref(c), _ptr(packed, np.float32), ctypes.byref(h)))
+    return h.value
+
+
+def fb_free(model: int) -> None:
+    load_library().fb_free(model)
+
+
+def fb_set_stream(model: int, stream) -> None:
+    """stream: a torch.cuda.Stream, a raw cudaStream_t int, or None (model's own)."""
+    s = getattr(stream, "cuda_stream", stream)
+    _check(load_library().fb_set_stream(model, s))
+
+
+def fb_encode_text(model: int, text_ctx) -> None:
+    _check(load_library().fb_encode_text(model, _ptr(text_ctx, np.float32)))
+
+
+def fb_draft(model: int, latents, n: int, text_ctx, schedule, skip_mask=None,
+             proxy_plan=None) -> None:
+    sched = np.ascontiguousarray(schedule, np.float32)
+    sk = None if skip_mask is None else np.ascontiguousarray(skip_mask, np.uint8)
+    px = None if proxy_plan is None else np.ascontiguousarray(proxy_plan, np.int32)
+    n_steps = len(sched) - 1
+    for a in (sk, px):
+        if a is not None and a.shape[0] != n_steps:
+            raise ValueError("plan rows must equal len(schedule) - 1")
+    _check(load_library().fb_draft(model, _ptr(latents, np.float32), n,
+                                   _ptr(text_ctx, np.float32), _ptr(sched), n_steps,
+                                   _ptr(sk), _ptr(px)))
+
+
+def fb_refine(model: int, latent, text_ctx, full_schedule) -> None:
+    sched = np.ascontiguousarray(full_schedule, np.float32)
+    _check(load_library().fb_refine(model, _ptr(latent, np.float32), _ptr(text_ctx, np.float32),
+                                    _ptr(sched), len(sched) - 1))
+
+
+def fb_plan_from_phi(S, S_prime, n_skip, l_start, l_end, f_full, order, depth):
+    skip = np.zeros((S_prime, depth), np.uint8)
+    proxy = np.zeros((S_prime, depth), np.int32)
+    _check(load_library().fb_plan_from_phi(S, S_prime, n_skip, l_start, l_end, f_full, order,
+                                           depth, _ptr(skip), _ptr(proxy)))
+    return skip, proxy
+
+
+def fb_block_forward(model: int, layer: int, h, n: int, t: float) -> None:
+    _check(load_library().fb_block_forward(model, layer, _ptr(h), n, float(t)))
+
+
+def fb_set_timing(model: int, mask: int) -> None:
+    _check(load_library().fb_set_timing(model, int(mask)))
+
+
+def fb_get_stats(model: int) -> dict:
+    arr = (fb_kstat * len(KERNEL_KINDS))()
+    _check(load_library().fb_get_stats(model, ctypes.cast(arr, ctypes.c_void_p)))
+    return {KERNEL_KINDS[i]: dict(launches=int(arr[i].launches), ms=arr[i].ms,
+                                  flops=arr[i].flops, bytes=arr[i].bytes)
+            for i in range(len(KERNEL_KINDS))}
+
+
+def fb_reset_stats(model: int) -> None:
+    _check(load_library().fb_reset_stats(model))
+
+
+def fb_op_gemm(model, M, N, K, A, W, bias, epi, out, resid=None, gate=None, base=None,
+               delta=None, impl=0) -> None:
+    _check(load_library().fb_op_gemm(model, M, N, K, _ptr(A), _ptr(W), _ptr(bias), epi,
+                                     _ptr(out), _ptr(resid), _ptr(gate), _ptr(base),
+                                     _ptr(delta), impl))
+
+
+def fb_op_attention(model, Q, ldq, Kt, ldk, V, ldv, O, ldo, batch, Lq, Lkv, kv_batch_rows,
+                    heads, head_dim) -> None:
+    _check(load_library().fb_op_attention(model, _ptr(Q), ldq, _ptr(Kt), ldk, _ptr(V), ldv,
+                                          _ptr(O), ldo, batch, Lq, Lkv, kv_batch_rows, heads,
+                                          head_dim))
+
+
+class Model:
+    """Owns an fb_model handle; methods forward to the fb_* functions."""
+
+    def __init__(self, cfg: synth.Cfg, weights):
+        self.cfg = cfg
+        self.handle = fb_init_model(cfg, weights)
+
+    def close(self):
+        if self.handle:
+            fb_free(self.handle)
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    def __enter__(self):
+        return self
+
+    def __exit__(self, *exc):
+        self.close()
+
+    def set_stream(self, stream):
+        fb_set_stream(self.handle, stream)
+
+    def encode_text(self, ctx):
+        fb_encode_text(self.handle, ctx)
+
+    def draft(self, latents, text_ctx, schedule, skip_mask=None, proxy_plan=None, n=None):
+        n = latents.shape[0] if n is None else n
+        fb_draft(self.handle, latents, n, text_ctx, schedule, skip_mask, proxy_plan)
+
+    def refine(self, latent, text_ctx, schedule):
+        fb_refine(self.handle, latent, text_ctx, schedule)
+
+    def block_forward(self, layer, h, n, t):
+        fb_block_forward(self.handle, layer, h, n, t)
+
+    def set_timing(self, mask):
+        fb_set_timing(self.handle, mask)
+
+    def stats(self):
+        return fb_get_stats(self.handle)
+
+    def reset_stats(self):
+        fb_reset_stats(self.handle)

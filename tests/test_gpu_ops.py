@@ -1,0 +1,142 @@
+"""Kernel-level parity through the C-ABI single-op entry points: the tcgen05 GEMM (all
+epilogues, ragged M, both N tile widths), the CUDA-core GEMM, and flash attention
+(self / shared-K/V cross, head_dim 64 and 128, ragged tails) against the oracle's fp64
+primitives on the same bf16 inputs."""
+import numpy as np
+import pytest
+import torch
+
+from oracle import flashbon_oracle as O
+from paper_2607_04461_gb300 import flashbon as fb
+from paper_2607_04461_gb300 import synth
+from _metrics import rel_max
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def model():
+    fb.load_library()
+    m = fb.Model(synth.TINY, synth.make_weights(synth.TINY))
+    yield m
+    m.close()
+
+
+def randn(shape, seed, scale=1.0, dtype=torch.bfloat16):
+    g = torch.Generator().manual_seed(seed)
+    return (torch.randn(shape, generator=g) * scale).to(dtype).cuda()
+
+
+def f64(t):
+    return t.float().cpu().double().numpy()
+
+
+GEMM_SHAPES = [
+    (300, 256, 128),     # ragged M, BN=128, two K blocks
+    (1, 128, 64),        # one row, one K block
+    (2500, 384, 192),    # many tiles, BN=128
+    (4000, 4608, 256),   # >= one tile per SM at BN=256 (the QKV shape's N)
+    (640, 1536, 8960),   # long K (FFN down)
+]
+
+
+@pytest.mark.parametrize("M,N,K", GEMM_SHAPES)
+@pytest.mark.parametrize("epi", [0, 1, 2, 3])
+def test_gemm_tc(model, M, N, K, epi):
+    _gemm_case(model, M, N, K, epi, impl=0)
+
+
+@pytest.mark.parametrize("M,N,K", [(300, 256, 128), (77, 24, 40)])
+@pytest.mark.parametrize("epi", [0, 1, 2, 3])
+def test_gemm_simt(model, M, N, K, epi):
+    _gemm_case(model, M, N, K, epi, impl=1)
+
+
+def _gemm_case(model, M, N, K, epi, impl):
+    A = randn((M, K), 1)
+    W = randn((N, K), 2, scale=K ** -0.5)
+    bias = randn((N,), 3, dtype=torch.float32)
+    resid = randn((M, N), 4, dtype=torch.float32)
+    gate = randn((N,), 5, dtype=torch.float32)
+    base = randn((M, N), 6, dtype=torch.float32)
+    out = torch.empty((M, N), dtype=torch.bfloat16 if epi < 2 else torch.float32, device="cuda")
+    delta = torch.empty((M, N), dtype=torch.bfloat16, device="cuda")
+    fb.fb_op_gemm(model.handle, M, N, K, A, W, bias, epi, out,
+                  resid if epi >= 2 else None, gate if epi >= 2 else None,
+                  base if epi == 3 else None, delta if epi == 3 else None, impl)
+    torch.cuda.synchronize()
+    y = O.linear(f64(A), f64(W), f64(bias))
+    if epi == 0:
+        assert rel_max(f64(out), y) <= 1e-2
+    elif epi == 1:
+        assert rel_max(f64(out), O.gelu_tanh(y)) <= 1e-2
+    else:
+        want = f64(resid) + f64(gate) * y
+        assert rel_max(f64(out), want) <= 1e-4
+        if epi == 3:
+            assert rel_max(f64(delta), want - f64(base)) <= 1e-2
+
+
+def test_gemm_in_place_residual(model):
+    """out == resid and base == out (the block's last GEMM runs this way)."""
+    M, N, K = 257, 256, 128
+    A, W = randn((M, K), 11), randn((N, K), 12, scale=K ** -0.5)
+    h = randn((M, N), 13, dtype=torch.float32)
+    h0 = f64(h)
+    hb = randn((M, N), 14, dtype=torch.float32)
+    delta = torch.empty((M, N), dtype=torch.bfloat16, device="cuda")
+    fb.fb_op_gemm(model.handle, M, N, K, A, W, None, 3, h, hb, None, h, delta)
+    torch.cuda.synchronize()
+    want = f64(hb) + O.linear(f64(A), f64(W))
+    assert rel_max(f64(h), want) <= 1e-4
+    assert rel_max(f64(delta), want - h0) <= 1e-2
+
+
+ATTN_CASES = [
+    # batch, Lq, Lkv, heads, dh, shared_kv
+    (3, 150, 150, 2, 128, False),
+    (2, 70, 40, 3, 64, True),
+    (1, 1, 1, 1, 128, False),
+    (2, 1560, 512, 2, 128, True),
+    (1, 200, 333, 2, 64, False),
+]
+
+
+@pytest.mark.parametrize("batch,Lq,Lkv,heads,dh,shared", ATTN_CASES)
+def test_attention(model, batch, Lq, Lkv, heads, dh, shared):
+    D = heads * dh
+    q = randn((batch * Lq, D), 21)
+    kvb = 1 if shared else batch
+    k = randn((kvb * Lkv, D), 22)
+    v = randn((kvb * Lkv, D), 23)
+    o = torch.empty((batch * Lq, D), dtype=torch.bfloat16, device="cuda")
+    fb.fb_op_attention(model.handle, q, D, k, D, v, D, o, D, batch, Lq, Lkv,
+                       0 if shared else Lkv, heads, dh)
+    torch.cuda.synchronize()
+    qn, kn, vn, on = f64(q), f64(k), f64(v), f64(o)
+    for b in range(batch):
+        kb = 0 if shared else b
+        want = O.attention(qn[b * Lq:(b + 1) * Lq].reshape(Lq, heads, dh),
+                           kn[kb * Lkv:(kb + 1) * Lkv].reshape(Lkv, heads, dh),
+                           vn[kb * Lkv:(kb + 1) * Lkv].reshape(Lkv, heads, dh))
+        got = on[b * Lq:(b + 1) * Lq]
+        assert rel_max(got, want.reshape(Lq, D)) <= 2e-2
+        assert np.abs(got - want.reshape(Lq, D)).mean() <= 2e-3
+
+
+def test_attention_strided_qkv(model):
+    """Self-attention reading q, k, v from one packed [rows][3D] buffer."""
+    batch, L, heads, dh = 2, 97, 2, 128
+    D = heads * dh
+    qkv = randn((batch * L, 3 * D), 31)
+    o = torch.empty((batch * L, D), dtype=torch.bfloat16, device="cuda")
+    base = qkv.data_ptr()
+    fb.fb_op_attention(model.handle, base, 3 * D, base + 2 * D, 3 * D, base + 4 * D, 3 * D, o,
+                       D, batch, L, L, L, heads, dh)
+    torch.cuda.synchronize()
+    x = f64(qkv)
+    for b in range(batch):
+        r = x[b * L:(b + 1) * L]
+        want = O.attention(r[:, :D].reshape(L, heads, dh), r[:, D:2 * D].reshape(L, heads, dh),
+                           r[:, 2 * D:].reshape(L, heads, dh)).reshape(L, D)
+        assert rel_max(f64(o)[b * L:(b + 1) * L], want) <= 2e-2

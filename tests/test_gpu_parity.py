@@ -1,0 +1,284 @@
+"""Parity of the CUDA draft path (through the C-ABI) with the fp64 oracle.
+
+Small shapes are compared in full; the Wan2.1-1.3B-shaped workloads are run at full
+size in the configuration the benchmark uses and checked on sampled candidates the
+oracle computes one by one, plus properties that hold at any size."""
+import numpy as np
+import pytest
+import torch
+
+from oracle import flashbon_oracle as O
+from paper_2607_04461_gb300 import flashbon as fb
+from paper_2607_04461_gb300 import synth
+from _metrics import BLOCK_TOL, check_latents, rel_max
+
+pytestmark = pytest.mark.gpu
+
+
+def cuda(x):
+    return torch.from_numpy(np.ascontiguousarray(x)).cuda()
+
+
+@pytest.fixture(scope="module")
+def tiny():
+    cfg = synth.TINY
+    w = synth.make_weights(cfg, bf16=False, norm_std=0.2)
+    m = fb.Model(cfg, w)
+    yield cfg, w, m, O.OracleModel(cfg, w)
+    m.close()
+
+
+@pytest.fixture(scope="module")
+def small():
+    cfg = synth.SMALL
+    w = synth.make_weights(cfg, bf16=True, norm_std=0.2)
+    m = fb.Model(cfg, w)
+    yield cfg, w, m, O.OracleModel(cfg, w)
+    m.close()
+
+
+# ---- tiny DiT (2 blocks, hidden 128, 16 tokens, N=4, 4 steps, skip + proxy) ----------
+
+def test_tiny_draft_matches_oracle(tiny):
+    cfg, w, m, ref = tiny
+    z = synth.make_latents(cfg, 4)
+    ctx = synth.make_text(cfg)
+    sched = synth.make_schedule(4)
+    skip, proxy = synth.tiny_plan()
+    zd = cuda(z)
+    m.draft(zd, ctx, sched, skip, proxy)
+    got = zd.cpu().numpy()
+    want = ref.draft(z, ctx, sched, skip, proxy)
+    for j in range(4):
+        check_latents(got[j], want[j], z[j], label=f"tiny cand {j}")
+
+
+def test_tiny_host_and_device_latents_agree(tiny):
+    cfg, w, m, _ = tiny
+    z = synth.make_latents(cfg, 3)
+    ctx = synth.make_text(cfg)
+    sched = synth.make_schedule(4)
+    skip, proxy = synth.tiny_plan()
+    zh = z.copy()
+    m.draft(zh, ctx, sched, skip, proxy)
+    zd = cuda(z)
+    m.draft(zd, cuda(ctx), sched, skip, proxy)
+    np.testing.assert_array_equal(zh, zd.cpu().numpy())
+
+
+# ---- small shape: several tiles with ragged tails -------------------------------------
+
+def test_small_block_forward_each_layer(small):
+    cfg, w, m, ref = small
+    ctx = synth.make_text(cfg)
+    m.encode_text(ctx)
+    kv = ref.encode_text(ctx)
+    rng = np.random.default_rng(5)
+    n = cfg.max_n
+    h = rng.standard_normal((n * cfg.tokens, cfg.dim)).astype(np.float32)
+    t = 0.63
+    _, mod = ref.time_embed(np.float32(t))
+    for l in range(cfg.depth):
+        hd = cuda(h)
+        m.block_forward(l, hd, n, t)
+        got = hd.cpu().numpy().astype(np.float64) - h
+        for j in range(n):
+            hj = h[j * cfg.tokens:(j + 1) * cfg.tokens].astype(np.float64)
+            want = ref.block(l, hj, mod, kv[l]) - hj
+            e = rel_max(got[j * cfg.tokens:(j + 1) * cfg.tokens], want)
+            assert e <= BLOCK_TOL, f"layer {l} cand {j}: {e:.3e}"
+
+
+PLANS = {
+    "empty": lambda S, L: synth.empty_plan(S, L),
+    "skip_third_proxy_half": lambda S, L: synth.random_plan(S, L, 1 / 3, 0.5, seed=3),
+    "order1": lambda S, L: synth.random_plan(S, L, 0.0, 1.0, seed=4, order=1),
+    "phi_order2": lambda S, L: O.plan_from_phi(S + 2, S, 2, 2, 2, 2, 2, L),
+}
+
+
+@pytest.mark.parametrize("plan", list(PLANS))
+def test_small_draft_matches_oracle(small, plan):
+    cfg, w, m, ref = small
+    S = 5
+    z = synth.make_latents(cfg, cfg.max_n)
+    ctx = synth.make_text(cfg)
+    sched = synth.make_schedule(S)
+    skip, proxy = PLANS[plan](S, cfg.depth)
+    zd = cuda(z)
+    m.draft(zd, ctx, sched, skip, proxy)
+    got = zd.cpu().numpy()
+    want = ref.draft(z, ctx, sched, skip, proxy)
+    for j in range(cfg.max_n):
+        check_latents(got[j], want[j], z[j], label=f"{plan} cand {j}")
+
+
+def test_small_order2_taylor_with_three_anchors(small):
+    """Steps 0, 1, 2 computed; step 3 forecasts from three anchors (Eqs. 3-5)."""
+    cfg, w, m, ref = small
+    skip, proxy = synth.empty_plan(4, cfg.depth)
+    proxy[3, :] = synth.proxy_code(2, 2)
+    z = synth.make_latents(cfg, 2)
+    ctx = synth.make_text(cfg)
+    sched = synth.make_schedule(8)[:5]
+    zd = cuda(z)
+    m.draft(zd, ctx, sched, skip, proxy, n=2)
+    want = ref.draft(z, ctx, sched, skip, proxy)
+    for j in range(2):
+        check_latents(zd.cpu().numpy()[j], want[j], z[j], label=f"order2 cand {j}")
+
+
+def test_small_refine_and_markov(small):
+    """Refine matches the oracle; draft to step k then refine equals one full run
+    (bit-exact: same kernels on the same rows in the same order)."""
+    cfg, w, m, ref = small
+    S, k = 6, 2
+    z = synth.make_latents(cfg, 1)
+    ctx = synth.make_text(cfg)
+    sched = synth.make_schedule(S)
+    full = cuda(z)
+    m.draft(full, ctx, sched, *synth.empty_plan(S, cfg.depth))
+    part = cuda(z)
+    m.draft(part, ctx, sched[:k + 1], *synth.empty_plan(k, cfg.depth))
+    r = part[0].clone()
+    m.refine(r, ctx, sched[k:])
+    assert torch.equal(r, full[0])
+    want = ref.refine(part[0].cpu().numpy(), ctx, sched[k:])
+    check_latents(r.cpu().numpy(), want, part[0].cpu().numpy(), label="refine")
+
+
+def test_small_all_skipped_and_all_proxied(small):
+    cfg, w, m, ref = small
+    S = 3
+    z = synth.make_latents(cfg, 2)
+    ctx = synth.make_text(cfg)
+    sched = synth.make_schedule(S)
+    skip, proxy = synth.empty_plan(S, cfg.depth)
+    skip[0, :] = 1                      # step 0: every block skipped
+    proxy[2, :] = synth.proxy_code(1, 0)  # step 2: every block proxied from step 1
+    zd = cuda(z)
+    m.draft(zd, ctx, sched, skip, proxy, n=2)
+    want = ref.draft(z, ctx, sched, skip, proxy)
+    for j in range(2):
+        check_latents(zd.cpu().numpy()[j], want[j], z[j], label=f"skip/proxy-all cand {j}")
+
+
+def test_small_candidate_permutation_is_exact(small):
+    """Rows of different candidates never mix: permuting candidates permutes results."""
+    cfg, w, m, _ = small
+    z = synth.make_latents(cfg, 3)
+    ctx = synth.make_text(cfg)
+    sched = synth.make_schedule(3)
+    skip, proxy = synth.random_plan(3, cfg.depth, 1 / 3, 0.5, seed=9)
+    a, b = cuda(z), cuda(z[::-1])
+    m.draft(a, ctx, sched, skip, proxy)
+    m.draft(b, ctx, sched, skip, proxy)
+    assert torch.equal(a, b.flip(0))
+
+
+def test_edge_cases_and_errors(small):
+    cfg, w, m, _ = small
+    ctx = synth.make_text(cfg)
+    sched = synth.make_schedule(3)
+    z = cuda(synth.make_latents(cfg, 1))
+    z0 = z.clone()
+    m.draft(z, ctx, sched, n=0)                       # n == 0: no-op
+    assert torch.equal(z, z0)
+    fb.fb_draft(m.handle, z, 1, ctx, sched[:1])        # zero steps: no-op
+    assert torch.equal(z, z0)
+
+    def status(fn):
+        with pytest.raises(fb.FlashBonError) as e:
+            fn()
+        return e.value.status
+
+    big = cuda(synth.make_latents(cfg, cfg.max_n + 1))
+    assert status(lambda: m.draft(big, ctx, sched)) == fb.FB_EINVAL
+    assert status(lambda: m.draft(z, ctx, sched[::-1].copy())) == fb.FB_EINVAL
+    bad = sched.copy()
+    bad[1] = bad[0]
+    assert status(lambda: m.draft(z, ctx, bad)) == fb.FB_EINVAL
+    skip, proxy = synth.empty_plan(3, cfg.depth)
+    proxy[1, 0] = synth.proxy_code(1, 0)
+    assert status(lambda: m.draft(z, ctx, sched, skip, proxy)) == fb.FB_EPLAN
+    skip, proxy = synth.empty_plan(3, cfg.depth)
+    skip[0, 1] = 1
+    proxy[2, 1] = synth.proxy_code(0, 0)
+    assert status(lambda: m.draft(z, ctx, sched, skip, proxy)) == fb.FB_EPLAN
+    skip, proxy = synth.empty_plan(3, cfg.depth)
+    skip[2, 0] = 1
+    proxy[2, 0] = synth.proxy_code(0, 0)
+    assert status(lambda: m.draft(z, ctx, sched, skip, proxy)) == fb.FB_EPLAN
+    assert torch.equal(z, z0)                          # rejected calls changed nothing
+    assert status(lambda: m.block_forward(cfg.depth, z, 1, 0.5)) == fb.FB_EINVAL
+
+
+def test_block_forward_requires_text(small):
+    cfg, w, _, _ = small
+    with fb.Model(cfg.with_(depth=1, max_n=1), {k: v for k, v in w.items()
+                                                if not k.startswith("blocks.") or
+                                                k.startswith("blocks.0.")}) as m1:
+        h = torch.zeros((cfg.tokens, cfg.dim), device="cuda")
+        with pytest.raises(fb.FlashBonError) as e:
+            m1.block_forward(0, h, 1, 0.5)
+        assert e.value.status == fb.FB_ESTATE
+
+
+# ---- Wan2.1-1.3B shape at full size --------------------------------------------------
+
+def test_wan13_single_block_n16_sampled():
+    """One Wan2.1-1.3B-shaped block, N=16 (1560 tokens each), candidates 0 and 15."""
+    cfg = synth.WAN13.with_(depth=1, max_n=16)
+    w = synth.make_weights(cfg)
+    ctx = synth.make_text(cfg)
+    rng = np.random.default_rng(11)
+    n = 16
+    h = rng.standard_normal((n * cfg.tokens, cfg.dim)).astype(np.float32)
+    t = 0.5
+    with fb.Model(cfg, w) as m:
+        m.encode_text(ctx)
+        hd = cuda(h)
+        m.block_forward(0, hd, n, t)
+        got = hd.cpu().numpy().astype(np.float64) - h
+    ref = O.OracleModel(cfg, w)
+    kv = ref.encode_text(ctx)
+    _, mod = ref.time_embed(np.float32(t))
+    for j in (0, n - 1):
+        sl = slice(j * cfg.tokens, (j + 1) * cfg.tokens)
+        want = ref.block(0, h[sl].astype(np.float64), mod, kv[0]) - h[sl]
+        e = rel_max(got[sl], want)
+        assert e <= BLOCK_TOL, f"cand {j}: {e:.3e}"
+
+
+@pytest.fixture(scope="module")
+def wan13_pool():
+    cfg = synth.WAN13
+    w = synth.make_weights(cfg)
+    m = fb.Model(cfg, w)
+    yield cfg, w, m
+    m.close()
+
+
+def test_wan13_draft_pool_full_size(wan13_pool):
+    """The benchmark's draft pool: 30 blocks, N=32, 10 of 50 steps, 1/3 skipped per
+    step, half of the rest proxied on odd steps. Checked: candidate permutation is exact
+    at full size; the first two steps of candidate 0 match the oracle."""
+    cfg, w, m = wan13_pool
+    n, S = 32, 10
+    sched = synth.make_schedule(50)[:S + 1]
+    skip, proxy = synth.random_plan(S, cfg.depth, 1 / 3, 0.5, seed=7)
+    z = synth.make_latents(cfg, n)
+    ctx = synth.make_text(cfg)
+    a = cuda(z)
+    m.draft(a, ctx, sched, skip, proxy)
+    assert torch.isfinite(a).all()
+    perm = np.roll(np.arange(n), 5)
+    b = cuda(z[perm])
+    m.draft(b, ctx, sched, skip, proxy)
+    assert torch.equal(b, a[torch.from_numpy(perm).cuda()])
+    # oracle on candidate 0, first two steps of the same plan
+    two = cuda(z[:1])
+    m.draft(two, ctx, sched[:3], skip[:2], proxy[:2])
+    ref = O.OracleModel(cfg, w)
+    want = ref.draft(z[:1], ctx, sched[:3], skip[:2], proxy[:2])
+    check_latents(two.cpu().numpy()[0], want[0], z[0], label="wan13 cand 0, 2 steps")
