@@ -351,6 +351,46 @@ def run_gb300(args):
     return 0
 
 
+def run_probe(args):
+    """A few launches of one kernel on a case sized for an ncu capture (inputs larger
+    than L2, a few hundred MB on the device): gemm = the FFN up-projection shape
+    (8192 x 1536 -> 8960, GELU epilogue); gemm_resid = FFN down (8192 x 8960 -> 1536,
+    gated residual + contribution write); attn = self-attention over 1560 tokens,
+    4 candidates x 12 heads x 128."""
+    import torch
+    from paper_2607_04461_gb300 import flashbon as fb
+    torch.cuda.set_device(0)
+    cfg = synth.TINY
+    m = fb.Model(cfg, synth.make_weights(cfg))
+    g = torch.Generator().manual_seed(0)
+    rnd = lambda *s, dt=torch.bfloat16: (torch.randn(*s, generator=g) * 0.5).to(dt).cuda()  # noqa
+    if args.probe in ("gemm", "gemm_resid"):
+        M, D, F = 8192, 1536, 8960
+        if args.probe == "gemm":
+            A, W, out = rnd(M, D), rnd(F, D), torch.empty(M, F, dtype=torch.bfloat16, device="cuda")
+            b = rnd(F, dt=torch.float32)
+            call = lambda: fb.fb_op_gemm(m.handle, M, F, D, A, W, b, 1, out)  # noqa
+        else:
+            A, W, b = rnd(M, F), rnd(D, F), rnd(D, dt=torch.float32)
+            h, hb, gt = rnd(M, D, dt=torch.float32), rnd(M, D, dt=torch.float32), rnd(D, dt=torch.float32)
+            dl = torch.empty(M, D, dtype=torch.bfloat16, device="cuda")
+            call = lambda: fb.fb_op_gemm(m.handle, M, D, F, A, W, b, 3, h, hb, gt, h, dl)  # noqa
+    else:
+        n, P, H, dh = 4, 1560, 12, 128
+        qkv, o = rnd(n * P, 3 * H * dh), torch.empty(n * P, H * dh, dtype=torch.bfloat16, device="cuda")
+        base, D = qkv.data_ptr(), H * dh
+        call = lambda: fb.fb_op_attention(m.handle, base, 3 * D, base + 2 * D, 3 * D,  # noqa
+                                          base + 4 * D, 3 * D, o, D, n, P, P, P, H, dh)
+    m.reset_stats()
+    for _ in range(args.steps):
+        call()
+    torch.cuda.synchronize()
+    st = {k: v for k, v in m.stats().items() if v["launches"]}
+    print(json.dumps({"probe": args.probe, "launches": args.steps, "stats": st}))
+    m.close()
+    return 0
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -359,7 +399,10 @@ def main():
     ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
     ap.add_argument("--cpu-budget", type=float, default=15.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--probe", choices=["gemm", "gemm_resid", "attn"], default=None)
     args = ap.parse_args()
+    if args.probe:
+        return run_probe(args)
     if args.impl == "reference":
         return run_reference(args)
     return run_gb300(args)
