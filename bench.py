@@ -364,7 +364,9 @@ def run_probe(args):
     m = fb.Model(cfg, synth.make_weights(cfg))
     g = torch.Generator().manual_seed(0)
     rnd = lambda *s, dt=torch.bfloat16: (torch.randn(*s, generator=g) * 0.5).to(dt).cuda()  # noqa
-    if args.probe in ("gemm", "gemm_resid"):
+    if args.probe in ("gemm_shapes", "breakdown"):
+        call = None
+    elif args.probe in ("gemm", "gemm_resid"):
         M, D, F = 8192, 1536, 8960
         if args.probe == "gemm":
             A, W, out = rnd(M, D), rnd(F, D), torch.empty(M, F, dtype=torch.bfloat16, device="cuda")
@@ -381,6 +383,11 @@ def run_probe(args):
         base, D = qkv.data_ptr(), H * dh
         call = lambda: fb.fb_op_attention(m.handle, base, 3 * D, base + 2 * D, 3 * D,  # noqa
                                           base + 4 * D, 3 * D, o, D, n, P, P, P, H, dh)
+    if args.probe == "gemm_shapes":
+        return probe_gemm_shapes(m, rnd, args)
+    if args.probe == "breakdown":
+        m.close()
+        return probe_breakdown(args)
     m.reset_stats()
     for _ in range(args.steps):
         call()
@@ -388,6 +395,81 @@ def run_probe(args):
     st = {k: v for k, v in m.stats().items() if v["launches"]}
     print(json.dumps({"probe": args.probe, "launches": args.steps, "stats": st}))
     m.close()
+    return 0
+
+
+def probe_gemm_shapes(m, rnd, args):
+    """CUDA-event time of each block GEMM shape at the draft (N=32) and refine (N=1) row
+    counts, for the automatic kernel choice and the forced 1-SM kernel."""
+    import torch
+    from paper_2607_04461_gb300 import flashbon as fb
+    D, F = 1536, 8960
+    shapes = {"qkv": (3 * D, D, 0), "out": (D, D, 2), "cross_q": (D, D, 0),
+              "cross_out": (D, D, 2), "ffn_up": (F, D, 1), "ffn_down": (D, F, 3)}
+    res = {}
+    for M in (49920, 1560):
+        for name, (N, K, epi) in shapes.items():
+            A, W, b = rnd(M, K), rnd(N, K), rnd(N, dt=torch.float32)
+            out = torch.empty(M, N, dtype=torch.bfloat16 if epi < 2 else torch.float32, device="cuda")
+            r = rnd(M, N, dt=torch.float32) if epi >= 2 else None
+            dl = torch.empty(M, N, dtype=torch.bfloat16, device="cuda") if epi == 3 else None
+            for impl in (0, 2):
+                f = lambda: fb.fb_op_gemm(m.handle, M, N, K, A, W, b, epi, out, r, b if epi >= 2 else None,  # noqa
+                                          r if epi == 3 else None, dl, impl)
+                f()
+                torch.cuda.synchronize()
+                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                n = max(3, args.steps)
+                e0.record()
+                for _ in range(n):
+                    f()
+                e1.record()
+                torch.cuda.synchronize()
+                ms = e0.elapsed_time(e1) / n
+                res[f"M{M}/{name}/{'auto' if impl == 0 else '1sm'}"] = {
+                    "ms": round(ms, 4), "tflops": round(2 * M * N * K / ms / 1e9, 1)}
+            del A, W, out, r, dl
+    print(json.dumps({"probe": "gemm_shapes", "note": "each call includes one stream sync",
+                      "res": res}))
+    return 0
+
+
+def probe_breakdown(args):
+    """One bench step (draft + refine) with CUDA-event timing of every kernel class."""
+    import torch
+    from paper_2607_04461_gb300 import flashbon as fb
+    cfg, sched, skip, proxy = workload()
+    model = fb.Model(cfg, synth.make_weights(cfg))
+    z0 = torch.from_numpy(synth.make_latents(cfg, N_CAND)).cuda()
+    ctx = torch.from_numpy(synth.make_text(cfg)).cuda()
+    out = {}
+    for phase in ("draft", "refine"):
+        z = z0.clone()
+        for it in range(2):
+            model.reset_stats()
+            model.set_timing((1 << len(fb.KERNEL_KINDS)) - 1 if it else 0)
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            torch.cuda.synchronize()
+            e0.record()
+            if phase == "draft":
+                z.copy_(z0)
+                model.draft(z, ctx, sched[: S_DRAFT + 1], skip, proxy)
+            else:
+                zr = z0[0].clone()
+                model.refine(zr, ctx, sched[S_DRAFT:])
+            e1.record()
+            torch.cuda.synchronize()
+            if it:
+                st = model.stats()
+                out[phase] = {"wall_ms": e0.elapsed_time(e1),
+                              "kernels": {k: {"ms": round(v["ms"], 2), "launches": v["launches"],
+                                              "tflops": round(v["flops"] / v["ms"] / 1e9, 1) if v["ms"] else None,
+                                              "gbs": round(v["bytes"] / v["ms"] / 1e6, 1) if v["ms"] else None}
+                                          for k, v in st.items() if v["launches"]}}
+            else:
+                out[phase + "_untimed_ms"] = e0.elapsed_time(e1)
+    print(json.dumps({"probe": "breakdown", **out}))
+    model.close()
     return 0
 
 
@@ -399,7 +481,8 @@ def main():
     ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
     ap.add_argument("--cpu-budget", type=float, default=15.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--probe", choices=["gemm", "gemm_resid", "attn"], default=None)
+    ap.add_argument("--probe", choices=["gemm", "gemm_resid", "attn", "gemm_shapes", "breakdown"],
+                    default=None)
     args = ap.parse_args()
     if args.probe:
         return run_probe(args)

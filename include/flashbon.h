@@ -104,8 +104,9 @@ fb_status fb_encode_text(fb_model* m, const float* text_ctx);
  *            src_step < the current step, and the entry's skip bit must be 0.
  *            NULL skip_mask / proxy_plan mean "no skip" / "compute everything".
  *  Errors: FB_EINVAL (sizes, schedule), FB_EPLAN (plan rules above), FB_ENOMEM (proxy
- *  cache growth), FB_ECUDA. Latents are unchanged unless FB_OK is returned for a
- *  device pointer... (a device buffer may be partially updated on FB_ECUDA). */
+ *  cache growth), FB_ECUDA. Argument and plan errors are reported before any work is
+ *  enqueued and leave the latents unchanged; after FB_ECUDA a device buffer may be
+ *  partly updated. */
 fb_status fb_draft(fb_model* m, float* latents, int n, const float* text_ctx,
                    const float* schedule, int n_steps, const uint8_t* skip_mask,
                    const int32_t* proxy_plan);
@@ -170,8 +171,9 @@ const char* fb_kernel_name(int kind);
  *      equal out)
  *   3: as 2, and also delta bf16 = out - base[M][N] (fp32), base may equal out
  * A, W bf16 row-major, leading dimensions K; out / resid / base / delta leading
- * dimension N. impl: 0 = automatic (tcgen05 when N % 128 == 0 and K % 64 == 0),
- * 1 = force the CUDA-core kernel. */
+ * dimension N. impl: 0 = automatic (tcgen05 when N % 128 == 0 and K % 64 == 0: the
+ * 2-SM cta_group::2 kernel when N % 256 == 0, else the 1-SM kernel), 1 = force the
+ * CUDA-core kernel, 2 = force the 1-SM tcgen05 kernel (same shape rules). */
 fb_status fb_op_gemm(fb_model* m, int M, int N, int K, const void* A, const void* W,
                      const float* bias, int epi, void* out, const float* resid,
                      const float* gate, const float* base, void* delta, int impl);

@@ -249,14 +249,15 @@ fb_status end_call(fb_model* m) {
 }
 
 // ---- kernel wrappers with statistics ------------------------------------------------
-fb_status run_gemm(fb_model* m, const GemmArgs& g, int force_simt = 0) {
+// impl: 0 automatic, 1 CUDA-core kernel, 2 the 1-SM tcgen05 kernel
+fb_status run_gemm(fb_model* m, const GemmArgs& g, int impl = 0) {
   const double flops = 2.0 * g.M * (double)g.N * g.K;
   double bytes = 2.0 * ((double)g.M * g.K + (double)g.N * g.K);
   bytes += (g.kind <= EPI_GELU_BF16) ? 2.0 * g.M * g.N : 8.0 * g.M * g.N;
   if (g.kind == EPI_RESID_DELTA) bytes += 6.0 * g.M * g.N;
-  if (!force_simt && gemm_tc_supported(g)) {
+  if (impl != 1 && gemm_tc_supported(g)) {
     KTimer t(m, FB_K_GEMM_TC, flops, bytes);
-    CK(gemm_tc(g, m->derr, m->num_sms, m->st));
+    CK(gemm_tc(g, m->derr, m->num_sms, m->st, impl == 2));
   } else {
     KTimer t(m, FB_K_GEMM_SIMT, flops, bytes);
     CK(gemm_simt(g, m->st));
@@ -882,7 +883,8 @@ fb_status fb_op_gemm(fb_model* m, int M, int N, int K, const void* A, const void
   g.epi.base = base;
   g.epi.delta = (bf16*)delta;
   CKS(begin_call(m));
-  CKS(run_gemm(m, g, impl == 1));
+  if (impl < 0 || impl > 2) return fail(FB_EINVAL, "impl must be 0, 1 or 2");
+  CKS(run_gemm(m, g, impl));
   return end_call(m);
 }
 

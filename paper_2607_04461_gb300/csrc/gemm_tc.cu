@@ -201,6 +201,156 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   }
 }
 
+// ---- 2-SM variant -------------------------------------------------------------------
+// A cluster of two CTAs computes a 256 x 256 tile with tcgen05.mma.cta_group::2: CTA r
+// of the pair holds rows 128 r .. 128 r + 127 of the A tile and rows 128 r .. of the W
+// tile in its shared memory, and receives rows 128 r .. of the accumulator in its TMEM.
+// Per SM this moves 32 KB per K block instead of 48 KB for the same MMA work, so six
+// stages fit. The even CTA issues the MMAs; its "full" barriers count the TMA bytes of
+// both CTAs (the odd CTA's loads complete on them across the pair), its commits arrive on
+// the "empty" / "tmem_full" barriers of both CTAs, and both CTAs' epilogue warps release
+// an accumulator on its "tmem_empty" barrier.
+constexpr int C2_BN = 256;
+constexpr int C2_STAGES = 6;
+constexpr int C2_HALF_BYTES = 128 * BK * 2;          // 16 KB: 128 rows x 64 bf16
+constexpr int C2_STAGE_BYTES = 2 * C2_HALF_BYTES;    // this CTA's A rows + W rows
+constexpr int C2_TMEM_COLS = 2 * C2_BN;
+constexpr int C2_SMEM_BYTES = C2_STAGES * C2_STAGE_BYTES + 1024 + 256;
+
+template <int KIND>
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
+    gemm_tc2_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmW,
+                    int M, int N, int K, GemmEpi epi, int* err) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + C2_STAGES * C2_STAGE_BYTES);
+  uint64_t* empty = full + C2_STAGES;
+  uint64_t* tmem_full = empty + C2_STAGES;
+  uint64_t* tmem_empty = tmem_full + 2;
+  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(tmem_empty + 2);
+
+  const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+  const uint32_t rank = cluster_ctarank();
+  const int cluster = blockIdx.x >> 1, n_clusters = gridDim.x >> 1;
+  const int n_mt = (M + 2 * BM - 1) / (2 * BM), n_nt = N / C2_BN, n_tiles = n_mt * n_nt;
+  const int nk = K / BK;
+  bool failed = false;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < C2_STAGES; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(&tmem_full[a], 1);
+      mbar_init(&tmem_empty[a], 8);  // 4 epilogue warps x 2 CTAs
+    }
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    tma_prefetch_desc(&tmA);
+    tma_prefetch_desc(&tmW);
+  }
+  if (warp == 1) tmem_alloc_cg2(tmem_holder, C2_TMEM_COLS);
+  tc_fence_before();
+  cluster_sync();  // both CTAs' barriers initialised, TMEM allocated
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_holder;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ---------------- TMA producer (both CTAs) ----------------
+      int stage = 0;
+      uint32_t phase = 0;
+      for (int tile = cluster; tile < n_tiles && !failed; tile += n_clusters) {
+        const int m0 = (tile / n_nt) * 2 * BM, n0 = (tile % n_nt) * C2_BN;
+        for (int kb = 0; kb < nk; ++kb) {
+          if (!mbar_wait(&empty[stage], phase ^ 1u, err)) { failed = true; break; }
+          uint8_t* sa = smem + stage * C2_STAGE_BYTES;
+          if (rank == 0) mbar_expect_tx(&full[stage], 2 * C2_STAGE_BYTES);
+          const uint32_t fb = mapa_shared(smem_u32(&full[stage]), 0);
+          tma_load_2d_cg2(sa, &tmA, fb, kb * BK, m0 + BM * (int)rank);
+          tma_load_2d_cg2(sa + C2_HALF_BYTES, &tmW, fb, kb * BK, n0 + 128 * (int)rank);
+          if (++stage == C2_STAGES) { stage = 0; phase ^= 1u; }
+        }
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0 && rank == 0) {
+      // ---------------- MMA issuer (even CTA) ----------------
+      const uint32_t idesc = (1u << 4) | (1u << 7) | (1u << 10) |
+                             ((uint32_t)(C2_BN >> 3) << 17) | ((uint32_t)((2 * BM) >> 4) << 24);
+      int stage = 0;
+      uint32_t phase = 0;
+      int it = 0;
+      for (int tile = cluster; tile < n_tiles && !failed; tile += n_clusters, ++it) {
+        const int acc = it & 1;
+        const uint32_t acc_phase = (it >> 1) & 1;
+        if (!mbar_wait(&tmem_empty[acc], acc_phase ^ 1u, err)) { failed = true; break; }
+        tc_fence_after();
+        const uint32_t d_tmem = tmem_base + acc * C2_BN;
+        for (int kb = 0; kb < nk; ++kb) {
+          if (!mbar_wait(&full[stage], phase, err)) { failed = true; break; }
+          tc_fence_after();
+          const uint32_t sa = smem_u32(smem + stage * C2_STAGE_BYTES);
+          const uint64_t adesc = sdesc_sw128(sa), bdesc = sdesc_sw128(sa + C2_HALF_BYTES);
+#pragma unroll
+          for (int k = 0; k < BK / 16; ++k)
+            tc_mma_f16_cg2(d_tmem, adesc + 2 * k, bdesc + 2 * k, idesc, (kb | k) ? 1u : 0u);
+          tc_commit_mc(&empty[stage], 0x3);
+          if (++stage == C2_STAGES) { stage = 0; phase ^= 1u; }
+        }
+        if (!failed) tc_commit_mc(&tmem_full[acc], 0x3);
+      }
+    }
+  } else {
+    // ---------------- epilogue (warps 2..5 of both CTAs) ----------------
+    const int quarter = warp & 3;
+    const uint32_t te_remote = mapa_shared(smem_u32(&tmem_empty[0]), 0);
+    int it = 0;
+    for (int tile = cluster; tile < n_tiles; tile += n_clusters, ++it) {
+      const int acc = it & 1;
+      const uint32_t acc_phase = (it >> 1) & 1;
+      const int m0 = (tile / n_nt) * 2 * BM, n0 = (tile % n_nt) * C2_BN;
+      const bool ok = mbar_wait(&tmem_full[acc], acc_phase, err);
+      if (!__all_sync(0xffffffffu, ok)) { failed = true; break; }
+      tc_fence_after();
+      const int row = m0 + BM * (int)rank + quarter * 32 + lane;
+      const uint32_t taddr = tmem_base + ((uint32_t)(quarter * 32) << 16) + acc * C2_BN;
+#pragma unroll 1
+      for (int c = 0; c < C2_BN / 32; ++c) {
+        uint32_t r[32];
+        tmem_ld32(taddr + c * 32, r);
+        tmem_ld_wait();
+        if (row < M) {
+#pragma unroll
+          for (int g = 0; g < 4; ++g) {
+            float v[8];
+#pragma unroll
+            for (int j = 0; j < 8; ++j) v[j] = __uint_as_float(r[g * 8 + j]);
+            epi_apply8<KIND>(epi, row, n0 + c * 32 + g * 8, v);
+          }
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive_cluster(te_remote + acc * (uint32_t)sizeof(uint64_t));
+    }
+  }
+
+  if (failed || *(volatile int*)err != 0) {
+    // After a timeout, give TMA loads that may still be in flight time to land before
+    // the shared memory they target is released (they complete within microseconds).
+    const uint64_t t0 = fb_globaltimer();
+    while (fb_globaltimer() - t0 < 100000ull) __nanosleep(1000);
+  }
+  tc_fence_before();
+  cluster_sync();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc_cg2(tmem_base, C2_TMEM_COLS);
+  }
+}
+
 PFN_cuTensorMapEncodeTiled_v12000 get_encode() {
   static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
   if (!fn) {
@@ -256,6 +406,46 @@ cudaError_t dispatch_kind(const GemmArgs& g, int* err, int num_sms, cudaStream_t
   return cudaErrorInvalidValue;
 }
 
+template <int KIND>
+cudaError_t launch2(const GemmArgs& g, int* err, int num_sms, cudaStream_t st) {
+  CUtensorMap ma, mw;
+  if (!make_map(&ma, g.A, g.M, g.K, g.lda, BM) || !make_map(&mw, g.W, g.N, g.K, g.ldw, 128))
+    return cudaErrorInvalidValue;
+  cudaError_t e = cudaFuncSetAttribute(gemm_tc2_kernel<KIND>,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize, C2_SMEM_BYTES);
+  if (e != cudaSuccess) return e;
+  // as many clusters as can be resident at once (pairs must share a GPC)
+  static int max_clusters[4] = {0, 0, 0, 0};
+  int& mc = max_clusters[KIND];
+  if (mc == 0) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(num_sms, 1, 1);
+    cfg.blockDim = dim3(NUM_THREADS, 1, 1);
+    cfg.dynamicSmemBytes = C2_SMEM_BYTES;
+    int n = 0;
+    if (cudaOccupancyMaxActiveClusters(&n, gemm_tc2_kernel<KIND>, &cfg) != cudaSuccess || n < 1) {
+      cudaGetLastError();
+      n = num_sms / 2;
+    }
+    mc = n < num_sms / 2 ? n : num_sms / 2;
+  }
+  const int tiles = ((g.M + 2 * BM - 1) / (2 * BM)) * (g.N / C2_BN);
+  const int clusters = tiles < mc ? tiles : mc;
+  gemm_tc2_kernel<KIND><<<2 * clusters, NUM_THREADS, C2_SMEM_BYTES, st>>>(ma, mw, g.M, g.N, g.K,
+                                                                         g.epi, err);
+  return cudaGetLastError();
+}
+
+cudaError_t dispatch2(const GemmArgs& g, int* err, int num_sms, cudaStream_t st) {
+  switch (g.kind) {
+    case EPI_BF16: return launch2<EPI_BF16>(g, err, num_sms, st);
+    case EPI_GELU_BF16: return launch2<EPI_GELU_BF16>(g, err, num_sms, st);
+    case EPI_RESID: return launch2<EPI_RESID>(g, err, num_sms, st);
+    case EPI_RESID_DELTA: return launch2<EPI_RESID_DELTA>(g, err, num_sms, st);
+  }
+  return cudaErrorInvalidValue;
+}
+
 }  // namespace
 
 bool gemm_tc_supported(const GemmArgs& g) {
@@ -264,9 +454,11 @@ bool gemm_tc_supported(const GemmArgs& g) {
          g.ldw % 8 == 0 && g.epi.ldo % 8 == 0 && al16(g.A) && al16(g.W) && al16(g.epi.out);
 }
 
-cudaError_t gemm_tc(const GemmArgs& g, int* err, int num_sms, cudaStream_t st) {
+cudaError_t gemm_tc(const GemmArgs& g, int* err, int num_sms, cudaStream_t st, bool force_1sm) {
   if (!gemm_tc_supported(g)) return cudaErrorInvalidValue;
-  // BN = 256 halves the A re-reads; use it when it still gives every SM a tile.
+  // 2-SM 256 x 256 tiles whenever N allows; otherwise 1-SM 128 x BN tiles, BN = 256
+  // when that still gives every SM a tile.
+  if (g.N % C2_BN == 0 && !force_1sm && num_sms >= 2) return dispatch2(g, err, num_sms, st);
   const int mt = (g.M + BM - 1) / BM;
   if (g.N % 256 == 0 && mt * (g.N / 256) >= num_sms) return dispatch_kind<256>(g, err, num_sms, st);
   return dispatch_kind<128>(g, err, num_sms, st);

@@ -17,9 +17,11 @@ struct GemmArgs {
   int kind;       // EPI_*
   GemmEpi epi;
 };
-// tcgen05 path: requires N % 128 == 0, K % 64 == 0, 16-byte aligned rows.
+// tcgen05 path: requires N % 128 == 0, K % 64 == 0, 16-byte aligned rows. Uses the
+// 2-SM (cta_group::2) kernel when N % 256 == 0 unless force_1sm.
 bool gemm_tc_supported(const GemmArgs& g);
-cudaError_t gemm_tc(const GemmArgs& g, int* err, int num_sms, cudaStream_t st);
+cudaError_t gemm_tc(const GemmArgs& g, int* err, int num_sms, cudaStream_t st,
+                    bool force_1sm = false);
 // CUDA-core path: requires N % 8 == 0.
 cudaError_t gemm_simt(const GemmArgs& g, cudaStream_t st);
 

@@ -43,7 +43,20 @@ GEMM_SHAPES = [
 @pytest.mark.parametrize("M,N,K", GEMM_SHAPES)
 @pytest.mark.parametrize("epi", [0, 1, 2, 3])
 def test_gemm_tc(model, M, N, K, epi):
+    """Automatic choice: the 2-SM kernel when N % 256 == 0, else the 1-SM kernel."""
     _gemm_case(model, M, N, K, epi, impl=0)
+
+
+@pytest.mark.parametrize("M,N,K", [(300, 256, 128), (1560, 1536, 1536), (513, 512, 8960)])
+@pytest.mark.parametrize("epi", [0, 3])
+def test_gemm_tc_1sm_forced(model, M, N, K, epi):
+    _gemm_case(model, M, N, K, epi, impl=2)
+
+
+@pytest.mark.parametrize("M", [1, 129, 256, 257, 1560, 49920])
+def test_gemm_tc_2sm_ragged_rows(model, M):
+    """Pair tiles of 256 rows: rows of the odd CTA may lie wholly past M."""
+    _gemm_case(model, M, 512, 128, 0, impl=0)
 
 
 @pytest.mark.parametrize("M,N,K", [(300, 256, 128), (77, 24, 40)])
