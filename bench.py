@@ -382,7 +382,8 @@ def run_probe(args):
         qkv, o = rnd(n * P, 3 * H * dh), torch.empty(n * P, H * dh, dtype=torch.bfloat16, device="cuda")
         base, D = qkv.data_ptr(), H * dh
         call = lambda: fb.fb_op_attention(m.handle, base, 3 * D, base + 2 * D, 3 * D,  # noqa
-                                          base + 4 * D, 3 * D, o, D, n, P, P, P, H, dh)
+                                          base + 4 * D, 3 * D, o, D, n, P, P, P, H, dh,
+                                          1 if args.probe == "attn_mma" else 0)
     if args.probe == "gemm_shapes":
         return probe_gemm_shapes(m, rnd, args)
     if args.probe == "breakdown":
@@ -481,7 +482,8 @@ def main():
     ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
     ap.add_argument("--cpu-budget", type=float, default=15.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--probe", choices=["gemm", "gemm_resid", "attn", "gemm_shapes", "breakdown"],
+    ap.add_argument("--probe", choices=["gemm", "gemm_resid", "attn", "attn_mma", "gemm_shapes",
+                                        "breakdown"],
                     default=None)
     args = ap.parse_args()
     if args.probe:

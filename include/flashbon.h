@@ -180,10 +180,12 @@ fb_status fb_op_gemm(fb_model* m, int M, int N, int K, const void* A, const void
 /* fb_op_attention: O = softmax(Q K^T / sqrt(head_dim)) V per (batch, head), bf16 row
  * major; Q rows b*Lq..b*Lq+Lq-1 with row stride ldq elements, head h at column
  * h*head_dim; likewise K, V (kv_batch_rows = 0 shares one K/V across the batch,
- * otherwise the row offset between batches); O row stride ldo. */
+ * otherwise the row offset between batches); O row stride ldo. impl: 0 = automatic
+ * (the tcgen05 kernel for head_dim 128, the mma.sync kernel for 64), 1 = force the
+ * mma.sync kernel. */
 fb_status fb_op_attention(fb_model* m, const void* Q, int ldq, const void* K, int ldk,
                           const void* V, int ldv, void* O, int ldo, int batch, int Lq,
-                          int Lkv, int kv_batch_rows, int heads, int head_dim);
+                          int Lkv, int kv_batch_rows, int heads, int head_dim, int impl);
 
 #ifdef __cplusplus
 }

@@ -17,7 +17,8 @@ ROOT = os.path.dirname(PKG)
 CSRC = os.path.join(PKG, "csrc")
 BUILD = os.path.join(ROOT, "_build")
 LIB = os.path.join(PKG, "libflashbon.so")
-SOURCES = ["api.cu", "gemm_tc.cu", "gemm_simt.cu", "attention.cu", "pointwise.cu"]
+SOURCES = ["api.cu", "gemm_tc.cu", "gemm_simt.cu", "attention.cu", "attention_tc.cu",
+           "pointwise.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

@@ -278,12 +278,14 @@ GemmArgs gemm_args(int M, int N, int K, const bf16* A, const bf16* W, const floa
   return g;
 }
 
-fb_status run_attn(fb_model* m, const AttnArgs& a, int kind) {
+// impl: 0 automatic (tcgen05 for head_dim 128), 1 the mma.sync kernel
+fb_status run_attn(fb_model* m, const AttnArgs& a, int kind, int impl = 0) {
   const double flops = 4.0 * a.batch * a.heads * (double)a.Lq * a.Lkv * a.head_dim;
   const double kvb = (a.kv_batch_rows ? a.batch : 1) * 2.0 * a.Lkv * a.heads * a.head_dim * 2;
   const double bytes = 2.0 * a.batch * a.Lq * (double)a.heads * a.head_dim * 2 + kvb;
   KTimer t(m, kind, flops, bytes);
-  CK(attention(a, m->st));
+  if (impl == 0 && attention_tc_supported(a)) CK(attention_tc(a, m->derr, m->st));
+  else CK(attention(a, m->st));
   return FB_OK;
 }
 
@@ -890,8 +892,9 @@ fb_status fb_op_gemm(fb_model* m, int M, int N, int K, const void* A, const void
 
 fb_status fb_op_attention(fb_model* m, const void* Q, int ldq, const void* K, int ldk,
                           const void* V, int ldv, void* O, int ldo, int batch, int Lq, int Lkv,
-                          int kv_batch_rows, int heads, int head_dim) {
+                          int kv_batch_rows, int heads, int head_dim, int impl) {
   if (!m || !Q || !K || !V || !O) return fail(FB_EINVAL, "null argument");
+  if (impl < 0 || impl > 1) return fail(FB_EINVAL, "impl must be 0 or 1");
   if (batch < 1 || Lq < 1 || Lkv < 1 || heads < 1 || (head_dim != 64 && head_dim != 128))
     return fail(FB_EINVAL, "bad sizes");
   AttnArgs a{};
@@ -900,7 +903,7 @@ fb_status fb_op_attention(fb_model* m, const void* Q, int ldq, const void* K, in
   a.batch = batch; a.Lq = Lq; a.Lkv = Lkv; a.kv_batch_rows = kv_batch_rows;
   a.heads = heads; a.head_dim = head_dim;
   CKS(begin_call(m));
-  CKS(run_attn(m, a, FB_K_ATTN_SELF));
+  CKS(run_attn(m, a, FB_K_ATTN_SELF, impl));
   return end_call(m);
 }
 

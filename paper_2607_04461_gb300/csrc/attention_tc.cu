@@ -1,0 +1,364 @@
+// tcgen05 flash attention (head_dim 128) for the DiT block's self- and cross-attention:
+// O = softmax(Q K^T / sqrt(128)) V per (batch, head), non-causal, ragged tails masked.
+//
+// One CTA = one 128-query tile of one (batch, head); 6 warps:
+//  * warp 0, one thread: TMA producer. Q once (2 x [128 rows][64 cols] boxes), then
+//    128-key K and V tiles into a 2-deep ring (64 KB per stage), 128-byte swizzle.
+//  * warp 1: TMEM owner (512 columns: S0, S1, O) and, one thread, the MMA issuer:
+//    S_j = Q K_j^T into S[j % 2] (M=128, N=128 keys, K=128, both operands K-major),
+//    then, once the softmax has written P_j, O += P_j V_j (A = P from shared memory,
+//    K-major over keys; B = V, MN-major: the V tile is read as stored, [key][dim]).
+//  * warps 2-5: softmax, one query row per thread (TMEM lane = row). Each reads its S
+//    row (128 fp32), keeps the running row max m and sum l in registers, writes
+//    P = exp2(S * log2(e)/sqrt(d) - m) as bf16 into the swizzled P tile, and rescales its
+//    O row in TMEM only when the max grew by more than 2^8 since the last rescale
+//    (every term of O and l always uses the same m, so the result is exact). At the end
+//    each thread normalises its O row and stores it.
+// All waits are bounded; on a timeout the kernel records the error and drains.
+#include <cudaTypedefs.h>
+
+#include "kernels.h"
+
+namespace {
+
+constexpr int TB = 128;                    // queries per CTA = keys per KV tile
+constexpr int SUB = TB * 64 * 2;           // 16 KB: 128 rows x 64 bf16 (one swizzle width)
+constexpr int Q_BYTES = 2 * SUB;           // 32 KB
+constexpr int KV_BYTES = 4 * SUB;          // K (2 sub-tiles) + V (2 sub-tiles)
+constexpr int P_BYTES = 2 * SUB;
+constexpr int NSTAGE = 2;
+constexpr int SMEM_BYTES = Q_BYTES + NSTAGE * KV_BYTES + P_BYTES + 1024 + 256;
+constexpr int THREADS = 192;
+constexpr uint32_t TMEM_COLS = 512;        // S0 [0,128), S1 [128,256), O [256,384)
+constexpr uint32_t O_COL = 256;
+
+struct Params {
+  int Lq, Lkv, kv_batch_rows;
+  bf16* O;
+  int ldo;
+  float scale_log2;
+  int* err;
+};
+
+__device__ __forceinline__ uint64_t desc_k_sw128(uint32_t saddr) {
+  uint64_t d = (uint64_t)((saddr & 0x3FFFFu) >> 4);
+  d |= (uint64_t)1 << 16;               // leading byte offset (unused, K-major swizzled)
+  d |= (uint64_t)(1024 >> 4) << 32;     // 8-row groups 1024 B apart
+  d |= (uint64_t)1 << 46;
+  d |= (uint64_t)2 << 61;               // 128-byte swizzle
+  return d;
+}
+// MN-major, 128-byte swizzle: 64 consecutive N elements per 128-byte row, one row per K;
+// 8-row (K) groups 1024 B apart (stride byte offset), the next 64 N elements lbo bytes on.
+__device__ __forceinline__ uint64_t desc_mn_sw128(uint32_t saddr, uint32_t lbo) {
+  uint64_t d = (uint64_t)((saddr & 0x3FFFFu) >> 4);
+  d |= (uint64_t)((lbo >> 4) & 0x3FFFu) << 16;
+  d |= (uint64_t)(1024 >> 4) << 32;
+  d |= (uint64_t)1 << 46;
+  d |= (uint64_t)2 << 61;
+  return d;
+}
+
+__device__ __forceinline__ float ex2(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+__device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t* r) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], "
+      "{%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,"
+      "%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32};" ::"r"(taddr),
+      "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]),
+      "r"(r[8]), "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]),
+      "r"(r[15]), "r"(r[16]), "r"(r[17]), "r"(r[18]), "r"(r[19]), "r"(r[20]), "r"(r[21]),
+      "r"(r[22]), "r"(r[23]), "r"(r[24]), "r"(r[25]), "r"(r[26]), "r"(r[27]), "r"(r[28]),
+      "r"(r[29]), "r"(r[30]), "r"(r[31])
+      : "memory");
+}
+__device__ __forceinline__ void tmem_st_wait() {
+  asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void fence_async_smem() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
+__global__ void __launch_bounds__(THREADS, 1)
+    attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
+                   const __grid_constant__ CUtensorMap tmV, Params p) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint8_t* Qs = smem;
+  uint8_t* KVs = smem + Q_BYTES;
+  uint8_t* Ps = KVs + NSTAGE * KV_BYTES;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(Ps + P_BYTES);
+  uint64_t* q_full = bars;
+  uint64_t* kv_full = bars + 1;       // [2]
+  uint64_t* kv_empty = bars + 3;      // [2]
+  uint64_t* s_full = bars + 5;        // [2]
+  uint64_t* p_full = bars + 7;
+  uint64_t* o_done = bars + 8;
+  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(bars + 9);
+
+  const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+  const int qt = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
+  const int q_row0 = b * p.Lq + qt * TB;
+  const int kv_row0 = b * p.kv_batch_rows;
+  const int n_kv = (p.Lkv + TB - 1) / TB;
+  int* err = p.err;
+  bool failed = false;
+
+  if (threadIdx.x == 0) {
+    mbar_init(q_full, 1);
+    for (int s = 0; s < NSTAGE; ++s) {
+      mbar_init(&kv_full[s], 1);
+      mbar_init(&kv_empty[s], 1);
+      mbar_init(&s_full[s], 1);
+    }
+    mbar_init(p_full, 4);   // one arrival per softmax warp
+    mbar_init(o_done, 1);
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    tma_prefetch_desc(&tmQ);
+    tma_prefetch_desc(&tmK);
+    tma_prefetch_desc(&tmV);
+  }
+  if (warp == 1) tmem_alloc(tmem_holder, TMEM_COLS);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_holder;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ---------------- TMA producer ----------------
+      const int xq = h * 128;
+      mbar_expect_tx(q_full, Q_BYTES);
+      tma_load_2d(Qs, &tmQ, q_full, xq, q_row0);
+      tma_load_2d(Qs + SUB, &tmQ, q_full, xq + 64, q_row0);
+      for (int j = 0; j < n_kv; ++j) {
+        const int s = j & 1;
+        if (!mbar_wait(&kv_empty[s], ((j >> 1) & 1) ^ 1u, err)) { failed = true; break; }
+        uint8_t* st = KVs + s * KV_BYTES;
+        const int y = kv_row0 + j * TB;
+        mbar_expect_tx(&kv_full[s], KV_BYTES);
+        tma_load_2d(st, &tmK, &kv_full[s], xq, y);
+        tma_load_2d(st + SUB, &tmK, &kv_full[s], xq + 64, y);
+        tma_load_2d(st + 2 * SUB, &tmV, &kv_full[s], xq, y);
+        tma_load_2d(st + 3 * SUB, &tmV, &kv_full[s], xq + 64, y);
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      // ---------------- MMA issuer ----------------
+      const uint32_t idesc_s = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(TB >> 3) << 17) |
+                               ((uint32_t)(TB >> 4) << 24);
+      const uint32_t idesc_pv = idesc_s | (1u << 16);  // B (V) is MN-major
+      const uint32_t qa = smem_u32(Qs), pa = smem_u32(Ps);
+      auto issue_s = [&](int j) {
+        const uint32_t ka = smem_u32(KVs + (j & 1) * KV_BYTES);
+#pragma unroll
+        for (int kk = 0; kk < 8; ++kk) {
+          const uint32_t off = (kk >> 2) * SUB + (kk & 3) * 32;
+          tc_mma_f16(tmem + (j & 1) * TB, desc_k_sw128(qa + off), desc_k_sw128(ka + off), idesc_s,
+                     kk ? 1u : 0u);
+        }
+        tc_commit(&s_full[j & 1]);
+      };
+      if (mbar_wait(q_full, 0, err) && mbar_wait(&kv_full[0], 0, err)) {
+        tc_fence_after();
+        issue_s(0);
+        for (int j = 0; j < n_kv; ++j) {
+          if (j + 1 < n_kv) {
+            if (!mbar_wait(&kv_full[(j + 1) & 1], ((j + 1) >> 1) & 1, err)) { failed = true; break; }
+            tc_fence_after();
+            issue_s(j + 1);
+          }
+          if (!mbar_wait(p_full, j & 1, err)) { failed = true; break; }
+          tc_fence_after();
+          const uint32_t va = smem_u32(KVs + (j & 1) * KV_BYTES + 2 * SUB);
+#pragma unroll
+          for (int kk = 0; kk < 8; ++kk) {
+            const uint32_t off = (kk >> 2) * SUB + (kk & 3) * 32;
+            tc_mma_f16(tmem + O_COL, desc_k_sw128(pa + off), desc_mn_sw128(va + kk * 2048, SUB),
+                       idesc_pv, (j | kk) ? 1u : 0u);
+          }
+          tc_commit(&kv_empty[j & 1]);
+          tc_commit(o_done);
+        }
+      } else {
+        failed = true;
+      }
+    }
+  } else {
+    // ---------------- softmax (warps 2..5), one query row per thread ----------------
+    const int quarter = warp & 3;
+    const int r = quarter * 32 + lane;
+    const uint32_t lane_base = tmem + ((uint32_t)(quarter * 32) << 16);
+    float m_used = -INFINITY, l = 0.f;
+    uint8_t* prow = Ps + r * 128;  // this row inside each 64-key sub-tile
+    for (int j = 0; j < n_kv && !failed; ++j) {
+      const bool ok = mbar_wait(&s_full[j & 1], (j >> 1) & 1, err);
+      if (!__all_sync(0xffffffffu, ok)) { failed = true; break; }
+      tc_fence_after();
+      float s[128];
+#pragma unroll
+      for (int c = 0; c < 4; ++c) {
+        uint32_t u[32];
+        tmem_ld32(lane_base + (j & 1) * TB + c * 32, u);
+        tmem_ld_wait();
+#pragma unroll
+        for (int i = 0; i < 32; ++i) s[c * 32 + i] = __uint_as_float(u[i]) * p.scale_log2;
+      }
+      const int valid = p.Lkv - j * TB;  // keys of this tile that exist
+      float mx = -INFINITY;
+#pragma unroll
+      for (int i = 0; i < 128; ++i) {
+        if (i >= valid) s[i] = -INFINITY;
+        mx = fmaxf(mx, s[i]);
+      }
+      if (j > 0) {
+        // PV_{j-1} must be done before P is overwritten and before O is touched
+        const bool ok2 = mbar_wait(o_done, (j - 1) & 1, err);
+        if (!__all_sync(0xffffffffu, ok2)) { failed = true; break; }
+        tc_fence_after();
+      }
+      if (j == 0) {
+        m_used = mx;
+      } else if (__any_sync(0xffffffffu, mx > m_used + 8.f)) {
+        const float m_new = fmaxf(m_used, mx);
+        const float alpha = ex2(m_used - m_new);
+        m_used = m_new;
+        l *= alpha;
+#pragma unroll 1
+        for (int c = 0; c < 4; ++c) {
+          uint32_t u[32];
+          tmem_ld32(lane_base + O_COL + c * 32, u);
+          tmem_ld_wait();
+#pragma unroll
+          for (int i = 0; i < 32; ++i) u[i] = __float_as_uint(__uint_as_float(u[i]) * alpha);
+          tmem_st32(lane_base + O_COL + c * 32, u);
+        }
+        tmem_st_wait();
+      }
+      float lsum = 0.f;
+#pragma unroll
+      for (int ch = 0; ch < 16; ++ch) {  // 16-byte chunks of 8 keys
+        float e[8];
+#pragma unroll
+        for (int q = 0; q < 8; ++q) {
+          e[q] = ex2(s[ch * 8 + q] - m_used);
+          lsum += e[q];
+        }
+        uint4 v;
+        v.x = pack_bf16x2(e[0], e[1]);
+        v.y = pack_bf16x2(e[2], e[3]);
+        v.z = pack_bf16x2(e[4], e[5]);
+        v.w = pack_bf16x2(e[6], e[7]);
+        const int sub = ch >> 3, c16 = (ch & 7) ^ (r & 7);
+        *reinterpret_cast<uint4*>(prow + sub * SUB + c16 * 16) = v;
+      }
+      l += lsum;
+      fence_async_smem();  // P visible to the tensor core (async proxy)
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(p_full);
+    }
+    if (!failed) {
+      const bool ok = mbar_wait(o_done, (n_kv - 1) & 1, err);
+      if (__all_sync(0xffffffffu, ok)) {
+        tc_fence_after();
+        const float inv = 1.f / l;
+        const int qrow = qt * TB + r;
+        bf16* orow = p.O + (size_t)q_row0 * p.ldo + (size_t)r * p.ldo + h * 128;
+#pragma unroll 1
+        for (int c = 0; c < 4; ++c) {
+          uint32_t u[32];
+          tmem_ld32(lane_base + O_COL + c * 32, u);
+          tmem_ld_wait();
+          if (qrow < p.Lq) {
+#pragma unroll
+            for (int g = 0; g < 4; ++g) {
+              float v[8];
+#pragma unroll
+              for (int i = 0; i < 8; ++i) v[i] = __uint_as_float(u[g * 8 + i]) * inv;
+              store_bf16x8(orow + c * 32 + g * 8, v);
+            }
+          }
+        }
+      } else {
+        failed = true;
+      }
+    }
+  }
+
+  if (failed || *(volatile int*)err != 0) {
+    const uint64_t t0 = fb_globaltimer();  // let in-flight TMA loads land
+    while (fb_globaltimer() - t0 < 100000ull) __nanosleep(1000);
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, TMEM_COLS);
+  }
+}
+
+PFN_cuTensorMapEncodeTiled_v12000 encoder() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  if (!fn) {
+    cudaDriverEntryPointQueryResult q;
+    void* f = nullptr;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &f, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(f);
+  }
+  return fn;
+}
+
+bool map_128x64(CUtensorMap* m, const bf16* ptr, int rows, int cols, int ld) {
+  auto enc = encoder();
+  if (!enc) return false;
+  cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
+  cuuint64_t strides[1] = {(cuuint64_t)ld * sizeof(bf16)};
+  cuuint32_t box[2] = {64, (cuuint32_t)TB};
+  cuuint32_t estr[2] = {1, 1};
+  return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<bf16*>(ptr), dims, strides, box,
+             estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+}  // namespace
+
+bool attention_tc_supported(const AttnArgs& a) {
+  auto al16 = [](const void* q) { return (reinterpret_cast<uintptr_t>(q) & 15) == 0; };
+  return a.head_dim == 128 && a.Lq >= 1 && a.Lkv >= 1 && a.batch >= 1 && a.ldq % 8 == 0 &&
+         a.ldk % 8 == 0 && a.ldv % 8 == 0 && a.ldo % 8 == 0 && al16(a.Q) && al16(a.K) &&
+         al16(a.V) && al16(a.O);
+}
+
+cudaError_t attention_tc(const AttnArgs& a, int* err, cudaStream_t st) {
+  if (!attention_tc_supported(a)) return cudaErrorInvalidValue;
+  const int cols = a.heads * 128;
+  const int kv_rows = a.kv_batch_rows ? (a.batch - 1) * a.kv_batch_rows + a.Lkv : a.Lkv;
+  CUtensorMap mq, mk, mv;
+  if (!map_128x64(&mq, a.Q, a.batch * a.Lq, cols, a.ldq) ||
+      !map_128x64(&mk, a.K, kv_rows, cols, a.ldk) || !map_128x64(&mv, a.V, kv_rows, cols, a.ldv))
+    return cudaErrorInvalidValue;
+  cudaError_t e = cudaFuncSetAttribute(attn_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       SMEM_BYTES);
+  if (e != cudaSuccess) return e;
+  Params p;
+  p.Lq = a.Lq;
+  p.Lkv = a.Lkv;
+  p.kv_batch_rows = a.kv_batch_rows;
+  p.O = a.O;
+  p.ldo = a.ldo;
+  p.scale_log2 = 1.4426950408889634f / sqrtf(128.f);
+  p.err = err;
+  dim3 grid((a.Lq + TB - 1) / TB, a.heads, a.batch);
+  attn_tc_kernel<<<grid, THREADS, SMEM_BYTES, st>>>(mq, mk, mv, p);
+  return cudaGetLastError();
+}

@@ -55,9 +55,16 @@ __device__ __forceinline__ void store_f32x8(float* p, const float* v) {
   *reinterpret_cast<float4*>(p + 4) = make_float4(v[4], v[5], v[6], v[7]);
 }
 
+__device__ __forceinline__ float tanh_approx(float x) {
+  float y;
+  asm("tanh.approx.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+// GELU, tanh form. The hardware tanh (max relative error about 2^-11) is well inside
+// the bf16 rounding of the GEMM output that it feeds.
 __device__ __forceinline__ float gelu_tanh_f(float x) {
   const float k0 = 0.7978845608028654f;  // sqrt(2/pi)
-  return 0.5f * x * (1.f + tanhf(k0 * (x + 0.044715f * x * x * x)));
+  return 0.5f * x * (1.f + tanh_approx(k0 * (x + 0.044715f * x * x * x)));
 }
 __device__ __forceinline__ float silu_f(float x) { return x / (1.f + expf(-x)); }
 
@@ -244,6 +251,55 @@ struct GemmEpi {
   bf16* delta;         // bf16 [M][ldo] (EPI_RESID_DELTA)
   int ldo;
 };
+
+// Applies the epilogue to 32 consecutive accumulators v of row `row`, columns
+// col..col+31. Every global load of the chunk is issued before its first store (out may
+// alias resid / base element for element, so this order is safe), which keeps 32 B x 12
+// loads in flight per thread instead of serialising load -> store per 8 columns.
+template <int KIND>
+__device__ __forceinline__ void epi_apply32(const GemmEpi& e, int row, int col, float* v) {
+  const size_t off = (size_t)row * e.ldo + col;
+  if (KIND >= EPI_RESID) {
+    float r[32], g[32], b[32], bs[32];
+#pragma unroll
+    for (int j = 0; j < 32; j += 8) {
+      load_f32x8(e.resid + off + j, r + j);
+      if (e.gate) load_f32x8(e.gate + col + j, g + j);
+      if (e.bias) load_f32x8(e.bias + col + j, b + j);
+      if (KIND == EPI_RESID_DELTA) load_f32x8(e.base + off + j, bs + j);
+    }
+#pragma unroll
+    for (int j = 0; j < 32; ++j) {
+      const float a = v[j] + (e.bias ? b[j] : 0.f);
+      v[j] = r[j] + (e.gate ? g[j] : 1.f) * a;
+    }
+    if (KIND == EPI_RESID_DELTA) {
+#pragma unroll
+      for (int j = 0; j < 32; j += 8) {
+        float d[8];
+#pragma unroll
+        for (int q = 0; q < 8; ++q) d[q] = v[j + q] - bs[j + q];
+        store_bf16x8(e.delta + off + j, d);
+      }
+    }
+#pragma unroll
+    for (int j = 0; j < 32; j += 8) store_f32x8(reinterpret_cast<float*>(e.out) + off + j, v + j);
+  } else {
+    if (e.bias) {
+      float b[32];
+#pragma unroll
+      for (int j = 0; j < 32; j += 8) load_f32x8(e.bias + col + j, b + j);
+#pragma unroll
+      for (int j = 0; j < 32; ++j) v[j] += b[j];
+    }
+    if (KIND == EPI_GELU_BF16) {
+#pragma unroll
+      for (int j = 0; j < 32; ++j) v[j] = gelu_tanh_f(v[j]);
+    }
+#pragma unroll
+    for (int j = 0; j < 32; j += 8) store_bf16x8(reinterpret_cast<bf16*>(e.out) + off + j, v + j);
+  }
+}
 
 // Applies the epilogue to 8 consecutive accumulators v of row `row`, columns col..col+7.
 template <int KIND>

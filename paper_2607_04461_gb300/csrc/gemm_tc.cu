@@ -179,13 +179,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         tmem_ld32(taddr + c * 32, r);
         tmem_ld_wait();
         if (row < M) {
+          float v[32];
 #pragma unroll
-          for (int g = 0; g < 4; ++g) {
-            float v[8];
-#pragma unroll
-            for (int j = 0; j < 8; ++j) v[j] = __uint_as_float(r[g * 8 + j]);
-            epi_apply8<KIND>(epi, row, n0 + c * 32 + g * 8, v);
-          }
+          for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(r[j]);
+          epi_apply32<KIND>(epi, row, n0 + c * 32, v);
         }
       }
       tc_fence_before();
@@ -322,13 +319,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
         tmem_ld32(taddr + c * 32, r);
         tmem_ld_wait();
         if (row < M) {
+          float v[32];
 #pragma unroll
-          for (int g = 0; g < 4; ++g) {
-            float v[8];
-#pragma unroll
-            for (int j = 0; j < 8; ++j) v[j] = __uint_as_float(r[g * 8 + j]);
-            epi_apply8<KIND>(epi, row, n0 + c * 32 + g * 8, v);
-          }
+          for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(r[j]);
+          epi_apply32<KIND>(epi, row, n0 + c * 32, v);
         }
       }
       tc_fence_before();

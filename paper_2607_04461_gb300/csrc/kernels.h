@@ -34,7 +34,11 @@ struct AttnArgs {
   int kv_batch_rows;       // row offset of batch b's K/V (0 = shared)
   int heads, head_dim;
 };
+// mma.sync (warp-level) kernel: head_dim 64 or 128.
 cudaError_t attention(const AttnArgs& a, cudaStream_t st);
+// tcgen05/TMEM kernel: head_dim 128, 16-byte aligned rows.
+bool attention_tc_supported(const AttnArgs& a);
+cudaError_t attention_tc(const AttnArgs& a, int* err, cudaStream_t st);
 
 // ---- pointwise / small kernels ------------------------------------------------------
 // out[r][:] = bf16(LN(x[r][:]) * (mul_base + mul[:]) + add[:]), x fp32 [rows][D].

@@ -204,22 +204,23 @@ __global__ void __launch_bounds__(256) patch_embed_kernel(const float* __restric
 
 // ---------------------------------------------------------------------------------
 // head_euler: 32 tokens per CTA, 256 threads; K staged through shared memory in
-// chunks of 128. Thread -> output o = tid % PD, tokens (tid / PD) * TPT .. + TPT - 1.
+// chunks of 128. Thread -> output o = tid % PD and TPT = 32 PD / 256 consecutive tokens.
 constexpr int HE_TOK = 32, HE_KC = 128;
+template <int PD>
 __global__ void __launch_bounds__(256) head_euler_kernel(const bf16* __restrict__ a, int n,
                                                          int C, int H, int W, int p,
                                                          const bf16* __restrict__ Wh,
                                                          const float* __restrict__ bh, int D,
                                                          float dt, float* __restrict__ z) {
+  constexpr int TPT = HE_TOK * PD / 256;
   __shared__ float as[HE_TOK][HE_KC + 1];
-  __shared__ float ws[64][HE_KC + 1];
-  const int PD = C * p * p, gw = W / p, P = (H / p) * gw, M = n * P;
+  __shared__ float ws[PD][HE_KC + 1];
+  const int gw = W / p, P = (H / p) * gw, M = n * P;
   const int tok0 = blockIdx.x * HE_TOK;
   const int o = threadIdx.x % PD, grp = threadIdx.x / PD;
-  const int TPT = HE_TOK * PD / 256;  // tokens per thread (PD in {8,...,64}, PD | 256)
-  float acc[32];
+  float acc[TPT];
 #pragma unroll
-  for (int i = 0; i < 32; ++i) acc[i] = 0.f;
+  for (int i = 0; i < TPT; ++i) acc[i] = 0.f;
   for (int k0 = 0; k0 < D; k0 += HE_KC) {
     __syncthreads();
     for (int i = threadIdx.x; i < HE_TOK * HE_KC / 8; i += 256) {
@@ -237,22 +238,23 @@ __global__ void __launch_bounds__(256) head_euler_kernel(const bf16* __restrict_
       for (int j = 0; j < 8; ++j) ws[r][kc + j] = v[j];
     }
     __syncthreads();
-    if (grp * TPT < HE_TOK) {
-      for (int k = 0; k < HE_KC; ++k) {
-        const float wv = ws[o][k];
-        for (int i = 0; i < TPT; ++i) acc[i] += wv * as[grp * TPT + i][k];
-      }
+#pragma unroll 4
+    for (int k = 0; k < HE_KC; ++k) {
+      const float wv = ws[o][k];
+#pragma unroll
+      for (int i = 0; i < TPT; ++i) acc[i] += wv * as[grp * TPT + i][k];
     }
   }
-  if (grp * TPT >= HE_TOK) return;
   const float bias = bh[o];
   const int ch = o / (p * p), dy = (o / p) % p, dx = o % p;
+#pragma unroll
   for (int i = 0; i < TPT; ++i) {
     const int tok = tok0 + grp * TPT + i;
-    if (tok >= M) break;
-    const int b = tok / P, pt = tok % P, r = pt / gw, cc = pt % gw;
-    float* zp = z + (((size_t)b * C + ch) * H + r * p + dy) * W + cc * p + dx;
-    *zp += dt * (acc[i] + bias);
+    if (tok < M) {
+      const int b = tok / P, pt = tok % P, r = pt / gw, cc = pt % gw;
+      float* zp = z + (((size_t)b * C + ch) * H + r * p + dy) * W + cc * p + dx;
+      *zp += dt * (acc[i] + bias);
+    }
   }
 }
 
@@ -380,8 +382,15 @@ cudaError_t head_euler(const bf16* a, int n, int C, int H, int W, int p, const b
                        const float* bh, int D, float dt, float* z, cudaStream_t st) {
   const int PD = C * p * p, M = n * (H / p) * (W / p);
   if (M == 0) return cudaSuccess;
-  if (PD % 8 || PD > 64 || 256 % PD || D % 8) return cudaErrorInvalidValue;
-  head_euler_kernel<<<(M + HE_TOK - 1) / HE_TOK, 256, 0, st>>>(a, n, C, H, W, p, Wh, bh, D, dt, z);
+  if (D % 8) return cudaErrorInvalidValue;
+  const int grid = (M + HE_TOK - 1) / HE_TOK;
+  switch (PD) {
+    case 8: head_euler_kernel<8><<<grid, 256, 0, st>>>(a, n, C, H, W, p, Wh, bh, D, dt, z); break;
+    case 16: head_euler_kernel<16><<<grid, 256, 0, st>>>(a, n, C, H, W, p, Wh, bh, D, dt, z); break;
+    case 32: head_euler_kernel<32><<<grid, 256, 0, st>>>(a, n, C, H, W, p, Wh, bh, D, dt, z); break;
+    case 64: head_euler_kernel<64><<<grid, 256, 0, st>>>(a, n, C, H, W, p, Wh, bh, D, dt, z); break;
+    default: return cudaErrorInvalidValue;
+  }
   return cudaGetLastError();
 }
 

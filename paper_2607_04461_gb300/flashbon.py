@@ -76,7 +76,7 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
         "fb_reset_stats": (I, [P]),
         "fb_kernel_name": (ctypes.c_char_p, [I]),
         "fb_op_gemm": (I, [P, I, I, I, P, P, P, I, P, P, P, P, P, I]),
-        "fb_op_attention": (I, [P, P, I, P, I, P, I, P, I, I, I, I, I, I, I]),
+        "fb_op_attention": (I, [P, P, I, P, I, P, I, P, I, I, I, I, I, I, I, I]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(L, name)
@@ -216,10 +216,10 @@ def fb_op_gemm(model, M, N, K, A, W, bias, epi, out, resid=None, gate=None, base
 
 
 def fb_op_attention(model, Q, ldq, Kt, ldk, V, ldv, O, ldo, batch, Lq, Lkv, kv_batch_rows,
-                    heads, head_dim) -> None:
+                    heads, head_dim, impl=0) -> None:
     _check(load_library().fb_op_attention(model, _ptr(Q), ldq, _ptr(Kt), ldk, _ptr(V), ldv,
                                           _ptr(O), ldo, batch, Lq, Lkv, kv_batch_rows, heads,
-                                          head_dim))
+                                          head_dim, impl))
 
 
 class Model:

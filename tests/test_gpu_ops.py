@@ -112,11 +112,33 @@ ATTN_CASES = [
     (1, 1, 1, 1, 128, False),
     (2, 1560, 512, 2, 128, True),
     (1, 200, 333, 2, 64, False),
+    (2, 1560, 1560, 2, 128, False),   # Wan2.1 self-attention length, ragged last tile
+    (3, 256, 128, 1, 128, False),     # exact tile multiples
+    (2, 129, 257, 2, 128, True),      # one row / one key past a tile
 ]
 
 
+def test_attention_large_logits(model):
+    """Scores spanning many powers of two exercise the rescaling of O."""
+    batch, L, heads, dh = 2, 400, 2, 128
+    D = heads * dh
+    q = randn((batch * L, D), 41, scale=4.0)
+    k = randn((batch * L, D), 42, scale=4.0)
+    v = randn((batch * L, D), 43)
+    o = torch.empty((batch * L, D), dtype=torch.bfloat16, device="cuda")
+    fb.fb_op_attention(model.handle, q, D, k, D, v, D, o, D, batch, L, L, L, heads, dh)
+    torch.cuda.synchronize()
+    qn, kn, vn, on = f64(q), f64(k), f64(v), f64(o)
+    for b in range(batch):
+        sl = slice(b * L, (b + 1) * L)
+        want = O.attention(qn[sl].reshape(L, heads, dh), kn[sl].reshape(L, heads, dh),
+                           vn[sl].reshape(L, heads, dh)).reshape(L, D)
+        assert rel_max(on[sl], want) <= 2e-2
+
+
+@pytest.mark.parametrize("impl", [0, 1], ids=["auto", "mma_sync"])
 @pytest.mark.parametrize("batch,Lq,Lkv,heads,dh,shared", ATTN_CASES)
-def test_attention(model, batch, Lq, Lkv, heads, dh, shared):
+def test_attention(model, batch, Lq, Lkv, heads, dh, shared, impl):
     D = heads * dh
     q = randn((batch * Lq, D), 21)
     kvb = 1 if shared else batch
@@ -124,7 +146,7 @@ def test_attention(model, batch, Lq, Lkv, heads, dh, shared):
     v = randn((kvb * Lkv, D), 23)
     o = torch.empty((batch * Lq, D), dtype=torch.bfloat16, device="cuda")
     fb.fb_op_attention(model.handle, q, D, k, D, v, D, o, D, batch, Lq, Lkv,
-                       0 if shared else Lkv, heads, dh)
+                       0 if shared else Lkv, heads, dh, impl)
     torch.cuda.synchronize()
     qn, kn, vn, on = f64(q), f64(k), f64(v), f64(o)
     for b in range(batch):
