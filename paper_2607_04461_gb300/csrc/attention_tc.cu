@@ -305,6 +305,247 @@ __global__ void __launch_bounds__(THREADS, 1)
   }
 }
 
+// ---- two query tiles per CTA ---------------------------------------------------------
+// Same computation with 256 queries per CTA: tiles A and B share every K/V tile (half
+// the K/V traffic per FLOP). P is written back into the TMEM columns of its S tile
+// (bf16 pairs) and read from there as the A operand of the PV MMA, so shared memory only
+// holds Q_A, Q_B and the K/V ring. TMEM: S_A|P_A [0,128), S_B|P_B [128,256), O_A
+// [256,384), O_B [384,512). MMA order per KV tile j: PV_A(j), S_A(j+1), PV_B(j), S_B(j+1),
+// so each softmax group works while the tensor core runs the other group's MMAs.
+// tcgen05 operations of one thread execute in order, so S_A(j+1) overwrites P_A(j) only
+// after PV_A(j) has read it, and the commit that announces S_g(j+1) also covers PV_g(j)
+// (the softmax may then rescale O_g).
+constexpr int THREADS2 = 320;
+constexpr int SMEM2_BYTES = 2 * Q_BYTES + NSTAGE * KV_BYTES + 1024 + 256;
+
+__device__ __forceinline__ void tc_mma_f16_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t bdesc,
+                                              uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "r"(a_tmem), "l"(bdesc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
+__global__ void __launch_bounds__(THREADS2, 1)
+    attn_tc2_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
+                    const __grid_constant__ CUtensorMap tmV, Params p) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint8_t* Qs = smem;                  // [2 tiles][2 sub-tiles]
+  uint8_t* KVs = smem + 2 * Q_BYTES;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(KVs + NSTAGE * KV_BYTES);
+  uint64_t* q_full = bars;
+  uint64_t* kv_full = bars + 1;        // [2]
+  uint64_t* kv_empty = bars + 3;       // [2]
+  uint64_t* s_full = bars + 5;         // [2 groups]
+  uint64_t* p_full = bars + 7;         // [2 groups]
+  uint64_t* o_done = bars + 9;
+  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(bars + 10);
+
+  const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+  const int qb = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
+  const int q_row0 = b * p.Lq + qb * 2 * TB;
+  const int kv_row0 = b * p.kv_batch_rows;
+  const int n_kv = (p.Lkv + TB - 1) / TB;
+  int* err = p.err;
+  bool failed = false;
+
+  if (threadIdx.x == 0) {
+    mbar_init(q_full, 1);
+    for (int s = 0; s < 2; ++s) {
+      mbar_init(&kv_full[s], 1);
+      mbar_init(&kv_empty[s], 1);
+      mbar_init(&s_full[s], 1);
+      mbar_init(&p_full[s], 4);
+    }
+    mbar_init(o_done, 1);
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    tma_prefetch_desc(&tmQ);
+    tma_prefetch_desc(&tmK);
+    tma_prefetch_desc(&tmV);
+  }
+  if (warp == 1) tmem_alloc(tmem_holder, TMEM_COLS);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_holder;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      const int xq = h * 128;
+      mbar_expect_tx(q_full, 2 * Q_BYTES);
+      for (int g = 0; g < 2; ++g) {
+        tma_load_2d(Qs + g * Q_BYTES, &tmQ, q_full, xq, q_row0 + g * TB);
+        tma_load_2d(Qs + g * Q_BYTES + SUB, &tmQ, q_full, xq + 64, q_row0 + g * TB);
+      }
+      for (int j = 0; j < n_kv; ++j) {
+        const int s = j & 1;
+        if (!mbar_wait(&kv_empty[s], ((j >> 1) & 1) ^ 1u, err)) { failed = true; break; }
+        uint8_t* st = KVs + s * KV_BYTES;
+        const int y = kv_row0 + j * TB;
+        mbar_expect_tx(&kv_full[s], KV_BYTES);
+        tma_load_2d(st, &tmK, &kv_full[s], xq, y);
+        tma_load_2d(st + SUB, &tmK, &kv_full[s], xq + 64, y);
+        tma_load_2d(st + 2 * SUB, &tmV, &kv_full[s], xq, y);
+        tma_load_2d(st + 3 * SUB, &tmV, &kv_full[s], xq + 64, y);
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      const uint32_t idesc_s = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(TB >> 3) << 17) |
+                               ((uint32_t)(TB >> 4) << 24);
+      const uint32_t idesc_pv = idesc_s | (1u << 16);
+      const uint32_t qa = smem_u32(Qs);
+      auto issue_s = [&](int g, int j) {
+        const uint32_t ka = smem_u32(KVs + (j & 1) * KV_BYTES);
+        const uint32_t qg = qa + g * Q_BYTES;
+#pragma unroll
+        for (int kk = 0; kk < 8; ++kk) {
+          const uint32_t off = (kk >> 2) * SUB + (kk & 3) * 32;
+          tc_mma_f16(tmem + g * TB, desc_k_sw128(qg + off), desc_k_sw128(ka + off), idesc_s,
+                     kk ? 1u : 0u);
+        }
+        tc_commit(&s_full[g]);
+      };
+      auto issue_pv = [&](int g, int j) {
+        const uint32_t va = smem_u32(KVs + (j & 1) * KV_BYTES + 2 * SUB);
+#pragma unroll
+        for (int kk = 0; kk < 8; ++kk)
+          tc_mma_f16_ts(tmem + O_COL + g * TB, tmem + g * TB + kk * 8,
+                        desc_mn_sw128(va + kk * 2048, SUB), idesc_pv, (j | kk) ? 1u : 0u);
+      };
+      bool ok = mbar_wait(q_full, 0, err) && mbar_wait(&kv_full[0], 0, err);
+      if (ok) {
+        tc_fence_after();
+        issue_s(0, 0);
+        issue_s(1, 0);
+        for (int j = 0; j < n_kv && ok; ++j) {
+          const bool more = j + 1 < n_kv;
+          if (!(ok = mbar_wait(&p_full[0], j & 1, err))) break;
+          tc_fence_after();
+          issue_pv(0, j);
+          if (more) {
+            if (!(ok = mbar_wait(&kv_full[(j + 1) & 1], ((j + 1) >> 1) & 1, err))) break;
+            tc_fence_after();
+            issue_s(0, j + 1);
+          }
+          if (!(ok = mbar_wait(&p_full[1], j & 1, err))) break;
+          tc_fence_after();
+          issue_pv(1, j);
+          tc_commit(&kv_empty[j & 1]);
+          if (more) issue_s(1, j + 1);
+        }
+        if (ok) tc_commit(o_done);
+      }
+      failed = !ok;
+    }
+  } else {
+    // ---------------- softmax groups: warps 2-5 -> tile A, warps 6-9 -> tile B ----------
+    const int g = (warp - 2) >> 2;
+    const int quarter = warp & 3;
+    const int r = quarter * 32 + lane;
+    const uint32_t lane_base = tmem + ((uint32_t)(quarter * 32) << 16);
+    const uint32_t s_col = g * TB, o_col = O_COL + g * TB;
+    float m_used = -INFINITY, l = 0.f;
+    for (int j = 0; j < n_kv && !failed; ++j) {
+      const bool ok = mbar_wait(&s_full[g], j & 1, err);
+      if (!__all_sync(0xffffffffu, ok)) { failed = true; break; }
+      tc_fence_after();
+      float s[128];
+#pragma unroll
+      for (int c = 0; c < 4; ++c) {
+        uint32_t u[32];
+        tmem_ld32(lane_base + s_col + c * 32, u);
+        tmem_ld_wait();
+#pragma unroll
+        for (int i = 0; i < 32; ++i) s[c * 32 + i] = __uint_as_float(u[i]) * p.scale_log2;
+      }
+      const int valid = p.Lkv - j * TB;
+      float mx = -INFINITY;
+#pragma unroll
+      for (int i = 0; i < 128; ++i) {
+        if (i >= valid) s[i] = -INFINITY;
+        mx = fmaxf(mx, s[i]);
+      }
+      if (j == 0) {
+        m_used = mx;
+      } else if (__any_sync(0xffffffffu, mx > m_used + 8.f)) {
+        const float m_new = fmaxf(m_used, mx);
+        const float alpha = ex2(m_used - m_new);
+        m_used = m_new;
+        l *= alpha;
+#pragma unroll 1
+        for (int c = 0; c < 4; ++c) {
+          uint32_t u[32];
+          tmem_ld32(lane_base + o_col + c * 32, u);
+          tmem_ld_wait();
+#pragma unroll
+          for (int i = 0; i < 32; ++i) u[i] = __float_as_uint(__uint_as_float(u[i]) * alpha);
+          tmem_st32(lane_base + o_col + c * 32, u);
+        }
+      }
+      float lsum = 0.f;
+#pragma unroll
+      for (int c = 0; c < 2; ++c) {
+        uint32_t u[32];
+#pragma unroll
+        for (int i = 0; i < 32; ++i) {
+          const float e0 = ex2(s[c * 64 + 2 * i] - m_used);
+          const float e1 = ex2(s[c * 64 + 2 * i + 1] - m_used);
+          lsum += e0 + e1;
+          u[i] = pack_bf16x2(e0, e1);
+        }
+        tmem_st32(lane_base + s_col + c * 32, u);
+      }
+      l += lsum;
+      tmem_st_wait();
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&p_full[g]);
+    }
+    if (!failed) {
+      const bool ok = mbar_wait(o_done, 0, err);
+      if (__all_sync(0xffffffffu, ok)) {
+        tc_fence_after();
+        const float inv = 1.f / l;
+        const int qrow = qb * 2 * TB + g * TB + r;
+        bf16* orow = p.O + (size_t)(q_row0 + g * TB + r) * p.ldo + h * 128;
+#pragma unroll 1
+        for (int c = 0; c < 4; ++c) {
+          uint32_t u[32];
+          tmem_ld32(lane_base + o_col + c * 32, u);
+          tmem_ld_wait();
+          if (qrow < p.Lq) {
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+              float v[8];
+#pragma unroll
+              for (int i = 0; i < 8; ++i) v[i] = __uint_as_float(u[q * 8 + i]) * inv;
+              store_bf16x8(orow + c * 32 + q * 8, v);
+            }
+          }
+        }
+      } else {
+        failed = true;
+      }
+    }
+  }
+
+  if (failed || *(volatile int*)err != 0) {
+    const uint64_t t0 = fb_globaltimer();
+    while (fb_globaltimer() - t0 < 100000ull) __nanosleep(1000);
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, TMEM_COLS);
+  }
+}
+
 PFN_cuTensorMapEncodeTiled_v12000 encoder() {
   static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
   if (!fn) {
@@ -347,9 +588,9 @@ cudaError_t attention_tc(const AttnArgs& a, int* err, cudaStream_t st) {
   if (!map_128x64(&mq, a.Q, a.batch * a.Lq, cols, a.ldq) ||
       !map_128x64(&mk, a.K, kv_rows, cols, a.ldk) || !map_128x64(&mv, a.V, kv_rows, cols, a.ldv))
     return cudaErrorInvalidValue;
-  cudaError_t e = cudaFuncSetAttribute(attn_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       SMEM_BYTES);
-  if (e != cudaSuccess) return e;
+  int dev = 0, sms = 148;
+  if (cudaGetDevice(&dev) == cudaSuccess)
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
   Params p;
   p.Lq = a.Lq;
   p.Lkv = a.Lkv;
@@ -358,7 +599,21 @@ cudaError_t attention_tc(const AttnArgs& a, int* err, cudaStream_t st) {
   p.ldo = a.ldo;
   p.scale_log2 = 1.4426950408889634f / sqrtf(128.f);
   p.err = err;
-  dim3 grid((a.Lq + TB - 1) / TB, a.heads, a.batch);
-  attn_tc_kernel<<<grid, THREADS, SMEM_BYTES, st>>>(mq, mk, mv, p);
+  // 256-query CTAs share each K/V tile between two query tiles; with fewer than two
+  // such CTAs per SM the 128-query kernel keeps more SMs busy.
+  const long ctas2 = (long)((a.Lq + 2 * TB - 1) / (2 * TB)) * a.heads * a.batch;
+  if (ctas2 >= 2L * sms) {
+    cudaError_t e = cudaFuncSetAttribute(attn_tc2_kernel,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM2_BYTES);
+    if (e != cudaSuccess) return e;
+    dim3 grid((a.Lq + 2 * TB - 1) / (2 * TB), a.heads, a.batch);
+    attn_tc2_kernel<<<grid, THREADS2, SMEM2_BYTES, st>>>(mq, mk, mv, p);
+  } else {
+    cudaError_t e = cudaFuncSetAttribute(attn_tc_kernel,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
+    if (e != cudaSuccess) return e;
+    dim3 grid((a.Lq + TB - 1) / TB, a.heads, a.batch);
+    attn_tc_kernel<<<grid, THREADS, SMEM_BYTES, st>>>(mq, mk, mv, p);
+  }
   return cudaGetLastError();
 }

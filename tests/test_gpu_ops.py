@@ -115,6 +115,9 @@ ATTN_CASES = [
     (2, 1560, 1560, 2, 128, False),   # Wan2.1 self-attention length, ragged last tile
     (3, 256, 128, 1, 128, False),     # exact tile multiples
     (2, 129, 257, 2, 128, True),      # one row / one key past a tile
+    # grids of >= 2 CTAs per SM take the 256-query kernel (P kept in TMEM)
+    (4, 1560, 1560, 12, 128, False),
+    (9, 600, 512, 12, 128, True),     # last CTA: tile A partly valid, tile B past Lq
 ]
 
 
