@@ -13,6 +13,7 @@
 #include <cmath>
 #include <cstdarg>
 #include <cstdio>
+#include <cstdlib>
 #include <cstring>
 #include <map>
 #include <string>
@@ -20,6 +21,11 @@
 
 #include "../../include/flashbon.h"
 #include "kernels.h"
+
+bool fb_pdl_enabled() {
+  static const bool on = getenv("FB_NO_PDL") == nullptr;
+  return on;
+}
 
 namespace {
 

@@ -63,6 +63,8 @@ __device__ __forceinline__ void load_tile(bf16* tile, const bf16* base, int ld, 
 
 template <int DH>
 __global__ void __launch_bounds__(NT) flash_attn_kernel(AttnArgs a, float scale_log2) {
+  griddep_wait();
+  griddep_launch();
   extern __shared__ __align__(128) uint8_t smem_raw[];
   bf16* Qs = reinterpret_cast<bf16*>(smem_raw);
   bf16* Ks = Qs + BQ * DH;        // [2][BKV][DH]
@@ -212,7 +214,8 @@ cudaError_t launch(const AttnArgs& a, cudaStream_t st) {
   if (e != cudaSuccess) return e;
   dim3 grid((a.Lq + BQ - 1) / BQ, a.heads, a.batch);
   const float scale_log2 = 1.4426950408889634f / sqrtf((float)DH);
-  flash_attn_kernel<DH><<<grid, NT, smem, st>>>(a, scale_log2);
+  cudaError_t le = launch_k(flash_attn_kernel<DH>, grid, dim3(NT), smem, st, a, scale_log2);
+  if (le != cudaSuccess) return le;
   return cudaGetLastError();
 }
 }  // namespace

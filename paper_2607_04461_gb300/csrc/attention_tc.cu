@@ -129,6 +129,8 @@ __global__ void __launch_bounds__(THREADS, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_holder;
+  griddep_wait();
+  griddep_launch();
 
   if (warp == 0) {
     if (lane == 0) {
@@ -372,6 +374,8 @@ __global__ void __launch_bounds__(THREADS2, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_holder;
+  griddep_wait();
+  griddep_launch();
 
   if (warp == 0) {
     if (lane == 0) {
@@ -607,13 +611,15 @@ cudaError_t attention_tc(const AttnArgs& a, int* err, cudaStream_t st) {
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM2_BYTES);
     if (e != cudaSuccess) return e;
     dim3 grid((a.Lq + 2 * TB - 1) / (2 * TB), a.heads, a.batch);
-    attn_tc2_kernel<<<grid, THREADS2, SMEM2_BYTES, st>>>(mq, mk, mv, p);
+    e = launch_k(attn_tc2_kernel, grid, dim3(THREADS2), SMEM2_BYTES, st, mq, mk, mv, p);
+    if (e != cudaSuccess) return e;
   } else {
     cudaError_t e = cudaFuncSetAttribute(attn_tc_kernel,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
     if (e != cudaSuccess) return e;
     dim3 grid((a.Lq + TB - 1) / TB, a.heads, a.batch);
-    attn_tc_kernel<<<grid, THREADS, SMEM_BYTES, st>>>(mq, mk, mv, p);
+    e = launch_k(attn_tc_kernel, grid, dim3(THREADS), SMEM_BYTES, st, mq, mk, mv, p);
+    if (e != cudaSuccess) return e;
   }
   return cudaGetLastError();
 }

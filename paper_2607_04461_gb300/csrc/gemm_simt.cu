@@ -10,6 +10,8 @@ template <int KIND>
 __global__ void __launch_bounds__(256) gemm_simt_kernel(const bf16* __restrict__ A, int lda,
                                                         const bf16* __restrict__ W, int ldw,
                                                         int M, int N, int K, GemmEpi epi) {
+  griddep_wait();
+  griddep_launch();
   __shared__ float As[TK][TM + 1];
   __shared__ float Ws[TK][TN + 1];
   const int tid = threadIdx.x;
@@ -52,19 +54,18 @@ cudaError_t gemm_simt(const GemmArgs& g, cudaStream_t st) {
   dim3 grid((g.N + TN - 1) / TN, (g.M + TM - 1) / TM);
   switch (g.kind) {
     case EPI_BF16:
-      gemm_simt_kernel<EPI_BF16><<<grid, 256, 0, st>>>(g.A, g.lda, g.W, g.ldw, g.M, g.N, g.K, g.epi);
+      return launch_k(gemm_simt_kernel<EPI_BF16>, grid, dim3(256), 0, st, g.A, g.lda, g.W, g.ldw, g.M, g.N, g.K, g.epi);
       break;
     case EPI_GELU_BF16:
-      gemm_simt_kernel<EPI_GELU_BF16><<<grid, 256, 0, st>>>(g.A, g.lda, g.W, g.ldw, g.M, g.N, g.K, g.epi);
+      return launch_k(gemm_simt_kernel<EPI_GELU_BF16>, grid, dim3(256), 0, st, g.A, g.lda, g.W, g.ldw, g.M, g.N, g.K, g.epi);
       break;
     case EPI_RESID:
-      gemm_simt_kernel<EPI_RESID><<<grid, 256, 0, st>>>(g.A, g.lda, g.W, g.ldw, g.M, g.N, g.K, g.epi);
+      return launch_k(gemm_simt_kernel<EPI_RESID>, grid, dim3(256), 0, st, g.A, g.lda, g.W, g.ldw, g.M, g.N, g.K, g.epi);
       break;
     case EPI_RESID_DELTA:
-      gemm_simt_kernel<EPI_RESID_DELTA><<<grid, 256, 0, st>>>(g.A, g.lda, g.W, g.ldw, g.M, g.N, g.K, g.epi);
+      return launch_k(gemm_simt_kernel<EPI_RESID_DELTA>, grid, dim3(256), 0, st, g.A, g.lda, g.W, g.ldw, g.M, g.N, g.K, g.epi);
       break;
     default:
       return cudaErrorInvalidValue;
   }
-  return cudaGetLastError();
 }

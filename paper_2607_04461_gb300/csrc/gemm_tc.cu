@@ -94,6 +94,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_holder;
+  griddep_wait();  // inputs written by the previous kernel are visible from here on
+  griddep_launch();
 
   if (warp == 0) {
     if (lane == 0) {
@@ -252,6 +254,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
   cluster_sync();  // both CTAs' barriers initialised, TMEM allocated
   tc_fence_after();
   const uint32_t tmem_base = *tmem_holder;
+  griddep_wait();
+  griddep_launch();
 
   if (warp == 0) {
     if (lane == 0) {
@@ -384,9 +388,8 @@ cudaError_t launch(const GemmArgs& g, int* err, int num_sms, cudaStream_t st) {
   if (e != cudaSuccess) return e;
   const int tiles = ((g.M + BM - 1) / BM) * (g.N / BN);
   const int grid = tiles < num_sms ? tiles : num_sms;
-  gemm_tc_kernel<BN, KIND><<<grid, NUM_THREADS, C::SMEM_BYTES, st>>>(ma, mw, g.M, g.N, g.K,
-                                                                      g.epi, err);
-  return cudaGetLastError();
+  return launch_k(gemm_tc_kernel<BN, KIND>, dim3(grid), dim3(NUM_THREADS), C::SMEM_BYTES, st, ma,
+                  mw, g.M, g.N, g.K, g.epi, err);
 }
 
 template <int BN>
@@ -425,9 +428,8 @@ cudaError_t launch2(const GemmArgs& g, int* err, int num_sms, cudaStream_t st) {
   }
   const int tiles = ((g.M + 2 * BM - 1) / (2 * BM)) * (g.N / C2_BN);
   const int clusters = tiles < mc ? tiles : mc;
-  gemm_tc2_kernel<KIND><<<2 * clusters, NUM_THREADS, C2_SMEM_BYTES, st>>>(ma, mw, g.M, g.N, g.K,
-                                                                         g.epi, err);
-  return cudaGetLastError();
+  return launch_k(gemm_tc2_kernel<KIND>, dim3(2 * clusters), dim3(NUM_THREADS), C2_SMEM_BYTES, st,
+                  ma, mw, g.M, g.N, g.K, g.epi, err);
 }
 
 cudaError_t dispatch2(const GemmArgs& g, int* err, int num_sms, cudaStream_t st) {

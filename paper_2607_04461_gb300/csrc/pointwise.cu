@@ -36,6 +36,8 @@ __global__ void __launch_bounds__(THREADS) ln_mod_kernel(const float* __restrict
                                                          float eps, float mul_base,
                                                          const float* __restrict__ mul,
                                                          const float* __restrict__ add) {
+  griddep_wait();
+  griddep_launch();
   __shared__ float red[THREADS / 32 > 0 ? THREADS / 32 : 1];
   const size_t row = blockIdx.x;
   const float* xr = x + row * D;
@@ -73,8 +75,8 @@ __global__ void __launch_bounds__(THREADS) ln_mod_kernel(const float* __restrict
 template <int THREADS, int VPT>
 cudaError_t ln_mod_launch(const float* x, bf16* out, int rows, int D, float eps, float mb,
                           const float* mul, const float* add, cudaStream_t st) {
-  ln_mod_kernel<THREADS, VPT><<<rows, THREADS, 0, st>>>(x, out, D, eps, mb, mul, add);
-  return cudaGetLastError();
+  return launch_k(ln_mod_kernel<THREADS, VPT>, dim3(rows), dim3(THREADS), 0, st, x, out, D, eps, mb,
+                  mul, add);
 }
 
 // ---------------------------------------------------------------------------------
@@ -96,6 +98,8 @@ __global__ void __launch_bounds__(THREADS) qk_norm_rope_kernel(
     bf16* __restrict__ x, int ld, int D, int col0, const float* __restrict__ w0, int col1,
     const float* __restrict__ w1, float eps, const float2* __restrict__ rope, int tokens,
     int head_dim) {
+  griddep_wait();
+  griddep_launch();
   __shared__ float red[THREADS / 32 > 0 ? THREADS / 32 : 1];
   const size_t row = blockIdx.x;
   const int seg = blockIdx.y;
@@ -136,14 +140,15 @@ cudaError_t qkn_launch(bf16* x, int rows, int ld, int D, int nseg, int col0, con
                        int col1, const float* w1, float eps, const float2* rope, int tokens,
                        int head_dim, cudaStream_t st) {
   dim3 grid(rows, nseg);
-  qk_norm_rope_kernel<THREADS, VPT><<<grid, THREADS, 0, st>>>(x, ld, D, col0, w0, col1, w1,
-                                                             eps, rope, tokens, head_dim);
-  return cudaGetLastError();
+  return launch_k(qk_norm_rope_kernel<THREADS, VPT>, grid, dim3(THREADS), 0, st, x, ld, D, col0, w0,
+                  col1, w1, eps, rope, tokens, head_dim);
 }
 
 // ---------------------------------------------------------------------------------
 __global__ void __launch_bounds__(256) proxy_add_kernel(float* __restrict__ h, size_t n8,
                                                         ProxyTerms t) {
+  griddep_wait();
+  griddep_launch();
   for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < n8;
        i += (size_t)gridDim.x * blockDim.x) {
     float acc[8];
@@ -167,6 +172,8 @@ __global__ void __launch_bounds__(256) patch_embed_kernel(const float* __restric
                                                           const bf16* __restrict__ Wp,
                                                           const float* __restrict__ bp, int D,
                                                           float* __restrict__ h) {
+  griddep_wait();
+  griddep_launch();
   extern __shared__ float xs[];  // [PE_TOK][PD]
   const int PD = C * p * p, gw = W / p, P = (H / p) * gw;
   const int M = n * P;
@@ -212,6 +219,8 @@ __global__ void __launch_bounds__(256) head_euler_kernel(const bf16* __restrict_
                                                          const bf16* __restrict__ Wh,
                                                          const float* __restrict__ bh, int D,
                                                          float dt, float* __restrict__ z) {
+  griddep_wait();
+  griddep_launch();
   constexpr int TPT = HE_TOK * PD / 256;
   __shared__ float as[HE_TOK][HE_KC + 1];
   __shared__ float ws[PD][HE_KC + 1];
@@ -265,6 +274,8 @@ __global__ void __launch_bounds__(256) gemv_kernel(const bf16* __restrict__ W,
                                                    const float* __restrict__ x,
                                                    float* __restrict__ y, int O, int K,
                                                    int act_in, int act_out) {
+  griddep_wait();
+  griddep_launch();
   const int warp = (blockIdx.x * blockDim.x + threadIdx.x) / 32, lane = threadIdx.x % 32;
   if (warp >= O) return;
   const bf16* wr = W + (size_t)warp * K;
@@ -285,6 +296,8 @@ __global__ void __launch_bounds__(256) gemv_kernel(const bf16* __restrict__ W,
 }
 
 __global__ void timestep_sincos_kernel(float t, int dim, float* emb) {
+  griddep_wait();
+  griddep_launch();
   const int half = dim / 2;
   for (int k = threadIdx.x; k < half; k += blockDim.x) {
     // f_k = 10000^(-k/half); the argument is formed in double for accuracy at 1000 t
@@ -299,6 +312,8 @@ __global__ void mod_prepare_kernel(const float* __restrict__ mod,
                                    const float* __restrict__ tables, int L, int D,
                                    float* __restrict__ modl, const float* __restrict__ htab,
                                    const float* __restrict__ temb, float* __restrict__ head_mod) {
+  griddep_wait();
+  griddep_launch();
   const size_t n6 = 6 * (size_t)D;
   for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < (size_t)L * n6;
        i += (size_t)gridDim.x * blockDim.x)
@@ -308,6 +323,8 @@ __global__ void mod_prepare_kernel(const float* __restrict__ mod,
 }
 
 __global__ void f32_to_bf16_kernel(const float* __restrict__ x, bf16* __restrict__ y, size_t n) {
+  griddep_wait();
+  griddep_launch();
   for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < n;
        i += (size_t)gridDim.x * blockDim.x)
     y[i] = __float2bfloat16_rn(x[i]);
@@ -364,8 +381,7 @@ cudaError_t proxy_add(float* h, size_t n_elems, const ProxyTerms& t, cudaStream_
   if (n_elems == 0 || t.n == 0) return cudaSuccess;
   if (n_elems % 8) return cudaErrorInvalidValue;
   const size_t n8 = n_elems / 8;
-  proxy_add_kernel<<<grid_for(n8, 256), 256, 0, st>>>(h, n8, t);
-  return cudaGetLastError();
+  return launch_k(proxy_add_kernel, dim3(grid_for(n8, 256)), dim3(256), 0, st, h, n8, t);
 }
 
 cudaError_t patch_embed(const float* z, int n, int C, int H, int W, int p, const bf16* Wp,
@@ -373,9 +389,8 @@ cudaError_t patch_embed(const float* z, int n, int C, int H, int W, int p, const
   const int PD = C * p * p, M = n * (H / p) * (W / p);
   if (M == 0) return cudaSuccess;
   if (PD % 8 || PD > 64) return cudaErrorInvalidValue;
-  patch_embed_kernel<<<(M + PE_TOK - 1) / PE_TOK, 256, PE_TOK * PD * sizeof(float), st>>>(
-      z, n, C, H, W, p, Wp, bp, D, h);
-  return cudaGetLastError();
+  return launch_k(patch_embed_kernel, dim3((M + PE_TOK - 1) / PE_TOK), dim3(256),
+                  PE_TOK * PD * sizeof(float), st, z, n, C, H, W, p, Wp, bp, D, h);
 }
 
 cudaError_t head_euler(const bf16* a, int n, int C, int H, int W, int p, const bf16* Wh,
@@ -385,36 +400,32 @@ cudaError_t head_euler(const bf16* a, int n, int C, int H, int W, int p, const b
   if (D % 8) return cudaErrorInvalidValue;
   const int grid = (M + HE_TOK - 1) / HE_TOK;
   switch (PD) {
-    case 8: head_euler_kernel<8><<<grid, 256, 0, st>>>(a, n, C, H, W, p, Wh, bh, D, dt, z); break;
-    case 16: head_euler_kernel<16><<<grid, 256, 0, st>>>(a, n, C, H, W, p, Wh, bh, D, dt, z); break;
-    case 32: head_euler_kernel<32><<<grid, 256, 0, st>>>(a, n, C, H, W, p, Wh, bh, D, dt, z); break;
-    case 64: head_euler_kernel<64><<<grid, 256, 0, st>>>(a, n, C, H, W, p, Wh, bh, D, dt, z); break;
+    case 8: return launch_k(head_euler_kernel<8>, dim3(grid), dim3(256), 0, st, a, n, C, H, W, p, Wh, bh, D, dt, z);
+    case 16: return launch_k(head_euler_kernel<16>, dim3(grid), dim3(256), 0, st, a, n, C, H, W, p, Wh, bh, D, dt, z);
+    case 32: return launch_k(head_euler_kernel<32>, dim3(grid), dim3(256), 0, st, a, n, C, H, W, p, Wh, bh, D, dt, z);
+    case 64: return launch_k(head_euler_kernel<64>, dim3(grid), dim3(256), 0, st, a, n, C, H, W, p, Wh, bh, D, dt, z);
     default: return cudaErrorInvalidValue;
   }
-  return cudaGetLastError();
 }
 
 cudaError_t gemv(const bf16* W, const float* b, const float* x, float* y, int O, int K,
                  int act_in, int act_out, cudaStream_t st) {
   if (K % 8) return cudaErrorInvalidValue;
-  gemv_kernel<<<(O * 32 + 255) / 256, 256, 0, st>>>(W, b, x, y, O, K, act_in, act_out);
-  return cudaGetLastError();
+  return launch_k(gemv_kernel, dim3((O * 32 + 255) / 256), dim3(256), 0, st, W, b, x, y, O, K,
+                  act_in, act_out);
 }
 
 cudaError_t timestep_sincos(float t, int dim, float* emb, cudaStream_t st) {
-  timestep_sincos_kernel<<<1, 128, 0, st>>>(t, dim, emb);
-  return cudaGetLastError();
+  return launch_k(timestep_sincos_kernel, dim3(1), dim3(128), 0, st, t, dim, emb);
 }
 
 cudaError_t mod_prepare(const float* mod, const float* tables, int L, int D, float* modl,
                         const float* htab, const float* temb, float* head_mod, cudaStream_t st) {
-  mod_prepare_kernel<<<grid_for((size_t)L * 6 * D, 256), 256, 0, st>>>(mod, tables, L, D, modl,
-                                                                       htab, temb, head_mod);
-  return cudaGetLastError();
+  return launch_k(mod_prepare_kernel, dim3(grid_for((size_t)L * 6 * D, 256)), dim3(256), 0, st, mod,
+                  tables, L, D, modl, htab, temb, head_mod);
 }
 
 cudaError_t f32_to_bf16(const float* x, bf16* y, size_t n, cudaStream_t st) {
   if (n == 0) return cudaSuccess;
-  f32_to_bf16_kernel<<<grid_for(n, 256), 256, 0, st>>>(x, y, n);
-  return cudaGetLastError();
+  return launch_k(f32_to_bf16_kernel, dim3(grid_for(n, 256)), dim3(256), 0, st, x, y, n);
 }
