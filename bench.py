@@ -160,11 +160,11 @@ def read_peaks():
     return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}, "fallback"
 
 
-def gemm_traffic_per_launch():
-    """DRAM bytes per tcgen05 GEMM launch from the committed ncu summary, if it was taken
-    on the current kernel source (else None)."""
+def gemm_traffic_ratio():
+    """DRAM traffic / algorithmic bytes of the tcgen05 GEMM from the committed ncu summary,
+    if it was taken on the current kernel source (else None)."""
     src = os.path.join(ROOT, "paper_2607_04461_gb300", "csrc", "gemm_tc.cu")
-    summ = os.path.join(ROOT, "profiles", "gemm_tc_wan13.md")
+    summ = os.path.join(ROOT, "profiles", "gemm_tc_ffn_wan13.md")
     if not os.path.exists(summ):
         return None
     sha = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
@@ -173,9 +173,9 @@ def gemm_traffic_per_launch():
         if line.startswith("bench-key "):
             k, _, v = line[len("bench-key "):].partition(":")
             vals[k.strip()] = v.strip()
-    if vals.get("kernel_sha") != sha or "traffic_bytes_per_launch" not in vals:
+    if vals.get("kernel_sha") != sha or "traffic_ratio_to_algorithmic" not in vals:
         return None
-    return float(vals["traffic_bytes_per_launch"])
+    return float(vals["traffic_ratio_to_algorithmic"])
 
 
 def dist_env():
@@ -323,7 +323,8 @@ def run_gb300(args):
     g = stats["gemm_tc"]
     achieved = g["flops"] / (g["ms"] / 1e3) / 1e12 if g["ms"] > 0 else None
     peak = peaks["bf16_tflops_sustained"]
-    traffic = gemm_traffic_per_launch()
+    ratio = gemm_traffic_ratio()
+    traffic = ratio * g["bytes"] / g["launches"] if (ratio and g["launches"]) else None
     launches = sum(s["launches"] for s in launch_stats.values())
     algo_flops = N_CAND * computed_blocks(skip, proxy) * block_flops(cfg) + \
         (S_TOTAL - S_DRAFT) * cfg.depth * block_flops(cfg)
@@ -336,6 +337,9 @@ def run_gb300(args):
                         "unit": "TFLOP/s", "frac": (achieved / peak) if achieved else None,
                         "peak_kind": f"bf16 sustained, {peak_kind}",
                         "traffic": traffic,
+                        "traffic_note": "DRAM bytes per launch: ncu traffic/algorithmic ratio "
+                                        "of the FFN probes x this run's algorithmic bytes "
+                                        "per GEMM launch (profiles/gemm_tc_ffn_wan13.md)",
                         "launches": g["launches"], "ms": g["ms"] / args.steps,
                         "measured_in": "timed pass 2 (same steps, per-launch CUDA events on "
                                        "the library stream)",
