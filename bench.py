@@ -47,11 +47,23 @@ def workload():
     return cfg, sched, skip, proxy
 
 
-def config_dict(cfg):
-    return {"workload": "wan2.1-1.3B draft pool: N=32, 480x832 (1560 tokens), 10 of 50 "
+VARIANTS = {
+    "base": "",
+    "cfg": "; classifier-free guidance w=5 (16 candidates, 32 rows with the unconditional pass)",
+    "sde": "; Euler-Maruyama SDE steps, a=0.7, caller-supplied N(0,1) draws",
+}
+
+
+def n_candidates(variant):
+    return N_CAND // 2 if variant == "cfg" else N_CAND
+
+
+def config_dict(cfg, variant="base"):
+    n = n_candidates(variant)
+    return {"workload": f"wan2.1-1.3B draft pool: N={n}, 480x832 (1560 tokens), 10 of 50 "
                         "steps, 1/3 blocks skipped, half of the rest proxied on odd steps, "
-                        "then a 40-step full refine of candidate 0",
-            "n_candidates": N_CAND, "tokens": cfg.tokens, "dim": cfg.dim, "depth": cfg.depth,
+                        "then a 40-step full refine of candidate 0" + VARIANTS[variant],
+            "n_candidates": n, "tokens": cfg.tokens, "dim": cfg.dim, "depth": cfg.depth,
             "draft_steps": S_DRAFT, "refine_steps": S_TOTAL - S_DRAFT,
             "l2": "inputs larger than L2 (2.6 GB weights), no flush"}
 
@@ -228,28 +240,37 @@ def run_gb300(args):
         dist.init_process_group("nccl", device_id=torch.device("cuda", local))
         pg = dist
     cfg, sched, skip, proxy = workload()
+    NC = n_candidates(args.variant)
     t_setup = time.time()
     w = synth.make_weights(cfg)
     model = fb.Model(cfg, w)
     del w
     stream = torch.cuda.Stream()
     model.set_stream(stream)
-    # each rank drafts its own 32 candidates (weak scaling, no collective on the path)
-    z0 = torch.from_numpy(synth.make_latents(cfg, N_CAND, first=rank * N_CAND)).cuda()
+    # each rank drafts its own candidates (weak scaling, no collective on the path)
+    z0 = torch.from_numpy(synth.make_latents(cfg, NC, first=rank * NC)).cuda()
     ctx_h = synth.make_text(cfg)
     ctx = torch.from_numpy(ctx_h).cuda()
     z = torch.empty_like(z0)
     zr = torch.empty_like(z0[0])
     draft_sched, tail = sched[: S_DRAFT + 1], sched[S_DRAFT:]
+    opts_d = opts_r = None
+    if args.variant == "cfg":
+        ctx_u = torch.from_numpy(synth.make_text(cfg, seed=8)).cuda()
+        opts_d = opts_r = fb.make_opts(5.0, ctx_u)
+    elif args.variant == "sde":
+        nd = torch.from_numpy(synth.make_noise(cfg, S_DRAFT, NC, seed=2000 + rank)).cuda()
+        nr = torch.from_numpy(synth.make_noise(cfg, S_TOTAL - S_DRAFT, 1, seed=3000 + rank)).cuda()
+        opts_d, opts_r = fb.make_opts(sde_a=0.7, noise=nd), fb.make_opts(sde_a=0.7, noise=nr)
     setup_s = time.time() - t_setup
 
     def dev_step():
         with torch.cuda.stream(stream):
             z.copy_(z0)
-        model.draft(z, ctx, draft_sched, skip, proxy)
+        model.draft(z, ctx, draft_sched, skip, proxy, opts=opts_d)
         with torch.cuda.stream(stream):
             zr.copy_(z[0])
-        model.refine(zr, ctx, tail)
+        model.refine(zr, ctx, tail, opts=opts_r)
 
     for _ in range(args.warmup):
         dev_step()
@@ -288,7 +309,7 @@ def run_gb300(args):
         ms = float(t.item())
         pg.barrier()
     ms_step = ms / args.steps
-    value = ws * N_CAND / (ms_step / 1e3)
+    value = ws * NC / (ms_step / 1e3)
 
     # end to end through the C-ABI with host buffers (pinned), copies inside the region
     zh = torch.empty(z0.shape, dtype=torch.float32, pin_memory=True)
@@ -299,9 +320,9 @@ def run_gb300(args):
 
     def host_step():
         zh.copy_(z0h)
-        model.draft(zh, ctxh, draft_sched, skip, proxy)
+        model.draft(zh, ctxh, draft_sched, skip, proxy, opts=opts_d)
         zrh.copy_(zh[0])
-        model.refine(zrh, ctxh, tail)
+        model.refine(zrh, ctxh, tail, opts=opts_r)
 
     host_step()
     torch.cuda.synchronize()
@@ -316,8 +337,8 @@ def run_gb300(args):
         pg.all_reduce(t, op=pg.ReduceOp.MAX)
         e2e_s = float(t.item())
     zbytes = z0.numel() * 4
-    h2d = zbytes + 2 * ctx_h.nbytes + zbytes // N_CAND
-    d2h = zbytes + zbytes // N_CAND
+    h2d = zbytes + 2 * ctx_h.nbytes + zbytes // NC
+    d2h = zbytes + zbytes // NC
 
     peaks, peak_kind = read_peaks()
     g = stats["gemm_tc"]
@@ -326,12 +347,13 @@ def run_gb300(args):
     ratio = gemm_traffic_ratio()
     traffic = ratio * g["bytes"] / g["launches"] if (ratio and g["launches"]) else None
     launches = sum(s["launches"] for s in launch_stats.values())
-    algo_flops = N_CAND * computed_blocks(skip, proxy) * block_flops(cfg) + \
-        (S_TOTAL - S_DRAFT) * cfg.depth * block_flops(cfg)
+    passes = 2 if args.variant == "cfg" else 1
+    algo_flops = passes * (NC * computed_blocks(skip, proxy) * block_flops(cfg) +
+                           (S_TOTAL - S_DRAFT) * cfg.depth * block_flops(cfg))
     out = {"metric": METRIC, "value": value, "unit": "candidates/s", "n_gpus": ws,
            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_step,
            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
-           "data": "synthetic", "config": config_dict(cfg),
+           "data": "synthetic", "config": config_dict(cfg, args.variant),
            "roofline": {"bound": "tensor", "kernel": "gemm_tc (tcgen05/TMEM GEMM, all "
                         "projections)", "achieved": achieved, "peak": peak,
                         "unit": "TFLOP/s", "frac": (achieved / peak) if achieved else None,
@@ -346,7 +368,7 @@ def run_gb300(args):
                         "pass2_ms_per_step": ms_instrumented / args.steps},
            "step_tflops": algo_flops / (ms_step / 1e3) / 1e12,
            "step_frac_of_peak": algo_flops / (ms_step / 1e3) / 1e12 / peak,
-           "e2e": {"value": ws * N_CAND / e2e_s, "unit": "candidates/s",
+           "e2e": {"value": ws * NC / e2e_s, "unit": "candidates/s",
                    "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h)},
            "gpu_launches": int(launches),
            "clocks": clk.summary(),
@@ -354,7 +376,7 @@ def run_gb300(args):
                            "gflop": v["flops"] / args.steps / 1e9}
                        for k, v in launch_stats.items() if v["launches"]},
            "setup_s": setup_s}
-    if rank == 0 and ws == 1 and not args.no_cpu_baseline:
+    if rank == 0 and ws == 1 and not args.no_cpu_baseline and args.variant == "base":
         pb, nb = oracle_sample(cfg, sched, skip, proxy, args.cpu_budget)
         v = oracle_cands_per_s(pb, cfg, skip, proxy)
         out["cpu_baseline"] = {
@@ -502,6 +524,9 @@ def main():
     ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
     ap.add_argument("--cpu-budget", type=float, default=15.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--variant", choices=list(VARIANTS), default="base",
+                    help="base: the draft-pool workload; cfg / sde: the same with guidance "
+                         "or SDE steps")
     ap.add_argument("--probe", choices=["gemm", "gemm_resid", "attn", "attn_mma", "gemm_shapes",
                                         "breakdown"],
                     default=None)

@@ -118,6 +118,33 @@ fb_status fb_draft(fb_model* m, float* latents, int n, const float* text_ctx,
 fb_status fb_refine(fb_model* m, float* latent, const float* text_ctx,
                     const float* full_schedule, int n_steps);
 
+/* ---- sampler options (§8 NEXT rows: guidance and the SDE step) -----------------
+ * guidance / text_uncond: classifier-free guidance. When text_uncond is not NULL every
+ * step also runs an unconditional pass (text_uncond, [text_len][text_dim] fp32, host or
+ * device) through the same plan with its own proxy cache, and uses
+ * v = v_u + guidance * (v_c - v_u). The conditional and unconditional rows form one
+ * batch of 2n candidates, so 2n <= max_n is required (FB_EINVAL otherwise).
+ * sde_a / noise: sde_a = 0 is the Euler step of the flow-matching ODE; sde_a > 0 is the
+ * Euler-Maruyama step of the equivalent SDE (App. A.1):
+ *   z <- z + [v + s^2/(2t) (z + (1-t) v)] dt + s sqrt(|dt|) eps,  dt = t' - t,
+ *   s = sde_a sqrt(t / (1 - t)), evaluated at t' when t = 1,
+ * with eps read from noise: [n_steps][n][latent_c][latent_h][latent_w] fp32 standard
+ * normal draws supplied by the caller (host or device), required when sde_a > 0. */
+typedef struct fb_sampler_opts {
+  float guidance;
+  const float* text_uncond;
+  float sde_a;
+  const float* noise;
+} fb_sampler_opts;
+
+/* fb_draft_ex / fb_refine_ex: fb_draft / fb_refine with sampler options (opts may be
+ * NULL: no guidance, ODE steps). fb_refine_ex's noise is [n_steps][1][C][H][W]. */
+fb_status fb_draft_ex(fb_model* m, float* latents, int n, const float* text_ctx,
+                      const float* schedule, int n_steps, const uint8_t* skip_mask,
+                      const int32_t* proxy_plan, const fb_sampler_opts* opts);
+fb_status fb_refine_ex(fb_model* m, float* latent, const float* text_ctx,
+                       const float* full_schedule, int n_steps, const fb_sampler_opts* opts);
+
 /* fb_plan_from_phi: expands phi = (S', n_skip, l_start, l_end, f_full) (§4.1,
  * "Configuration Space") into skip_mask [S'][depth] and proxy_plan [S'][depth]
  * (caller-allocated host arrays). Layers l_start..l_end are 1-indexed as in the paper

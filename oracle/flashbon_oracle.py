@@ -37,6 +37,12 @@ Readings where the paper is silent or ambiguous (all arithmetic in fp64):
      every non-skipped layer from the last full step;
   R4 n_skip: layers in L_skip (1-indexed in the paper) are skipped at steps k >= n_skip;
   R5 schedule t_i = 1 - i/S; the embedding sees 1000 t.
+  R6 classifier-free guidance (used by the paper only for its GRPO experiments): the
+     conditional and unconditional passes run through the same plan, each with its own
+     proxy cache, and the step uses v = v_u + w (v_c - v_u);
+  R7 SDE sampling (App. A.1, Euler-Maruyama form of the reverse SDE): with dt = t' - t < 0
+     the noise term is sigma_t sqrt(|dt|) eps; sigma_t = a sqrt(t / (1 - t)) is undefined
+     at t = 1, where it is evaluated at the next timestep t' instead.
 """
 from __future__ import annotations
 
@@ -154,6 +160,26 @@ def taylor_forecast(anchors, t):
     _, h3 = anchors[2]
     hddot = (h1 - 2.0 * h2 + h3) / (F64(tau1) - F64(tau2)) ** 2
     return h1 + dt * hdot + 0.5 * dt * dt * hddot
+
+
+def sde_sigma(t, t_next, a):
+    """sigma_t = a sqrt(t / (1 - t)) (App. A.1); at t = 1 evaluated at t_next (R7)."""
+    te = F64(t_next) if F64(t) >= 1.0 else F64(t)
+    return F64(a) * np.sqrt(te / (1.0 - te))
+
+
+def euler_maruyama_step(z, v, t, t_next, a, eps):
+    """One step of App. A.1's update, with dt = t_next - t:
+        z + [v + sigma^2 / (2 t) (z + (1 - t) v)] dt + sigma sqrt(|dt|) eps."""
+    t, t_next = F64(t), F64(t_next)
+    dt = t_next - t
+    sig = sde_sigma(t, t_next, a)
+    return z + (v + sig * sig / (2.0 * t) * (z + (1.0 - t) * v)) * dt + sig * np.sqrt(abs(dt)) * eps
+
+
+def guided_velocity(v_cond, v_uncond, w):
+    """Classifier-free guidance: v = v_u + w (v_c - v_u)."""
+    return v_uncond + F64(w) * (v_cond - v_uncond)
 
 
 # ----------------------------------------------------------------------------------
@@ -297,51 +323,78 @@ class OracleModel:
         return linear(a, w["head.w"], w["head.b"])
 
     # -- sampler ----------------------------------------------------------------------
-    def sample_one(self, z, ctx_kv, schedule, skip, proxy, trace=None):
+    def _blocks(self, i, h, t, mod, ctx_kv, skip, proxy, anchors, needed, cache, trace):
+        """Blocks of step i on h: skip (Eq. 6), compute (Eq. 7, caching Delta_l when a
+        later proxy needs it) or proxy (Eqs. 3-5)."""
+        for l in range(self.cfg.depth):
+            if skip[i][l]:
+                continue
+            if int(proxy[i][l]) == COMPUTE:
+                h_new = self.block(l, h, mod, ctx_kv[l])
+                if (i, l) in needed:
+                    cache[(i, l)] = (t, h_new - h)
+                h = h_new
+            else:
+                h = h + taylor_forecast([cache[(s, l)] for s in anchors[(i, l)]], t)
+            if trace is not None:
+                trace.append((i, l, h.copy()))
+        return h
+
+    def sample_one(self, z, ctx_kv, schedule, skip, proxy, trace=None, ctx_kv_uncond=None,
+                   guidance=1.0, sde_a=0.0, noise=None):
         """One candidate through len(schedule)-1 steps under (skip, proxy).
 
         Step i goes from t = schedule[i] to t' = schedule[i+1]: h_0 = PatchEmbed(z);
-        for each block, skip (Eq. 6), compute (Eq. 7, caching Delta_l when a later
-        proxy needs it) or proxy (Eqs. 3-5); v = Head(h); z <- z + (t' - t) v."""
+        the blocks; v = Head(h); z <- z + (t' - t) v (the Euler step of dx = v dt).
+        With ctx_kv_uncond the step runs a second, unconditional pass with its own proxy
+        cache and uses the guided velocity (R6). With sde_a > 0 the step is App. A.1's
+        Euler-Maruyama update with the standard normal draws noise[i] (R7)."""
         cfg = self.cfg
         sched = np.asarray(schedule, F64)
         n_steps = len(sched) - 1
         anchors = resolve_plan(skip, proxy)
         needed = {(s, l) for (k, l), steps in anchors.items() for s in steps}
-        cache = {}
+        passes = [ctx_kv] if ctx_kv_uncond is None else [ctx_kv, ctx_kv_uncond]
+        caches = [{} for _ in passes]
         z = np.asarray(z, F64).copy()
         for i in range(n_steps):
             t, t_next = sched[i], sched[i + 1]
             temb, mod = self.time_embed(t)
-            h = self.patch_embed(z)
-            for l in range(cfg.depth):
-                if skip[i][l]:
-                    continue
-                if int(proxy[i][l]) == COMPUTE:
-                    h_new = self.block(l, h, mod, ctx_kv[l])
-                    if (i, l) in needed:
-                        cache[(i, l)] = (t, h_new - h)
-                    h = h_new
-                else:
-                    h = h + taylor_forecast([cache[(s, l)] for s in anchors[(i, l)]], t)
-                if trace is not None:
-                    trace.append((i, l, h.copy()))
-            v = self.head(h, temb)
-            z = z + (t_next - t) * unpatchify(v, cfg.latent_c, cfg.latent_h,
-                                              cfg.latent_w, cfg.patch)
+            vs = []
+            for kv, cache in zip(passes, caches):
+                h = self._blocks(i, self.patch_embed(z), t, mod, kv, skip, proxy, anchors,
+                                 needed, cache, trace if kv is ctx_kv else None)
+                vs.append(unpatchify(self.head(h, temb), cfg.latent_c, cfg.latent_h,
+                                     cfg.latent_w, cfg.patch))
+            v = vs[0] if len(vs) == 1 else guided_velocity(vs[0], vs[1], guidance)
+            if sde_a > 0:
+                z = euler_maruyama_step(z, v, t, t_next, sde_a, np.asarray(noise[i], F64))
+            else:
+                z = z + (t_next - t) * v
         return z
 
-    def draft(self, z_T, ctx, schedule, skip, proxy, candidates=None):
+    def draft(self, z_T, ctx, schedule, skip, proxy, candidates=None, ctx_uncond=None,
+              guidance=1.0, sde_a=0.0, noise=None):
         """Stage 1 (Eq. 8): each candidate's z_T through the truncated, accelerated
-        schedule. Candidates are independent; `candidates` picks a subset."""
+        schedule. Candidates are independent; `candidates` picks a subset. noise, when
+        sde_a > 0, is [n_steps][N][C][H][W] (indexed by the candidate's position in z_T)."""
         z_T = np.asarray(z_T)
         idx = range(z_T.shape[0]) if candidates is None else candidates
         kv = self.encode_text(ctx)
-        return np.stack([self.sample_one(z_T[j], kv, schedule, skip, proxy) for j in idx])
+        kvu = None if ctx_uncond is None else self.encode_text(ctx_uncond)
+        out = []
+        for j in idx:
+            nz = None if noise is None else np.asarray(noise)[:, j]
+            out.append(self.sample_one(z_T[j], kv, schedule, skip, proxy, ctx_kv_uncond=kvu,
+                                       guidance=guidance, sde_a=sde_a, noise=nz))
+        return np.stack(out)
 
-    def refine(self, z, ctx, schedule):
-        """Stage 3: resume from a cached latent with phi_full (no skip, no proxy)."""
+    def refine(self, z, ctx, schedule, ctx_uncond=None, guidance=1.0, sde_a=0.0, noise=None):
+        """Stage 3: resume from a cached latent with phi_full (no skip, no proxy).
+        noise, when sde_a > 0, is [n_steps][C][H][W]."""
         n = len(schedule) - 1
         skip = np.zeros((n, self.cfg.depth), np.uint8)
         proxy = np.full((n, self.cfg.depth), COMPUTE, np.int32)
-        return self.sample_one(z, self.encode_text(ctx), schedule, skip, proxy)
+        kvu = None if ctx_uncond is None else self.encode_text(ctx_uncond)
+        return self.sample_one(z, self.encode_text(ctx), schedule, skip, proxy,
+                               ctx_kv_uncond=kvu, guidance=guidance, sde_a=sde_a, noise=noise)

@@ -152,6 +152,9 @@ struct fb_model {
   bf16 *act = nullptr, *qkv = nullptr, *ao = nullptr, *cqb = nullptr, *ffh = nullptr;
   float* ctx_f = nullptr;
   bf16 *ctx_b = nullptr, *ctx_h = nullptr, *ctx_p = nullptr, *kvctx = nullptr;
+  bf16* kvctx_u = nullptr;  // unconditional context (guidance), allocated on first use
+  float* noise = nullptr;   // device copy of host SDE draws, grown on demand
+  size_t noise_elems = 0;
   bool text_ready = false;
   float *emb = nullptr, *th1 = nullptr, *temb = nullptr, *mod = nullptr, *modl = nullptr,
         *hmod = nullptr;
@@ -311,7 +314,7 @@ fb_status run_qkn(fb_model* m, bf16* x, int rows, int ld, int nseg, int col0, co
 }
 
 // ---- text encoding (once per call) --------------------------------------------------
-fb_status encode_text(fb_model* m, const float* ctx) {
+fb_status encode_text(fb_model* m, const float* ctx, bf16* kv_dst) {
   const fb_cfg& c = m->c;
   const size_t nctx = (size_t)c.text_len * c.text_dim;
   cudaPointerAttributes at{};
@@ -330,11 +333,11 @@ fb_status encode_text(fb_model* m, const float* ctx) {
                             m->ctx_h)));
   CKS(run_gemm(m, gemm_args(T, D, D, m->ctx_h, m->text_w2, m->text_b2, EPI_BF16, m->ctx_p)));
   for (int l = 0; l < c.depth; ++l) {
-    bf16* kv = m->kvctx + (size_t)l * T * 2 * D;
+    bf16* kv = kv_dst + (size_t)l * T * 2 * D;
     CKS(run_gemm(m, gemm_args(T, 2 * D, D, m->ctx_p, m->L[l].ckv, m->L[l].cbkv, EPI_BF16, kv)));
     CKS(run_qkn(m, kv, T, 2 * D, 1, 0, m->L[l].cnk, 0, m->L[l].cnk, nullptr));
   }
-  m->text_ready = true;
+  if (kv_dst == m->kvctx) m->text_ready = true;
   return FB_OK;
 }
 
@@ -353,7 +356,9 @@ fb_status time_embed(fb_model* m, float t) {
 }
 
 // ---- one block B_l (Eq. 7) on h = hA (rows M), optional contribution write ----------
-fb_status block_forward(fb_model* m, int l, float* h, int n, bf16* delta) {
+// n: candidates (rows n*P). n_uncond > 0: the last n_uncond candidates are the
+// unconditional rows of guidance and attend to the unconditional text context.
+fb_status block_forward(fb_model* m, int l, float* h, int n, bf16* delta, int n_uncond = 0) {
   const fb_cfg& c = m->c;
   const int D = c.dim, M = n * m->P;
   const Layer& w = m->L[l];
@@ -383,12 +388,14 @@ fb_status block_forward(fb_model* m, int l, float* h, int n, bf16* delta) {
   CKS(run_ln(m, hB, m->act, M, 0.f, w.n3w, w.n3b));
   CKS(run_gemm(m, gemm_args(M, D, D, m->act, w.cq, w.cbq, EPI_BF16, m->cqb)));
   CKS(run_qkn(m, m->cqb, M, D, 1, 0, w.cnq, 0, w.cnq, nullptr));
-  {
-    const bf16* kv = m->kvctx + (size_t)l * c.text_len * 2 * D;
+  for (int part = 0; part < (n_uncond ? 2 : 1); ++part) {
+    const int n0 = part ? n - n_uncond : 0, nb = n_uncond ? (part ? n_uncond : n - n_uncond) : n;
+    const bf16* kv = (part ? m->kvctx_u : m->kvctx) + (size_t)l * c.text_len * 2 * D;
     AttnArgs a{};
-    a.Q = m->cqb; a.K = kv; a.V = kv + D; a.O = m->ao;
+    a.Q = m->cqb + (size_t)n0 * m->P * D; a.K = kv; a.V = kv + D;
+    a.O = m->ao + (size_t)n0 * m->P * D;
     a.ldq = D; a.ldk = a.ldv = 2 * D; a.ldo = D;
-    a.batch = n; a.Lq = m->P; a.Lkv = c.text_len; a.kv_batch_rows = 0;
+    a.batch = nb; a.Lq = m->P; a.Lkv = c.text_len; a.kv_batch_rows = 0;
     a.heads = c.heads; a.head_dim = c.head_dim;
     CKS(run_attn(m, a, FB_K_ATTN_CROSS));
   }
@@ -524,10 +531,20 @@ bool is_device_ptr(const void* p) {
   return at.type == cudaMemoryTypeDevice || at.type == cudaMemoryTypeManaged;
 }
 
-// The sampler loop shared by fb_draft and fb_refine (latents z on the device).
-fb_status sample(fb_model* m, float* z, int n, const float* sched, int S, const Plan& plan) {
+struct SampOpts {
+  bool guided = false;
+  float w = 1.f;
+  float sde_a = 0.f;
+  const float* noise = nullptr;  // device, [S][n][C][H][W]
+};
+
+// The sampler loop shared by fb_draft and fb_refine (latents z on the device). With
+// guidance the batch holds 2n candidates' rows: n conditional, then n unconditional.
+fb_status sample(fb_model* m, float* z, int n, const float* sched, int S, const Plan& plan,
+                 const SampOpts& so) {
   const fb_cfg& c = m->c;
-  const size_t slot_elems = (size_t)n * m->P * c.dim;
+  const int nr = so.guided ? 2 * n : n;  // candidates' rows in the batch
+  const size_t slot_elems = (size_t)nr * m->P * c.dim;
   const size_t need = slot_elems * plan.n_slots;
   if (need > m->anchor_elems) {
     CK(cudaStreamSynchronize(m->st));
@@ -540,20 +557,21 @@ fb_status sample(fb_model* m, float* z, int n, const float* sched, int S, const 
     CKS(dalloc_t(m, &m->anchors, need));
     m->anchor_elems = need;
   }
-  const int M = n * m->P;
+  const int M = nr * m->P;
+  const size_t zn = (size_t)n * c.latent_c * c.latent_h * c.latent_w;
   for (int k = 0; k < S; ++k) {
     const float t = sched[k], t1 = sched[k + 1];
     CKS(time_embed(m, t));
-    {
-      KTimer kt(m, FB_K_EMBED, 2.0 * M * (double)c.dim * m->PD,
-                4.0 * M * (double)(c.dim + m->PD));
+    for (int u = 0; u < (so.guided ? 2 : 1); ++u) {
+      KTimer kt(m, FB_K_EMBED, 2.0 * n * m->P * (double)c.dim * m->PD,
+                4.0 * n * m->P * (double)(c.dim + m->PD));
       CK(patch_embed(z, n, c.latent_c, c.latent_h, c.latent_w, c.patch, m->patch_w, m->patch_b,
-                     c.dim, m->hA, m->st));
+                     c.dim, m->hA + (size_t)u * n * m->P * c.dim, m->st));
     }
     for (const Action& a : plan.steps[k]) {
       if (a.type == 0) {
         bf16* d = a.slot >= 0 ? m->anchors + (size_t)a.slot * slot_elems : nullptr;
-        CKS(block_forward(m, a.layer, m->hA, n, d));
+        CKS(block_forward(m, a.layer, m->hA, nr, d, so.guided ? n : 0));
       } else {
         for (size_t i0 = 0; i0 < a.terms.size(); i0 += FB_PROXY_MAX_TERMS) {
           ProxyTerms pt{};
@@ -570,25 +588,74 @@ fb_status sample(fb_model* m, float* z, int n, const float* sched, int S, const 
     }
     CKS(run_ln(m, m->hA, m->act, M, 1.f, m->hmod + c.dim, m->hmod));
     {
+      HeadStep hs{};
+      hs.dt = t1 - t;
+      hs.t = t;
+      hs.w = so.w;
+      hs.uncond_rows = so.guided ? n * m->P : 0;
+      if (so.sde_a > 0.f) {
+        // App. A.1: sigma_t = a sqrt(t / (1 - t)), evaluated at t' when t = 1
+        const double td = t, te = td >= 1.0 ? (double)t1 : td;
+        const double sig = so.sde_a * std::sqrt(te / (1.0 - te));
+        hs.sde_c = (float)(sig * sig / (2.0 * td));
+        hs.nscale = (float)(sig * std::sqrt(std::fabs((double)t1 - td)));
+        hs.noise = so.noise + (size_t)k * zn;
+      }
       KTimer kt(m, FB_K_HEAD, 2.0 * M * (double)c.dim * m->PD,
                 2.0 * M * (double)c.dim + 8.0 * M * m->PD);
       CK(head_euler(m->act, n, c.latent_c, c.latent_h, c.latent_w, c.patch, m->head_w, m->head_b,
-                    c.dim, t1 - t, z, m->st));
+                    c.dim, hs, z, m->st));
     }
   }
   return FB_OK;
 }
 
 fb_status run_sampler(fb_model* m, float* latents, int n, const float* text_ctx,
-                      const float* sched, int S, const Plan& plan) {
+                      const float* sched, int S, const Plan& plan,
+                      const fb_sampler_opts* opts) {
   const fb_cfg& c = m->c;
   const size_t zn = (size_t)n * c.latent_c * c.latent_h * c.latent_w;
+  SampOpts so;
+  if (opts) {
+    so.guided = opts->text_uncond != nullptr;
+    so.w = opts->guidance;
+    so.sde_a = opts->sde_a;
+    if (!(std::isfinite(so.w)) || !(so.sde_a >= 0.f) || !std::isfinite(so.sde_a))
+      return fail(FB_EINVAL, "guidance must be finite and sde_a >= 0");
+    if (so.sde_a > 0.f && !opts->noise) return fail(FB_EINVAL, "sde_a > 0 needs noise");
+    if (so.guided && 2 * n > c.max_n)
+      return fail(FB_EINVAL, "guidance needs 2n <= max_n (n=%d, max_n=%d)", n, c.max_n);
+  }
+  if (so.guided && !m->kvctx_u)
+    CKS(dalloc_t(m, &m->kvctx_u, (size_t)c.depth * c.text_len * 2 * c.dim));
+  if (so.sde_a > 0.f) {
+    if (is_device_ptr(opts->noise)) {
+      so.noise = opts->noise;
+    } else {
+      const size_t ne = zn * S;
+      if (ne > m->noise_elems) {
+        CK(cudaStreamSynchronize(m->st));
+        if (m->noise) {
+          cudaFree(m->noise);
+          m->allocs.erase(std::find(m->allocs.begin(), m->allocs.end(), (void*)m->noise));
+          m->noise = nullptr;
+          m->noise_elems = 0;
+        }
+        CKS(dalloc_t(m, &m->noise, ne));
+        m->noise_elems = ne;
+      }
+      CK(cudaMemcpyAsync(m->noise, opts->noise, ne * sizeof(float), cudaMemcpyHostToDevice,
+                         m->st));
+      so.noise = m->noise;
+    }
+  }
   CKS(begin_call(m));
-  CKS(encode_text(m, text_ctx));
+  CKS(encode_text(m, text_ctx, m->kvctx));
+  if (so.guided) CKS(encode_text(m, opts->text_uncond, m->kvctx_u));
   const bool dev = is_device_ptr(latents);
   float* z = dev ? latents : m->zbuf;
   if (!dev) CK(cudaMemcpyAsync(z, latents, zn * sizeof(float), cudaMemcpyHostToDevice, m->st));
-  CKS(sample(m, z, n, sched, S, plan));
+  CKS(sample(m, z, n, sched, S, plan, so));
   if (!dev) CK(cudaMemcpyAsync(latents, z, zn * sizeof(float), cudaMemcpyDeviceToHost, m->st));
   return end_call(m);
 }
@@ -787,13 +854,19 @@ fb_status fb_set_stream(fb_model* m, void* stream) {
 fb_status fb_encode_text(fb_model* m, const float* text_ctx) {
   if (!m || !text_ctx) return fail(FB_EINVAL, "null argument");
   CKS(begin_call(m));
-  CKS(encode_text(m, text_ctx));
+  CKS(encode_text(m, text_ctx, m->kvctx));
   return end_call(m);
 }
 
 fb_status fb_draft(fb_model* m, float* latents, int n, const float* text_ctx,
                    const float* schedule, int n_steps, const uint8_t* skip_mask,
                    const int32_t* proxy_plan) {
+  return fb_draft_ex(m, latents, n, text_ctx, schedule, n_steps, skip_mask, proxy_plan, nullptr);
+}
+
+fb_status fb_draft_ex(fb_model* m, float* latents, int n, const float* text_ctx,
+                      const float* schedule, int n_steps, const uint8_t* skip_mask,
+                      const int32_t* proxy_plan, const fb_sampler_opts* opts) {
   if (!m) return fail(FB_EINVAL, "model is NULL");
   if (n < 0 || n > m->c.max_n) return fail(FB_EINVAL, "n=%d outside [0, max_n=%d]", n, m->c.max_n);
   if (n_steps < 0) return fail(FB_EINVAL, "n_steps < 0");
@@ -802,11 +875,16 @@ fb_status fb_draft(fb_model* m, float* latents, int n, const float* text_ctx,
   CKS(check_schedule(schedule, n_steps));
   Plan plan;
   CKS(analyse_plan(m->c, schedule, n_steps, skip_mask, proxy_plan, &plan));
-  return run_sampler(m, latents, n, text_ctx, schedule, n_steps, plan);
+  return run_sampler(m, latents, n, text_ctx, schedule, n_steps, plan, opts);
 }
 
 fb_status fb_refine(fb_model* m, float* latent, const float* text_ctx,
                     const float* full_schedule, int n_steps) {
+  return fb_refine_ex(m, latent, text_ctx, full_schedule, n_steps, nullptr);
+}
+
+fb_status fb_refine_ex(fb_model* m, float* latent, const float* text_ctx,
+                       const float* full_schedule, int n_steps, const fb_sampler_opts* opts) {
   if (!m) return fail(FB_EINVAL, "model is NULL");
   if (n_steps < 0) return fail(FB_EINVAL, "n_steps < 0");
   if (n_steps == 0) return FB_OK;
@@ -814,7 +892,7 @@ fb_status fb_refine(fb_model* m, float* latent, const float* text_ctx,
   CKS(check_schedule(full_schedule, n_steps));
   Plan plan;
   CKS(analyse_plan(m->c, full_schedule, n_steps, nullptr, nullptr, &plan));
-  return run_sampler(m, latent, 1, text_ctx, full_schedule, n_steps, plan);
+  return run_sampler(m, latent, 1, text_ctx, full_schedule, n_steps, plan, opts);
 }
 
 fb_status fb_plan_from_phi(int S, int S_prime, int n_skip, int l_start, int l_end, int f_full,

@@ -61,9 +61,17 @@ cudaError_t proxy_add(float* h, size_t n_elems, const ProxyTerms& t, cudaStream_
 // h[(b*P + tok)][:] = W_p * patch(z_b, tok) + b_p.
 cudaError_t patch_embed(const float* z, int n, int C, int H, int W, int p, const bf16* Wp,
                         const float* bp, int D, float* h, cudaStream_t st);
-// z[b] += dt * unpatchify(a * Wh^T + bh), a bf16 [n*P][D].
+// v = unpatchify(a * Wh^T + bh) from a bf16 [n*P][D]; with guidance (uncond_rows > 0) also
+// v_u from rows uncond_rows.. and v = v_u + w (v - v_u). Then the step on z[b]:
+//   ODE (noise == null): z += dt v
+//   SDE: z += (v + sde_c (z + (1 - t) v)) dt + nscale * noise[b]   (noise like z)
+struct HeadStep {
+  float dt, t, w, sde_c, nscale;
+  int uncond_rows;        // 0: no guidance
+  const float* noise;     // null: ODE step
+};
 cudaError_t head_euler(const bf16* a, int n, int C, int H, int W, int p, const bf16* Wh,
-                       const float* bh, int D, float dt, float* z, cudaStream_t st);
+                       const float* bh, int D, const HeadStep& hs, float* z, cudaStream_t st);
 // y[o] = act_out(b[o] + sum_k W[o][k] act_in(x[k])), act: 0 none, 1 SiLU.
 cudaError_t gemv(const bf16* W, const float* b, const float* x, float* y, int O, int K,
                  int act_in, int act_out, cudaStream_t st);

@@ -211,33 +211,35 @@ __global__ void __launch_bounds__(256) patch_embed_kernel(const float* __restric
 
 // ---------------------------------------------------------------------------------
 // head_euler: 32 tokens per CTA, 256 threads; K staged through shared memory in
-// chunks of 128. Thread -> output o = tid % PD and TPT = 32 PD / 256 consecutive tokens.
-constexpr int HE_TOK = 32, HE_KC = 128;
+// chunks of 64. Thread -> output o = tid % PD and TPT = 32 PD / 256 consecutive tokens.
+// With guidance each thread also accumulates the unconditional row of its tokens.
+constexpr int HE_TOK = 32, HE_KC = 64;
 template <int PD>
 __global__ void __launch_bounds__(256) head_euler_kernel(const bf16* __restrict__ a, int n,
                                                          int C, int H, int W, int p,
                                                          const bf16* __restrict__ Wh,
                                                          const float* __restrict__ bh, int D,
-                                                         float dt, float* __restrict__ z) {
-  griddep_wait();
-  griddep_launch();
+                                                         HeadStep hs, float* __restrict__ z) {
   constexpr int TPT = HE_TOK * PD / 256;
-  __shared__ float as[HE_TOK][HE_KC + 1];
+  __shared__ float as[2][HE_TOK][HE_KC + 1];
   __shared__ float ws[PD][HE_KC + 1];
   const int gw = W / p, P = (H / p) * gw, M = n * P;
+  const bool guided = hs.uncond_rows > 0;
   const int tok0 = blockIdx.x * HE_TOK;
   const int o = threadIdx.x % PD, grp = threadIdx.x / PD;
-  float acc[TPT];
+  float acc[TPT], accu[TPT];
 #pragma unroll
-  for (int i = 0; i < TPT; ++i) acc[i] = 0.f;
+  for (int i = 0; i < TPT; ++i) acc[i] = accu[i] = 0.f;
   for (int k0 = 0; k0 < D; k0 += HE_KC) {
     __syncthreads();
-    for (int i = threadIdx.x; i < HE_TOK * HE_KC / 8; i += 256) {
-      const int t = i / (HE_KC / 8), kc = (i % (HE_KC / 8)) * 8;
+    for (int i = threadIdx.x; i < 2 * HE_TOK * HE_KC / 8; i += 256) {
+      const int u = i / (HE_TOK * HE_KC / 8), rem = i % (HE_TOK * HE_KC / 8);
+      const int t = rem / (HE_KC / 8), kc = (rem % (HE_KC / 8)) * 8;
       float v[8] = {0, 0, 0, 0, 0, 0, 0, 0};
-      if (tok0 + t < M && k0 + kc < D) load_bf16x8(a + (size_t)(tok0 + t) * D + k0 + kc, v);
+      if ((u == 0 || guided) && tok0 + t < M && k0 + kc < D)
+        load_bf16x8(a + (size_t)(tok0 + t + u * hs.uncond_rows) * D + k0 + kc, v);
 #pragma unroll
-      for (int j = 0; j < 8; ++j) as[t][kc + j] = v[j];
+      for (int j = 0; j < 8; ++j) as[u][t][kc + j] = v[j];
     }
     for (int i = threadIdx.x; i < PD * HE_KC / 8; i += 256) {
       const int r = i / (HE_KC / 8), kc = (i % (HE_KC / 8)) * 8;
@@ -251,7 +253,10 @@ __global__ void __launch_bounds__(256) head_euler_kernel(const bf16* __restrict_
     for (int k = 0; k < HE_KC; ++k) {
       const float wv = ws[o][k];
 #pragma unroll
-      for (int i = 0; i < TPT; ++i) acc[i] += wv * as[grp * TPT + i][k];
+      for (int i = 0; i < TPT; ++i) {
+        acc[i] += wv * as[0][grp * TPT + i][k];
+        accu[i] += wv * as[1][grp * TPT + i][k];
+      }
     }
   }
   const float bias = bh[o];
@@ -260,9 +265,18 @@ __global__ void __launch_bounds__(256) head_euler_kernel(const bf16* __restrict_
   for (int i = 0; i < TPT; ++i) {
     const int tok = tok0 + grp * TPT + i;
     if (tok < M) {
+      float v = acc[i] + bias;
+      if (guided) {
+        const float vu = accu[i] + bias;
+        v = vu + hs.w * (v - vu);
+      }
       const int b = tok / P, pt = tok % P, r = pt / gw, cc = pt % gw;
-      float* zp = z + (((size_t)b * C + ch) * H + r * p + dy) * W + cc * p + dx;
-      *zp += dt * (acc[i] + bias);
+      const size_t zi = (((size_t)b * C + ch) * H + r * p + dy) * W + cc * p + dx;
+      const float zo = z[zi];
+      if (hs.noise)
+        z[zi] = zo + (v + hs.sde_c * (zo + (1.f - hs.t) * v)) * hs.dt + hs.nscale * hs.noise[zi];
+      else
+        z[zi] = zo + hs.dt * v;
     }
   }
 }
@@ -394,16 +408,16 @@ cudaError_t patch_embed(const float* z, int n, int C, int H, int W, int p, const
 }
 
 cudaError_t head_euler(const bf16* a, int n, int C, int H, int W, int p, const bf16* Wh,
-                       const float* bh, int D, float dt, float* z, cudaStream_t st) {
+                       const float* bh, int D, const HeadStep& hs, float* z, cudaStream_t st) {
   const int PD = C * p * p, M = n * (H / p) * (W / p);
   if (M == 0) return cudaSuccess;
   if (D % 8) return cudaErrorInvalidValue;
-  const int grid = (M + HE_TOK - 1) / HE_TOK;
+  const dim3 grid((M + HE_TOK - 1) / HE_TOK);
   switch (PD) {
-    case 8: return launch_k(head_euler_kernel<8>, dim3(grid), dim3(256), 0, st, a, n, C, H, W, p, Wh, bh, D, dt, z);
-    case 16: return launch_k(head_euler_kernel<16>, dim3(grid), dim3(256), 0, st, a, n, C, H, W, p, Wh, bh, D, dt, z);
-    case 32: return launch_k(head_euler_kernel<32>, dim3(grid), dim3(256), 0, st, a, n, C, H, W, p, Wh, bh, D, dt, z);
-    case 64: return launch_k(head_euler_kernel<64>, dim3(grid), dim3(256), 0, st, a, n, C, H, W, p, Wh, bh, D, dt, z);
+    case 8: return launch_k(head_euler_kernel<8>, grid, dim3(256), 0, st, a, n, C, H, W, p, Wh, bh, D, hs, z);
+    case 16: return launch_k(head_euler_kernel<16>, grid, dim3(256), 0, st, a, n, C, H, W, p, Wh, bh, D, hs, z);
+    case 32: return launch_k(head_euler_kernel<32>, grid, dim3(256), 0, st, a, n, C, H, W, p, Wh, bh, D, hs, z);
+    case 64: return launch_k(head_euler_kernel<64>, grid, dim3(256), 0, st, a, n, C, H, W, p, Wh, bh, D, hs, z);
     default: return cudaErrorInvalidValue;
   }
 }

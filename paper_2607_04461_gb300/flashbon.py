@@ -36,6 +36,11 @@ class fb_cfg(ctypes.Structure):
         ("eps_ln", ctypes.c_float), ("eps_rms", ctypes.c_float), ("rope_theta", ctypes.c_float)]
 
 
+class fb_sampler_opts(ctypes.Structure):
+    _fields_ = [("guidance", ctypes.c_float), ("text_uncond", ctypes.c_void_p),
+                ("sde_a", ctypes.c_float), ("noise", ctypes.c_void_p)]
+
+
 class fb_kstat(ctypes.Structure):
     _fields_ = [("launches", ctypes.c_uint64), ("ms", ctypes.c_double),
                 ("flops", ctypes.c_double), ("bytes", ctypes.c_double)]
@@ -44,7 +49,7 @@ class fb_kstat(ctypes.Structure):
 EXPORTS = ["fb_weights_count", "fb_weights_entry", "fb_init_model", "fb_free", "fb_set_stream",
            "fb_encode_text", "fb_draft", "fb_refine", "fb_plan_from_phi", "fb_block_forward",
            "fb_last_error", "fb_set_timing", "fb_get_stats", "fb_reset_stats", "fb_kernel_name",
-           "fb_op_gemm", "fb_op_attention"]
+           "fb_op_gemm", "fb_op_attention", "fb_draft_ex", "fb_refine_ex"]
 
 _lib = None
 
@@ -68,6 +73,8 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
         "fb_encode_text": (I, [P, P]),
         "fb_draft": (I, [P, P, I, P, P, I, P, P]),
         "fb_refine": (I, [P, P, P, P, I]),
+        "fb_draft_ex": (I, [P, P, I, P, P, I, P, P, ctypes.POINTER(fb_sampler_opts)]),
+        "fb_refine_ex": (I, [P, P, P, P, I, ctypes.POINTER(fb_sampler_opts)]),
         "fb_plan_from_phi": (I, [I, I, I, I, I, I, I, I, P, P]),
         "fb_block_forward": (I, [P, I, P, I, F]),
         "fb_last_error": (ctypes.c_char_p, []),
@@ -180,6 +187,32 @@ def fb_refine(model: int, latent, text_ctx, full_schedule) -> None:
                                     _ptr(sched), len(sched) - 1))
 
 
+def make_opts(guidance=1.0, text_uncond=None, sde_a=0.0, noise=None):
+    """fb_sampler_opts; keeps references to the buffers it points to."""
+    o = fb_sampler_opts(float(guidance), _ptr(text_uncond, np.float32), float(sde_a),
+                        _ptr(noise, np.float32))
+    o._keep = (text_uncond, noise)
+    return o
+
+
+def fb_draft_ex(model: int, latents, n: int, text_ctx, schedule, skip_mask=None,
+                proxy_plan=None, opts=None) -> None:
+    sched = np.ascontiguousarray(schedule, np.float32)
+    sk = None if skip_mask is None else np.ascontiguousarray(skip_mask, np.uint8)
+    px = None if proxy_plan is None else np.ascontiguousarray(proxy_plan, np.int32)
+    _check(load_library().fb_draft_ex(model, _ptr(latents, np.float32), n,
+                                      _ptr(text_ctx, np.float32), _ptr(sched), len(sched) - 1,
+                                      _ptr(sk), _ptr(px),
+                                      None if opts is None else ctypes.byref(opts)))
+
+
+def fb_refine_ex(model: int, latent, text_ctx, full_schedule, opts=None) -> None:
+    sched = np.ascontiguousarray(full_schedule, np.float32)
+    _check(load_library().fb_refine_ex(model, _ptr(latent, np.float32),
+                                       _ptr(text_ctx, np.float32), _ptr(sched), len(sched) - 1,
+                                       None if opts is None else ctypes.byref(opts)))
+
+
 def fb_plan_from_phi(S, S_prime, n_skip, l_start, l_end, f_full, order, depth):
     skip = np.zeros((S_prime, depth), np.uint8)
     proxy = np.zeros((S_prime, depth), np.int32)
@@ -252,12 +285,19 @@ class Model:
     def encode_text(self, ctx):
         fb_encode_text(self.handle, ctx)
 
-    def draft(self, latents, text_ctx, schedule, skip_mask=None, proxy_plan=None, n=None):
+    def draft(self, latents, text_ctx, schedule, skip_mask=None, proxy_plan=None, n=None,
+              opts=None):
         n = latents.shape[0] if n is None else n
-        fb_draft(self.handle, latents, n, text_ctx, schedule, skip_mask, proxy_plan)
+        if opts is None:
+            fb_draft(self.handle, latents, n, text_ctx, schedule, skip_mask, proxy_plan)
+        else:
+            fb_draft_ex(self.handle, latents, n, text_ctx, schedule, skip_mask, proxy_plan, opts)
 
-    def refine(self, latent, text_ctx, schedule):
-        fb_refine(self.handle, latent, text_ctx, schedule)
+    def refine(self, latent, text_ctx, schedule, opts=None):
+        if opts is None:
+            fb_refine(self.handle, latent, text_ctx, schedule)
+        else:
+            fb_refine_ex(self.handle, latent, text_ctx, schedule, opts)
 
     def block_forward(self, layer, h, n, t):
         fb_block_forward(self.handle, layer, h, n, t)

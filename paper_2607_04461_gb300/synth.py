@@ -158,6 +158,13 @@ def make_text(cfg: Cfg, seed: int = 7) -> np.ndarray:
     return rng.standard_normal((cfg.text_len, cfg.text_dim), dtype=np.float32)
 
 
+def make_noise(cfg: Cfg, n_steps: int, n: int, seed: int = 2000) -> np.ndarray:
+    """Standard normal draws for SDE steps: [n_steps][n][C][H][W] float32."""
+    rng = np.random.default_rng(seed)
+    return rng.standard_normal((n_steps, n, cfg.latent_c, cfg.latent_h, cfg.latent_w),
+                               dtype=np.float32)
+
+
 def make_schedule(S: int) -> np.ndarray:
     """t_i = 1 - i/S for i = 0..S (float32)."""
     return (1.0 - np.arange(S + 1, dtype=np.float64) / S).astype(np.float32)

@@ -282,3 +282,72 @@ def test_wan13_draft_pool_full_size(wan13_pool):
     ref = O.OracleModel(cfg, w)
     want = ref.draft(z[:1], ctx, sched[:3], skip[:2], proxy[:2])
     check_latents(two.cpu().numpy()[0], want[0], z[0], label="wan13 cand 0, 2 steps")
+
+
+# ---- NEXT rows: classifier-free guidance and SDE steps -------------------------------
+
+@pytest.fixture(scope="module")
+def small4():
+    cfg = synth.SMALL.with_(max_n=4)
+    w = synth.make_weights(cfg, bf16=True, norm_std=0.2)
+    m = fb.Model(cfg, w)
+    yield cfg, w, m, O.OracleModel(cfg, w)
+    m.close()
+
+
+@pytest.mark.parametrize("mode", ["cfg", "sde", "cfg_sde"])
+def test_small_guidance_and_sde_match_oracle(small4, mode):
+    cfg, w, m, ref = small4
+    S, n = 4, 2
+    z = synth.make_latents(cfg, n)
+    ctx, ctx_u = synth.make_text(cfg), synth.make_text(cfg, seed=8)
+    sched = synth.make_schedule(S)
+    skip, proxy = synth.random_plan(S, cfg.depth, 1 / 3, 0.5, seed=5, order=1)
+    guided, sde = "cfg" in mode, "sde" in mode
+    noise = synth.make_noise(cfg, S, n) if sde else None
+    opts = fb.make_opts(guidance=4.5 if guided else 1.0, text_uncond=ctx_u if guided else None,
+                        sde_a=0.7 if sde else 0.0, noise=noise)
+    zd = cuda(z)
+    m.draft(zd, ctx, sched, skip, proxy, opts=opts)
+    want = ref.draft(z, ctx, sched, skip, proxy, ctx_uncond=ctx_u if guided else None,
+                     guidance=4.5, sde_a=0.7 if sde else 0.0, noise=noise)
+    for j in range(n):
+        check_latents(zd.cpu().numpy()[j], want[j], z[j], label=f"{mode} cand {j}")
+
+
+def test_guided_refine_with_sde_matches_oracle(small4):
+    cfg, w, m, ref = small4
+    S = 3
+    z = synth.make_latents(cfg, 1)[0]
+    ctx, ctx_u = synth.make_text(cfg), synth.make_text(cfg, seed=8)
+    sched = synth.make_schedule(6)[3:]
+    noise = synth.make_noise(cfg, S, 1, seed=77)
+    zd = cuda(z)
+    m.refine(zd, ctx, sched, opts=fb.make_opts(5.0, ctx_u, 0.3, cuda(noise)))
+    want = ref.refine(z, ctx, sched, ctx_uncond=ctx_u, guidance=5.0, sde_a=0.3, noise=noise[:, 0])
+    check_latents(zd.cpu().numpy(), want, z, label="guided SDE refine")
+
+
+def test_guidance_weight_one_is_the_conditional_draft(small4):
+    cfg, w, m, _ = small4
+    z = synth.make_latents(cfg, 2)
+    ctx, ctx_u = synth.make_text(cfg), synth.make_text(cfg, seed=8)
+    sched = synth.make_schedule(3)
+    a, b = cuda(z), cuda(z)
+    m.draft(a, ctx, sched)
+    m.draft(b, ctx, sched, opts=fb.make_opts(1.0, ctx_u))
+    d = (a - b).abs().max().item()
+    assert d <= 1e-5 * max(1.0, a.abs().max().item()), d
+
+
+def test_guidance_and_sde_argument_errors(small4):
+    cfg, w, m, _ = small4
+    ctx = synth.make_text(cfg)
+    sched = synth.make_schedule(2)
+    z = cuda(synth.make_latents(cfg, 3))
+    with pytest.raises(fb.FlashBonError) as e:      # 2n > max_n
+        m.draft(z, ctx, sched, opts=fb.make_opts(3.0, ctx))
+    assert e.value.status == fb.FB_EINVAL
+    with pytest.raises(fb.FlashBonError) as e:      # SDE without draws
+        m.draft(z, ctx, sched, opts=fb.make_opts(sde_a=0.5))
+    assert e.value.status == fb.FB_EINVAL

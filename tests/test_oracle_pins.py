@@ -359,3 +359,65 @@ def test_candidates_are_independent():
     sk, px = synth.tiny_plan()
     all3 = m.draft(z, ctx, sched, sk, px)
     np.testing.assert_array_equal(m.draft(z, ctx, sched, sk, px, candidates=[2])[0], all3[2])
+
+
+# -- NEXT rows: classifier-free guidance and the SDE step (App. A.1) ------------------------
+
+def test_sde_step_hand_value():
+    # t = 0.5, t' = 0.4, a = 0.3: sigma = 0.3; drift 2 + 0.09/1.0 * (1 + 0.5*2) = 2.18
+    z = O.euler_maruyama_step(np.array([1.0]), np.array([2.0]), 0.5, 0.4, 0.3, np.array([0.5]))
+    assert z[0] == pytest.approx(1.0 - 0.218 + 0.3 * math.sqrt(0.1) * 0.5, abs=1e-14)
+
+
+def test_sde_step_with_a0_is_the_ode_step():
+    z, v, eps = rng.standard_normal(50), rng.standard_normal(50), rng.standard_normal(50)
+    np.testing.assert_array_equal(O.euler_maruyama_step(z, v, 0.7, 0.6, 0.0, eps), z + (0.6 - 0.7) * v)
+
+
+def test_sde_sigma_at_t1_uses_next_timestep():
+    assert O.sde_sigma(1.0, 0.98, 0.7) == pytest.approx(0.7 * math.sqrt(0.98 / 0.02))
+    assert O.sde_sigma(0.5, 0.48, 0.7) == pytest.approx(0.7)
+
+
+def test_sde_preserves_rectified_flow_marginals():
+    """App. A.1: the SDE keeps the ODE's marginals. Toy problem with a known velocity:
+    x_0 ~ N(0, s^2), x_1 ~ N(0, 1), x_t = (1-t) x_0 + t x_1 has variance
+    (1-t)^2 s^2 + t^2 and marginal velocity v(x, t) = x (t - (1-t) s^2) / var_t. Start
+    from N(0, 1) at t = 1 and integrate to t = 0.25 with many particles."""
+    s2 = 0.25
+    var = lambda t: (1 - t) ** 2 * s2 + t * t  # noqa: E731
+    vel = lambda x, t: x * (t - (1 - t) * s2) / var(t)  # noqa: E731
+    g = np.random.default_rng(3)
+    x = g.standard_normal(200_000)
+    ts = np.linspace(1.0, 0.25, 301)
+    for t, tn in zip(ts[:-1], ts[1:]):
+        x = O.euler_maruyama_step(x, vel(x, t), t, tn, 0.7, g.standard_normal(x.size))
+    assert x.var() == pytest.approx(var(0.25), rel=0.03)
+    # a drift correction with the wrong sign does not preserve the marginals
+    y = g.standard_normal(200_000)
+    for t, tn in zip(ts[:-1], ts[1:]):
+        sig = O.sde_sigma(t, tn, 0.7)
+        v = vel(y, t)
+        y = y + (v - sig * sig / (2 * t) * (y + (1 - t) * v)) * (tn - t) + \
+            sig * math.sqrt(t - tn) * g.standard_normal(y.size)
+    assert abs(y.var() / var(0.25) - 1) > 0.1
+
+
+def test_guided_velocity_endpoints():
+    vc, vu = rng.standard_normal(9), rng.standard_normal(9)
+    np.testing.assert_array_equal(O.guided_velocity(vc, vu, 1.0), vu + (vc - vu))
+    np.testing.assert_allclose(O.guided_velocity(vc, vu, 1.0), vc, rtol=0, atol=1e-15)
+    np.testing.assert_array_equal(O.guided_velocity(vc, vu, 0.0), vu)
+
+
+def test_cfg_with_identical_contexts_is_unguided():
+    cfg, w = _tiny()
+    m = O.OracleModel(cfg, w)
+    z = synth.make_latents(cfg, 1)
+    ctx = synth.make_text(cfg)
+    sched = synth.make_schedule(3)
+    sk, px = synth.empty_plan(3, 2)
+    px[2, 0] = synth.proxy_code(1, 1)
+    a = m.draft(z, ctx, sched, sk, px)
+    b = m.draft(z, ctx, sched, sk, px, ctx_uncond=ctx, guidance=4.0)
+    np.testing.assert_allclose(a, b, rtol=1e-12, atol=1e-12)
