@@ -12,8 +12,11 @@
  *    last failing call on the calling thread.
  *  - The caller owns every input and output buffer. The model owns its device weights,
  *    activation buffers and the proxy cache.
- *  - All work is enqueued on the model's stream (fb_set_stream, default: a stream the
- *    model creates) and the call returns after that stream has finished the work.
+ *  - All work is enqueued on the model's stream (fb_set_stream; default: a blocking
+ *    stream the model creates, ordered with the legacy default stream, so inputs written
+ *    there are complete before the model reads them) and the call returns after that
+ *    stream has finished the work. With a caller's stream set, the caller orders its own
+ *    writes of the inputs before the call (same stream or an event).
  *  - "host or device" pointers are classified with cudaPointerGetAttributes: device
  *    (or managed) memory is used in place; host memory is staged through device
  *    buffers inside the call.

@@ -726,7 +726,9 @@ fb_status fb_init_model(const fb_cfg* cfg, const float* weights_host, fb_model**
     cudaGetLastError();
     return bail(fail(FB_ECUDA, "no CUDA device"));
   }
-  if (cudaStreamCreateWithFlags(&m->own, cudaStreamNonBlocking) != cudaSuccess)
+  // A blocking stream: its work is ordered after work the caller put on the legacy
+  // default stream (e.g. copies that fill the input buffers) and vice versa.
+  if (cudaStreamCreateWithFlags(&m->own, cudaStreamDefault) != cudaSuccess)
     return bail(fail(FB_ECUDA, "cudaStreamCreate failed"));
   m->st = m->own;
   if (cudaMallocHost(&m->herr, sizeof(int)) != cudaSuccess)
