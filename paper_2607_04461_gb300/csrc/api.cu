@@ -26,6 +26,11 @@ bool fb_pdl_enabled() {
   static const bool on = getenv("FB_NO_PDL") == nullptr;
   return on;
 }
+namespace {
+thread_local bool g_prev_op_is_kernel = false;
+}
+bool fb_prev_op_is_kernel() { return g_prev_op_is_kernel; }
+void fb_set_prev_op_is_kernel(bool v) { g_prev_op_is_kernel = v; }
 
 namespace {
 
@@ -203,7 +208,10 @@ struct KTimer {
     if (m->timing_mask & (1u << k)) {
       a = get();
       b = get();
-      if (a && b) cudaEventRecord(a, m->st);
+      if (a && b) {
+        cudaEventRecord(a, m->st);
+        fb_stream_op_not_kernel();
+      }
     }
   }
   cudaEvent_t get() {
@@ -222,6 +230,7 @@ struct KTimer {
   ~KTimer() {
     if (a && b) {
       cudaEventRecord(b, m->st);
+      fb_stream_op_not_kernel();
       m->pending.push_back({kind, a, b});
     } else {
       if (a) m->ev_pool.push_back(a);
@@ -241,13 +250,16 @@ void collect_timings(fb_model* m) {
   m->pending.clear();
 }
 
-// Starts an API call: clears the device error word.
+// Starts an API call: clears the device error word. Work the caller queued on the
+// stream before the call is not one of our kernels either.
 fb_status begin_call(fb_model* m) {
+  fb_stream_op_not_kernel();
   CK(cudaMemsetAsync(m->derr, 0, sizeof(int), m->st));
   return FB_OK;
 }
 // Ends an API call: waits for the stream, checks the device error word.
 fb_status end_call(fb_model* m) {
+  fb_stream_op_not_kernel();
   CK(cudaMemcpyAsync(m->herr, m->derr, sizeof(int), cudaMemcpyDeviceToHost, m->st));
   CK(cudaStreamSynchronize(m->st));
   collect_timings(m);
@@ -322,6 +334,7 @@ fb_status encode_text(fb_model* m, const float* ctx, bf16* kv_dst) {
   if (cudaPointerGetAttributes(&at, ctx) != cudaSuccess) cudaGetLastError();
   if (at.type != cudaMemoryTypeDevice && at.type != cudaMemoryTypeManaged) {
     CK(cudaMemcpyAsync(m->ctx_f, ctx, nctx * sizeof(float), cudaMemcpyHostToDevice, m->st));
+    fb_stream_op_not_kernel();
     src = m->ctx_f;
   }
   {
@@ -547,6 +560,7 @@ fb_status sample(fb_model* m, float* z, int n, const float* sched, int S, const 
   const size_t slot_elems = (size_t)nr * m->P * c.dim;
   const size_t need = slot_elems * plan.n_slots;
   if (need > m->anchor_elems) {
+    fb_stream_op_not_kernel();
     CK(cudaStreamSynchronize(m->st));
     if (m->anchors) {
       cudaFree(m->anchors);
@@ -644,6 +658,7 @@ fb_status run_sampler(fb_model* m, float* latents, int n, const float* text_ctx,
         CKS(dalloc_t(m, &m->noise, ne));
         m->noise_elems = ne;
       }
+      fb_stream_op_not_kernel();
       CK(cudaMemcpyAsync(m->noise, opts->noise, ne * sizeof(float), cudaMemcpyHostToDevice,
                          m->st));
       so.noise = m->noise;
@@ -654,9 +669,15 @@ fb_status run_sampler(fb_model* m, float* latents, int n, const float* text_ctx,
   if (so.guided) CKS(encode_text(m, opts->text_uncond, m->kvctx_u));
   const bool dev = is_device_ptr(latents);
   float* z = dev ? latents : m->zbuf;
-  if (!dev) CK(cudaMemcpyAsync(z, latents, zn * sizeof(float), cudaMemcpyHostToDevice, m->st));
+  if (!dev) {
+    CK(cudaMemcpyAsync(z, latents, zn * sizeof(float), cudaMemcpyHostToDevice, m->st));
+    fb_stream_op_not_kernel();
+  }
   CKS(sample(m, z, n, sched, S, plan, so));
-  if (!dev) CK(cudaMemcpyAsync(latents, z, zn * sizeof(float), cudaMemcpyDeviceToHost, m->st));
+  if (!dev) {
+    fb_stream_op_not_kernel();
+    CK(cudaMemcpyAsync(latents, z, zn * sizeof(float), cudaMemcpyDeviceToHost, m->st));
+  }
   return end_call(m);
 }
 
@@ -757,6 +778,7 @@ fb_status fb_init_model(const fb_cfg* cfg, const float* weights_host, fb_model**
     if (e.kind == W_MAT) {
       dst = reinterpret_cast<bf16*>(m->wmat) + mo;
       mo += e.numel;
+      fb_stream_op_not_kernel();
       if (cudaMemcpyAsync(stage, src, e.numel * 4, cudaMemcpyHostToDevice, m->st) != cudaSuccess ||
           f32_to_bf16(stage, reinterpret_cast<bf16*>(dst), e.numel, m->st) != cudaSuccess ||
           cudaStreamSynchronize(m->st) != cudaSuccess)
@@ -850,6 +872,7 @@ fb_status fb_set_stream(fb_model* m, void* stream) {
   if (!m) return fail(FB_EINVAL, "model is NULL");
   CK(cudaStreamSynchronize(m->st));
   m->st = stream ? reinterpret_cast<cudaStream_t>(stream) : m->own;
+  fb_stream_op_not_kernel();
   return FB_OK;
 }
 

@@ -39,9 +39,15 @@ __device__ __forceinline__ void griddep_launch() {
 }
 
 #ifdef __CUDACC__
-// Launches kern with programmatic stream serialisation (unless FB_NO_PDL is set in the
-// environment, read once).
+// The programmatic relaxation only orders a kernel after a preceding KERNEL that calls
+// griddepcontrol; a copy, memset or event record before it gives no such ordering. So
+// the attribute is used only when the previous operation this host thread put on the
+// stream was one of these kernels: every other stream operation of the library calls
+// fb_stream_op_not_kernel(). FB_NO_PDL in the environment (read once) disables it.
 bool fb_pdl_enabled();
+bool fb_prev_op_is_kernel();
+void fb_set_prev_op_is_kernel(bool v);
+inline void fb_stream_op_not_kernel() { fb_set_prev_op_is_kernel(false); }
 template <typename... KArgs, typename... Args>
 inline cudaError_t launch_k(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem,
                             cudaStream_t st, Args... args) {
@@ -54,8 +60,10 @@ inline cudaError_t launch_k(void (*kern)(KArgs...), dim3 grid, dim3 block, size_
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = fb_pdl_enabled() ? 1 : 0;
-  return cudaLaunchKernelEx(&cfg, kern, static_cast<KArgs>(args)...);
+  cfg.numAttrs = (fb_pdl_enabled() && fb_prev_op_is_kernel()) ? 1 : 0;
+  const cudaError_t e = cudaLaunchKernelEx(&cfg, kern, static_cast<KArgs>(args)...);
+  fb_set_prev_op_is_kernel(e == cudaSuccess);
+  return e;
 }
 #endif
 

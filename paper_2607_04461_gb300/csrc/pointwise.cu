@@ -220,6 +220,8 @@ __global__ void __launch_bounds__(256) head_euler_kernel(const bf16* __restrict_
                                                          const bf16* __restrict__ Wh,
                                                          const float* __restrict__ bh, int D,
                                                          HeadStep hs, float* __restrict__ z) {
+  griddep_wait();
+  griddep_launch();
   constexpr int TPT = HE_TOK * PD / 256;
   __shared__ float as[2][HE_TOK][HE_KC + 1];
   __shared__ float ws[PD][HE_KC + 1];

@@ -1,0 +1,41 @@
+"""Static checks on the CUDA sources (no GPU needed)."""
+import os
+import re
+
+CSRC = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))),
+                    "paper_2607_04461_gb300", "csrc")
+
+
+def kernels():
+    for f in sorted(os.listdir(CSRC)):
+        if not f.endswith(".cu"):
+            continue
+        src = open(os.path.join(CSRC, f)).read()
+        for m in re.finditer(r"__global__[^{;]*?\b(\w+)\s*\(", src, flags=re.S):
+            # body: from the first "{" after the signature to its matching "}"
+            i = src.index("{", m.end())
+            depth, j = 0, i
+            while True:
+                if src[j] == "{":
+                    depth += 1
+                elif src[j] == "}":
+                    depth -= 1
+                    if depth == 0:
+                        break
+                j += 1
+            yield f, m.group(1), src[i:j]
+
+
+def test_every_kernel_waits_for_its_predecessor():
+    """Kernels are launched with programmatic stream serialisation, so each must call
+    griddep_wait() before it reads what the previous kernel wrote."""
+    found = list(kernels())
+    assert len(found) >= 15
+    missing = [f"{f}:{name}" for f, name, body in found if "griddep_wait()" not in body]
+    assert not missing, missing
+
+
+def test_every_kernel_is_launched_through_launch_k():
+    for f in os.listdir(CSRC):
+        if f.endswith(".cu"):
+            assert "<<<" not in open(os.path.join(CSRC, f)).read(), f
