@@ -190,6 +190,18 @@ def gemm_traffic_ratio():
     return float(vals["traffic_ratio_to_algorithmic"])
 
 
+def aggregate(ms_local, n_local, world, reduce_max=None):
+    """Whole-job throughput: every rank drafts n_local candidates; the job's time is the
+    slowest rank's (max over ranks). reduce_max(x) returns the max of x over ranks."""
+    ms = reduce_max(ms_local) if reduce_max else ms_local
+    return ms, world * n_local / (ms / 1e3)
+
+
+def rank_candidates(rank, n_local):
+    """Candidate indices (latent seeds 1000 + index) drafted by `rank`."""
+    return list(range(rank * n_local, (rank + 1) * n_local))
+
+
 def dist_env():
     ws = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
@@ -248,7 +260,7 @@ def run_gb300(args):
     stream = torch.cuda.Stream()
     model.set_stream(stream)
     # each rank drafts its own candidates (weak scaling, no collective on the path)
-    z0 = torch.from_numpy(synth.make_latents(cfg, NC, first=rank * NC)).cuda()
+    z0 = torch.from_numpy(synth.make_latents(cfg, NC, first=rank_candidates(rank, NC)[0])).cuda()
     ctx_h = synth.make_text(cfg)
     ctx = torch.from_numpy(ctx_h).cuda()
     z = torch.empty_like(z0)
@@ -303,13 +315,13 @@ def run_gb300(args):
     stats = model.stats()
     model.set_timing(0)
     ms_instrumented = e2.elapsed_time(e3)
-    if pg:
-        t = torch.tensor([ms], device="cuda")
+    def reduce_max(x):
+        t = torch.tensor([x], device="cuda")
         pg.all_reduce(t, op=pg.ReduceOp.MAX)
-        ms = float(t.item())
+        return float(t.item())
+    ms_step, value = aggregate(ms / args.steps, NC, ws, reduce_max if pg else None)
+    if pg:
         pg.barrier()
-    ms_step = ms / args.steps
-    value = ws * NC / (ms_step / 1e3)
 
     # end to end through the C-ABI with host buffers (pinned), copies inside the region
     zh = torch.empty(z0.shape, dtype=torch.float32, pin_memory=True)

@@ -159,6 +159,24 @@ fb_status fb_plan_from_phi(int S, int S_prime, int n_skip, int l_start, int l_en
                            int f_full, int order, int depth, uint8_t* skip_mask,
                            int32_t* proxy_plan);
 
+/* ---- Stage 2 selection (§4.2), host only ---------------------------------------
+ * fb_select_elo: multi-stage selection over M drafts. scores: [M] pointwise verifier
+ * scores (1..10), seeding Elo ratings r = 1500 + (s - 5) * 100. Keeps the top
+ * ceil(rho1 M) by rating (ties: lower index), runs ceil(kappa M1) comparisons between
+ * adjacent entries of the survivors sorted by rating (passes from the top, re-sorted
+ * before each pass), keeps the top ceil(rho2 M1), plays every pair of those in rating
+ * order, and writes the index with the highest rating to *winner. The paper gives
+ * neither the base K nor the expected score: k_base (32 is usual) times 1.2 / 1.0 / 0.7
+ * for the verifier's high / medium / low confidence, and E_a = 1 / (1 + 10^((r_b - r_a)
+ * / 400)). compare(user, a, b, &confidence) returns non-zero if a is preferred and sets
+ * confidence to 0 (high), 1 (medium) or 2 (low). out_ratings: [M] final ratings or NULL;
+ * out_calls: number of pairwise calls or NULL. FB_EINVAL for bad arguments or a
+ * confidence outside 0..2 (then treated as medium). Runs on the calling thread. */
+typedef int (*fb_pair_verifier)(void* user, int a, int b, int* confidence);
+fb_status fb_select_elo(const int32_t* scores, int M, double rho1, double rho2,
+                        double kappa, double k_base, fb_pair_verifier compare, void* user,
+                        int* winner, double* out_ratings, int* out_calls);
+
 /* fb_block_forward: one block B_layer (Eq. 7) in place on h [n * tokens][dim] fp32
  * DEVICE memory (candidate-major rows), with the modulation of timestep t and the
  * text context of the last fb_encode_text (FB_ESTATE without one). */

@@ -43,6 +43,9 @@ Readings where the paper is silent or ambiguous (all arithmetic in fp64):
   R7 SDE sampling (App. A.1, Euler-Maruyama form of the reverse SDE): with dt = t' - t < 0
      the noise term is sigma_t sqrt(|dt|) eps; sigma_t = a sqrt(t / (1 - t)) is undefined
      at t = 1, where it is evaluated at the next timestep t' instead.
+  R8 Elo selection (§4.2 Stage 2): base K and the expected-score formula are not given;
+     K = 32 and the logistic 400-point expected score are used; the adjacent comparisons
+     are passes over the rating-sorted survivors; ties go to the lower index.
 """
 from __future__ import annotations
 
@@ -398,3 +401,67 @@ class OracleModel:
         kvu = None if ctx_uncond is None else self.encode_text(ctx_uncond)
         return self.sample_one(z, self.encode_text(ctx), schedule, skip, proxy,
                                ctx_kv_uncond=kvu, guidance=guidance, sde_a=sde_a, noise=noise)
+
+
+# ----------------------------------------------------------------------------------
+# Stage 2: multi-stage selection with Elo ratings (§4.2)
+# ----------------------------------------------------------------------------------
+
+CONF_MULT = (1.2, 1.0, 0.7)  # confidence high / medium / low scales K (§4.2 footnote)
+
+
+def elo_seed(score):
+    """r^(0) = 1500 + (s - 5) * 100."""
+    return 1500.0 + (float(score) - 5.0) * 100.0
+
+
+def elo_update(ra, rb, a_wins, k):
+    """Standard Elo: expected score E_a = 1 / (1 + 10^((r_b - r_a) / 400)) (R8: the
+    paper does not print it)."""
+    ea = 1.0 / (1.0 + 10.0 ** ((rb - ra) / 400.0))
+    sa = 1.0 if a_wins else 0.0
+    return ra + k * (sa - ea), rb + k * ((1.0 - sa) - (1.0 - ea))
+
+
+def _top(ids, r, count):
+    """The `count` best by rating; ties go to the lower index."""
+    return sorted(ids, key=lambda j: (-r[j], j))[:count]
+
+
+def elo_select(scores, compare, rho1=0.5, rho2=0.5, kappa=1.5, k_base=32.0):
+    """Pointwise pruning + Elo seeding, sparse adjacent comparisons, dense tournament.
+
+    compare(a, b) -> (a_preferred: bool, confidence in {0, 1, 2}). Readings (R8): base K
+    = k_base; the ceil(kappa M1) adjacent comparisons are passes over the list sorted by
+    rating (from the top), the list re-sorted before each pass; the tournament plays the
+    pairs (i, j), i < j, of the survivors in rating order. Returns (winner, ratings,
+    pairwise calls)."""
+    import math
+    M = len(scores)
+    r = {j: elo_seed(scores[j]) for j in range(M)}
+    calls = 0
+
+    def play(a, b):
+        nonlocal calls
+        a_wins, conf = compare(a, b)
+        calls += 1
+        r[a], r[b] = elo_update(r[a], r[b], a_wins, k_base * CONF_MULT[conf])
+
+    ceil = lambda x: math.ceil(x - 1e-9)  # noqa: E731  (0.3 * 20 is 6, not 7)
+    s1 = _top(range(M), r, ceil(rho1 * M))
+    c2 = ceil(kappa * len(s1))
+    done = 0
+    while done < c2 and len(s1) > 1:
+        order = _top(s1, r, len(s1))
+        for i in range(len(order) - 1):
+            if done == c2:
+                break
+            play(order[i], order[i + 1])
+            done += 1
+    s2 = _top(s1, r, ceil(rho2 * len(s1)))
+    order = _top(s2, r, len(s2))
+    for i in range(len(order)):
+        for j in range(i + 1, len(order)):
+            play(order[i], order[j])
+    winner = _top(s2, r, 1)[0]
+    return winner, [r[j] for j in range(M)], calls

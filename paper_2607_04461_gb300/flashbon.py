@@ -49,7 +49,10 @@ class fb_kstat(ctypes.Structure):
 EXPORTS = ["fb_weights_count", "fb_weights_entry", "fb_init_model", "fb_free", "fb_set_stream",
            "fb_encode_text", "fb_draft", "fb_refine", "fb_plan_from_phi", "fb_block_forward",
            "fb_last_error", "fb_set_timing", "fb_get_stats", "fb_reset_stats", "fb_kernel_name",
-           "fb_op_gemm", "fb_op_attention", "fb_draft_ex", "fb_refine_ex"]
+           "fb_op_gemm", "fb_op_attention", "fb_draft_ex", "fb_refine_ex", "fb_select_elo"]
+
+PAIR_VERIFIER = ctypes.CFUNCTYPE(ctypes.c_int, ctypes.c_void_p, ctypes.c_int, ctypes.c_int,
+                                 ctypes.POINTER(ctypes.c_int))
 
 _lib = None
 
@@ -62,7 +65,7 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
     if not os.path.exists(path):
         raise FileNotFoundError(f"{path} not built: run paper_2607_04461_gb300.build.build()")
     L = ctypes.CDLL(path)
-    P, I, S, F = ctypes.c_void_p, ctypes.c_int, ctypes.c_size_t, ctypes.c_float
+    P, I, S, F, D = ctypes.c_void_p, ctypes.c_int, ctypes.c_size_t, ctypes.c_float, ctypes.c_double
     sig = {
         "fb_weights_count": (I, [ctypes.POINTER(fb_cfg), ctypes.POINTER(I), ctypes.POINTER(S)]),
         "fb_weights_entry": (I, [ctypes.POINTER(fb_cfg), I, ctypes.POINTER(ctypes.c_char_p),
@@ -75,6 +78,8 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
         "fb_refine": (I, [P, P, P, P, I]),
         "fb_draft_ex": (I, [P, P, I, P, P, I, P, P, ctypes.POINTER(fb_sampler_opts)]),
         "fb_refine_ex": (I, [P, P, P, P, I, ctypes.POINTER(fb_sampler_opts)]),
+        "fb_select_elo": (I, [P, I, D, D, D, D, PAIR_VERIFIER, P, ctypes.POINTER(I),
+                              ctypes.POINTER(ctypes.c_double), ctypes.POINTER(I)]),
         "fb_plan_from_phi": (I, [I, I, I, I, I, I, I, I, P, P]),
         "fb_block_forward": (I, [P, I, P, I, F]),
         "fb_last_error": (ctypes.c_char_p, []),
@@ -211,6 +216,26 @@ def fb_refine_ex(model: int, latent, text_ctx, full_schedule, opts=None) -> None
     _check(load_library().fb_refine_ex(model, _ptr(latent, np.float32),
                                        _ptr(text_ctx, np.float32), _ptr(sched), len(sched) - 1,
                                        None if opts is None else ctypes.byref(opts)))
+
+
+def fb_select_elo(scores, compare, rho1=0.5, rho2=0.5, kappa=1.5, k_base=32.0):
+    """Stage 2 selection. compare(a, b) -> (a_preferred, confidence 0/1/2).
+    Returns (winner, ratings [M], pairwise calls)."""
+    sc = np.ascontiguousarray(scores, np.int32)
+    M = sc.size
+
+    def cb(user, a, b, conf_ptr):
+        pref, conf = compare(a, b)
+        conf_ptr[0] = int(conf)
+        return 1 if pref else 0
+    fn = PAIR_VERIFIER(cb)
+    winner, calls = ctypes.c_int(), ctypes.c_int()
+    ratings = np.zeros(M, np.float64)
+    _check(load_library().fb_select_elo(_ptr(sc), M, rho1, rho2, kappa, k_base, fn, None,
+                                        ctypes.byref(winner),
+                                        ratings.ctypes.data_as(ctypes.POINTER(ctypes.c_double)),
+                                        ctypes.byref(calls)))
+    return winner.value, ratings, calls.value
 
 
 def fb_plan_from_phi(S, S_prime, n_skip, l_start, l_end, f_full, order, depth):

@@ -134,3 +134,36 @@ def test_null_model_is_rejected(lib):
     assert lib.fb_refine(None, None, None, None, 1) == fb.FB_EINVAL
     assert lib.fb_block_forward(None, 0, None, 1, 0.5) == fb.FB_EINVAL
     lib.fb_free(None)
+
+
+# ---- Stage 2 selection (host logic) ---------------------------------------------------
+
+@pytest.mark.parametrize("seed", range(12))
+def test_select_elo_matches_oracle(lib, seed):
+    g = np.random.default_rng(seed)
+    M = int(g.integers(1, 40))
+    quality = g.standard_normal(M)
+    scores = np.clip(np.round(5 + 2 * quality + g.standard_normal(M)), 1, 10).astype(np.int32)
+    noise = g.standard_normal((M, M))
+
+    def cmp(a, b):   # noisy, confidence from the margin
+        d = quality[a] - quality[b] + 0.3 * noise[a, b]
+        return d > 0, 0 if abs(d) > 1 else (1 if abs(d) > 0.3 else 2)
+    rho1, rho2, kappa = [(0.5, 0.5, 1.5), (1.0, 0.25, 3.0), (0.3, 1.0, 0.0)][seed % 3]
+    if seed == 5:
+        M, rho1 = 20, 0.3     # ceil(0.3 * 20) = 6 on both sides
+        scores, quality = scores[:M] if len(scores) >= M else np.resize(scores, M), \
+            np.resize(quality, M)
+        noise = np.resize(noise, (M, M))
+    w, r, calls = fb.fb_select_elo(scores, cmp, rho1, rho2, kappa)
+    w0, r0, calls0 = O.elo_select(scores, cmp, rho1, rho2, kappa)
+    assert (w, calls) == (w0, calls0)
+    np.testing.assert_allclose(r, r0, rtol=0, atol=1e-9)
+
+
+def test_select_elo_rejects_bad_confidence(lib):
+    with pytest.raises(fb.FlashBonError) as e:
+        fb.fb_select_elo([5, 6, 7], lambda a, b: (True, 5), 1.0, 1.0, 1.0)
+    assert e.value.status == fb.FB_EINVAL
+    with pytest.raises(fb.FlashBonError):
+        fb.fb_select_elo([5, 6], lambda a, b: (True, 0), 0.0, 1.0, 1.0)

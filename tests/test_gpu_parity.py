@@ -351,3 +351,33 @@ def test_guidance_and_sde_argument_errors(small4):
     with pytest.raises(fb.FlashBonError) as e:      # SDE without draws
         m.draft(z, ctx, sched, opts=fb.make_opts(sde_a=0.5))
     assert e.value.status == fb.FB_EINVAL
+
+
+def test_pipeline_draft_select_refine(small4):
+    """Stage 1 -> Stage 2 -> Stage 3 (§4.2): drafts on the GPU, a synthetic verifier (the
+    drafts' cosine to a hidden target; pairwise confidence from the margin) through the
+    library's Elo selection, and a full refine of the selected draft."""
+    cfg, w, m, ref = small4
+    n, S, Sp = 4, 6, 3
+    z = synth.make_latents(cfg, n)
+    ctx = synth.make_text(cfg)
+    sched = synth.make_schedule(S)
+    skip, proxy = synth.random_plan(Sp, cfg.depth, 1 / 3, 0.5, seed=11)
+    zd = cuda(z)
+    m.draft(zd, ctx, sched[:Sp + 1], skip, proxy)
+    drafts = zd.cpu().numpy().astype(np.float64)
+    target = synth.make_latents(cfg, 1, seed_base=99)[0].astype(np.float64).ravel()
+    q = np.array([d.ravel() @ target / np.linalg.norm(d) / np.linalg.norm(target)
+                  for d in drafts])
+    scores = np.clip(np.round(5 + 50 * q), 1, 10).astype(np.int32)
+
+    def cmp(a, b):
+        d = q[a] - q[b]
+        return d > 0, 0 if abs(d) > 0.02 else (1 if abs(d) > 0.005 else 2)
+    win, ratings, calls = fb.fb_select_elo(scores, cmp, 0.5, 0.5, 1.5)
+    assert win == O.elo_select(scores, cmp, 0.5, 0.5, 1.5)[0]
+    assert win == int(np.argmax(q))
+    r = zd[win].clone()
+    m.refine(r, ctx, sched[Sp:])
+    want = ref.refine(drafts[win], ctx, sched[Sp:])
+    check_latents(r.cpu().numpy(), want, drafts[win], label="refine of the selected draft")

@@ -421,3 +421,51 @@ def test_cfg_with_identical_contexts_is_unguided():
     a = m.draft(z, ctx, sched, sk, px)
     b = m.draft(z, ctx, sched, sk, px, ctx_uncond=ctx, guidance=4.0)
     np.testing.assert_allclose(a, b, rtol=1e-12, atol=1e-12)
+
+
+# -- NEXT row: multi-stage Elo selection (§4.2 Stage 2) -------------------------------------
+
+def test_elo_seed_values_from_the_paper():
+    assert O.elo_seed(5) == 1500.0 and O.elo_seed(10) == 2000.0 and O.elo_seed(1) == 1100.0
+
+
+def test_elo_update_hand_values():
+    # equal ratings: E = 1/2; high confidence K = 32 * 1.2 = 38.4 -> +/- 19.2
+    ra, rb = O.elo_update(1500.0, 1500.0, True, 32.0 * O.CONF_MULT[0])
+    assert (ra, rb) == (pytest.approx(1519.2), pytest.approx(1480.8))
+    # 400 points apart: E_a = 1/11; an upset with K = 32 moves a by 32 * 10/11
+    ra, rb = O.elo_update(1500.0, 1900.0, True, 32.0)
+    assert ra == pytest.approx(1500.0 + 32.0 * 10.0 / 11.0)
+    assert ra + rb == pytest.approx(3400.0)  # zero-sum
+
+
+def test_elo_select_call_counts_and_survivors():
+    """Defaults at M = 32: M1 = 16, C2 = 24 adjacent comparisons, M2 = 8, 28 tournament
+    games: 52 pairwise calls, the paper's 'roughly 3/2 M'."""
+    g = np.random.default_rng(0)
+    quality = g.standard_normal(32)
+    scores = np.clip(np.round(5 + 2 * quality), 1, 10).astype(int)
+    seen = []
+
+    def cmp(a, b):
+        seen.append((a, b))
+        return quality[a] > quality[b], 0
+    w, r, calls = O.elo_select(scores, cmp)
+    assert calls == 52 == len(seen)
+    assert len({x for p in seen for x in p}) <= 16          # only survivors of stage 1 play
+    assert w in {x for p in seen[24:] for x in p}           # the winner played the tournament
+
+
+def test_elo_select_finds_the_best_with_a_consistent_verifier():
+    g = np.random.default_rng(1)
+    for trial in range(20):
+        quality = g.standard_normal(24)
+        scores = np.clip(np.round(5 + 2 * quality), 1, 10).astype(int)
+        w, _, _ = O.elo_select(scores, lambda a, b: (quality[a] > quality[b], 1))
+        assert w == int(np.argmax(quality))
+
+
+def test_elo_select_ties_go_to_lower_index():
+    w, r, calls = O.elo_select([7, 7, 7, 7], lambda a, b: (a < b, 2), rho1=1.0, rho2=1.0,
+                               kappa=0.0)
+    assert w == 0 and calls == 6
