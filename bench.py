@@ -454,14 +454,16 @@ def run_probe(args):
 
 
 def probe_gemm_shapes(m, rnd, args):
-    """CUDA-event time of each block GEMM shape at the draft (N=32) and refine (N=1) row
-    counts, for the automatic kernel choice and the forced 1-SM kernel."""
+    """Per-launch time of each block GEMM shape at the draft (N=32) and refine (N=1) row
+    counts: `reps` back-to-back launches inside one call, timed with CUDA events on the
+    library's stream (fb_get_stats), for the automatic choice and the forced 1-SM kernel."""
     import torch
     from paper_2607_04461_gb300 import flashbon as fb
     D, F = 1536, 8960
     shapes = {"qkv": (3 * D, D, 0), "out": (D, D, 2), "cross_q": (D, D, 0),
               "cross_out": (D, D, 2), "ffn_up": (F, D, 1), "ffn_down": (D, F, 3)}
     res = {}
+    reps = max(5, args.steps)
     for M in (49920, 1560):
         for name, (N, K, epi) in shapes.items():
             A, W, b = rnd(M, K), rnd(N, K), rnd(N, dt=torch.float32)
@@ -472,20 +474,18 @@ def probe_gemm_shapes(m, rnd, args):
                 f = lambda: fb.fb_op_gemm(m.handle, M, N, K, A, W, b, epi, out, r, b if epi >= 2 else None,  # noqa
                                           r if epi == 3 else None, dl, impl)
                 f()
-                torch.cuda.synchronize()
-                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-                n = max(3, args.steps)
-                e0.record()
-                for _ in range(n):
-                    f()
-                e1.record()
-                torch.cuda.synchronize()
-                ms = e0.elapsed_time(e1) / n
+                fb.fb_set_op_repeat(m.handle, reps)
+                m.reset_stats()
+                m.set_timing(1 << fb.K["gemm_tc"])
+                f()
+                m.set_timing(0)
+                fb.fb_set_op_repeat(m.handle, 1)
+                st = m.stats()["gemm_tc"]
+                us = st["ms"] * 1e3 / st["launches"]
                 res[f"M{M}/{name}/{'auto' if impl == 0 else '1sm'}"] = {
-                    "ms": round(ms, 4), "tflops": round(2 * M * N * K / ms / 1e9, 1)}
+                    "us": round(us, 2), "tflops": round(2 * M * N * K / us / 1e6, 1)}
             del A, W, out, r, dl
-    print(json.dumps({"probe": "gemm_shapes", "note": "each call includes one stream sync",
-                      "res": res}))
+    print(json.dumps({"probe": "gemm_shapes", "res": res}))
     return 0
 
 

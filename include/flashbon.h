@@ -222,6 +222,9 @@ const char* fb_kernel_name(int kind);
  * dimension N. impl: 0 = automatic (tcgen05 when N % 128 == 0 and K % 64 == 0: the
  * 2-SM cta_group::2 kernel when N % 256 == 0, else the 1-SM kernel), 1 = force the
  * CUDA-core kernel, 2 = force the 1-SM tcgen05 kernel (same shape rules). */
+/* fb_set_op_repeat: fb_op_gemm / fb_op_attention launch their kernel n >= 1 times back
+ * to back (default 1), for timing a kernel without a stream synchronisation per launch. */
+fb_status fb_set_op_repeat(fb_model* m, int n);
 fb_status fb_op_gemm(fb_model* m, int M, int N, int K, const void* A, const void* W,
                      const float* bias, int epi, void* out, const float* resid,
                      const float* gate, const float* base, void* delta, int impl);

@@ -171,6 +171,7 @@ struct fb_model {
   int* herr = nullptr;  // pinned
   // statistics
   unsigned timing_mask = 0;
+  int op_repeat = 1;
   fb_kstat stats[FB_K_COUNT];
   std::vector<Pending> pending;
   std::vector<cudaEvent_t> ev_pool;
@@ -995,7 +996,7 @@ fb_status fb_op_gemm(fb_model* m, int M, int N, int K, const void* A, const void
   g.epi.delta = (bf16*)delta;
   CKS(begin_call(m));
   if (impl < 0 || impl > 2) return fail(FB_EINVAL, "impl must be 0, 1 or 2");
-  CKS(run_gemm(m, g, impl));
+  for (int r = 0; r < m->op_repeat; ++r) CKS(run_gemm(m, g, impl));
   return end_call(m);
 }
 
@@ -1012,8 +1013,14 @@ fb_status fb_op_attention(fb_model* m, const void* Q, int ldq, const void* K, in
   a.batch = batch; a.Lq = Lq; a.Lkv = Lkv; a.kv_batch_rows = kv_batch_rows;
   a.heads = heads; a.head_dim = head_dim;
   CKS(begin_call(m));
-  CKS(run_attn(m, a, FB_K_ATTN_SELF, impl));
+  for (int r = 0; r < m->op_repeat; ++r) CKS(run_attn(m, a, FB_K_ATTN_SELF, impl));
   return end_call(m);
+}
+
+fb_status fb_set_op_repeat(fb_model* m, int n) {
+  if (!m || n < 1) return fail(FB_EINVAL, "model is NULL or n < 1");
+  m->op_repeat = n;
+  return FB_OK;
 }
 
 }  // extern "C"

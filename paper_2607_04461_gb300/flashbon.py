@@ -49,7 +49,8 @@ class fb_kstat(ctypes.Structure):
 EXPORTS = ["fb_weights_count", "fb_weights_entry", "fb_init_model", "fb_free", "fb_set_stream",
            "fb_encode_text", "fb_draft", "fb_refine", "fb_plan_from_phi", "fb_block_forward",
            "fb_last_error", "fb_set_timing", "fb_get_stats", "fb_reset_stats", "fb_kernel_name",
-           "fb_op_gemm", "fb_op_attention", "fb_draft_ex", "fb_refine_ex", "fb_select_elo"]
+           "fb_op_gemm", "fb_op_attention", "fb_draft_ex", "fb_refine_ex", "fb_select_elo",
+           "fb_set_op_repeat"]
 
 PAIR_VERIFIER = ctypes.CFUNCTYPE(ctypes.c_int, ctypes.c_void_p, ctypes.c_int, ctypes.c_int,
                                  ctypes.POINTER(ctypes.c_int))
@@ -84,6 +85,7 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
         "fb_block_forward": (I, [P, I, P, I, F]),
         "fb_last_error": (ctypes.c_char_p, []),
         "fb_set_timing": (I, [P, I]),
+        "fb_set_op_repeat": (I, [P, I]),
         "fb_get_stats": (I, [P, P]),
         "fb_reset_stats": (I, [P]),
         "fb_kernel_name": (ctypes.c_char_p, [I]),
@@ -252,6 +254,10 @@ def fb_block_forward(model: int, layer: int, h, n: int, t: float) -> None:
 
 def fb_set_timing(model: int, mask: int) -> None:
     _check(load_library().fb_set_timing(model, int(mask)))
+
+
+def fb_set_op_repeat(model: int, n: int) -> None:
+    _check(load_library().fb_set_op_repeat(model, int(n)))
 
 
 def fb_get_stats(model: int) -> dict:
