@@ -303,18 +303,24 @@ template <int KIND>
 __device__ __forceinline__ void epi_apply32(const GemmEpi& e, int row, int col, float* v) {
   const size_t off = (size_t)row * e.ldo + col;
   if (KIND >= EPI_RESID) {
-    float r[32], g[32], b[32], bs[32];
+    // the row-dependent operands (HBM) first; gate and bias are the same for every row
+    // (L1-resident) and are read per 8 columns while computing
+    float r[32], bs[32];
 #pragma unroll
     for (int j = 0; j < 32; j += 8) {
       load_f32x8(e.resid + off + j, r + j);
-      if (e.gate) load_f32x8(e.gate + col + j, g + j);
-      if (e.bias) load_f32x8(e.bias + col + j, b + j);
       if (KIND == EPI_RESID_DELTA) load_f32x8(e.base + off + j, bs + j);
     }
 #pragma unroll
-    for (int j = 0; j < 32; ++j) {
-      const float a = v[j] + (e.bias ? b[j] : 0.f);
-      v[j] = r[j] + (e.gate ? g[j] : 1.f) * a;
+    for (int j = 0; j < 32; j += 8) {
+      float g[8], b[8];
+      if (e.gate) load_f32x8(e.gate + col + j, g);
+      if (e.bias) load_f32x8(e.bias + col + j, b);
+#pragma unroll
+      for (int q = 0; q < 8; ++q) {
+        const float a = v[j + q] + (e.bias ? b[q] : 0.f);
+        v[j + q] = r[j + q] + (e.gate ? g[q] : 1.f) * a;
+      }
     }
     if (KIND == EPI_RESID_DELTA) {
 #pragma unroll

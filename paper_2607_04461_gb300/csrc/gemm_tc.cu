@@ -10,10 +10,12 @@
 //  * warp 1: allocates 2*BN TMEM columns (two fp32 accumulators of 128 lanes x BN);
 //    one thread issues tcgen05.mma (M=128, N=BN, K=16, bf16 -> fp32), commits each
 //    stage back to its "empty" barrier and each finished tile to "tmem_full".
-//  * warps 2-5: epilogue. Warp w reads TMEM lanes 32*(w%4).. (its lane quarter) with
-//    tcgen05.ld, applies bias / GELU / gated residual / contribution write, stores to
-//    global, and releases the accumulator ("tmem_empty") so that the MMA of the tile
-//    after next can start while this epilogue runs.
+//  * warps 2-9: epilogue. Warp w reads TMEM lanes 32*(w%4).. (its lane quarter) and one
+//    half of the tile's columns ((w-2)/4) with tcgen05.ld, applies bias / GELU / gated
+//    residual / contribution write, stores to global, and releases the accumulator
+//    ("tmem_empty") so that the MMA of the tile after next can start while this
+//    epilogue runs. Two warps per lane quarter keep twice the epilogue's loads in
+//    flight, which the fp32 residual epilogues need to keep up with the mainloop.
 // Every mbarrier wait is bounded (mbar_wait): on timeout the kernel records the error,
 // stops issuing work, waits (bounded) for its own TMA loads, frees TMEM and returns.
 #include <cudaTypedefs.h>
@@ -24,7 +26,8 @@ namespace {
 
 constexpr int BM = 128;
 constexpr int BK = 64;  // 64 bf16 = 128 bytes: one swizzle row
-constexpr int NUM_THREADS = 192;
+constexpr int NUM_THREADS = 320;       // producer, MMA, 8 epilogue warps
+constexpr int EPI_THREADS = 256;
 
 template <int BN>
 struct TcCfg {
@@ -83,7 +86,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(&tmem_full[a], 1);
-      mbar_init(&tmem_empty[a], 128);
+      mbar_init(&tmem_empty[a], EPI_THREADS);
     }
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     tma_prefetch_desc(&tmA);
@@ -161,8 +164,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       }
     }
   } else {
-    // ---------------- epilogue (warps 2..5) ----------------
-    const int quarter = warp & 3;
+    // ---------------- epilogue (warps 2..9) ----------------
+    const int quarter = warp & 3, half = (warp - 2) >> 2;
     int it = 0;
     for (int tile = blockIdx.x; tile < n_tiles; tile += gridDim.x, ++it) {
       const int acc = it & 1;
@@ -176,7 +179,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       const int row = m0 + quarter * 32 + lane;
       const uint32_t taddr = tmem_base + ((uint32_t)(quarter * 32) << 16) + acc * BN;
 #pragma unroll 1
-      for (int c = 0; c < BN / 32; ++c) {
+      for (int c = half * (BN / 64); c < (half + 1) * (BN / 64); ++c) {
         uint32_t r[32];
         tmem_ld32(taddr + c * 32, r);
         tmem_ld_wait();
@@ -243,7 +246,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(&tmem_full[a], 1);
-      mbar_init(&tmem_empty[a], 8);  // 4 epilogue warps x 2 CTAs
+      mbar_init(&tmem_empty[a], 16);  // 8 epilogue warps x 2 CTAs
     }
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     tma_prefetch_desc(&tmA);
@@ -304,8 +307,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
       }
     }
   } else {
-    // ---------------- epilogue (warps 2..5 of both CTAs) ----------------
-    const int quarter = warp & 3;
+    // ---------------- epilogue (warps 2..9 of both CTAs) ----------------
+    const int quarter = warp & 3, half = (warp - 2) >> 2;
     const uint32_t te_remote = mapa_shared(smem_u32(&tmem_empty[0]), 0);
     int it = 0;
     for (int tile = cluster; tile < n_tiles; tile += n_clusters, ++it) {
@@ -318,7 +321,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
       const int row = m0 + BM * (int)rank + quarter * 32 + lane;
       const uint32_t taddr = tmem_base + ((uint32_t)(quarter * 32) << 16) + acc * C2_BN;
 #pragma unroll 1
-      for (int c = 0; c < C2_BN / 32; ++c) {
+      for (int c = half * (C2_BN / 64); c < (half + 1) * (C2_BN / 64); ++c) {
         uint32_t r[32];
         tmem_ld32(taddr + c * 32, r);
         tmem_ld_wait();
