@@ -282,6 +282,13 @@ __device__ __forceinline__ void tc_commit_mc(uint64_t* bar, uint16_t cta_mask) {
       : "memory");
 }
 
+// Bulk prefetch of [p, p + bytes) into L2 (p and bytes multiples of 16).
+__device__ __forceinline__ void prefetch_l2_bulk(const void* p, uint32_t bytes) {
+  asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(reinterpret_cast<uint64_t>(p)),
+               "r"(bytes)
+               : "memory");
+}
+
 // ---- GEMM epilogue (shared by the tcgen05 and CUDA-core GEMMs) --------------------
 enum { EPI_BF16 = 0, EPI_GELU_BF16 = 1, EPI_RESID = 2, EPI_RESID_DELTA = 3 };
 
@@ -294,6 +301,17 @@ struct GemmEpi {
   bf16* delta;         // bf16 [M][ldo] (EPI_RESID_DELTA)
   int ldo;
 };
+
+// Residual epilogues read fp32 rows from HBM; the epilogue warps prefetch their part of
+// the next tile's rows into L2 while the mainloop runs, so those reads hit L2.
+template <int KIND>
+__device__ __forceinline__ void epi_prefetch(const GemmEpi& e, int row, int col, int ncols) {
+  if (KIND >= EPI_RESID) {
+    const size_t off = (size_t)row * e.ldo + col;
+    prefetch_l2_bulk(e.resid + off, ncols * 4);
+    if (KIND == EPI_RESID_DELTA && e.base != e.resid) prefetch_l2_bulk(e.base + off, ncols * 4);
+  }
+}
 
 // Applies the epilogue to 32 consecutive accumulators v of row `row`, columns
 // col..col+31. Every global load of the chunk is issued before its first store (out may

@@ -171,6 +171,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       const int acc = it & 1;
       const uint32_t acc_phase = (it >> 1) & 1;
       const int m0 = (tile / n_nt) * BM, n0 = (tile % n_nt) * BN;
+      if (m0 + quarter * 32 + lane < M)
+        epi_prefetch<KIND>(epi, m0 + quarter * 32 + lane, n0 + half * (BN / 2), BN / 2);
       // every lane waits; the warp leaves together if any lane gave up, so the
       // .sync.aligned tcgen05.ld below is always executed by the whole warp
       const bool ok = mbar_wait(&tmem_full[acc], acc_phase, err);
@@ -315,6 +317,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
       const int acc = it & 1;
       const uint32_t acc_phase = (it >> 1) & 1;
       const int m0 = (tile / n_nt) * 2 * BM, n0 = (tile % n_nt) * C2_BN;
+      const int prow = m0 + BM * (int)rank + quarter * 32 + lane;
+      if (prow < M) epi_prefetch<KIND>(epi, prow, n0 + half * (C2_BN / 2), C2_BN / 2);
       const bool ok = mbar_wait(&tmem_full[acc], acc_phase, err);
       if (!__all_sync(0xffffffffu, ok)) { failed = true; break; }
       tc_fence_after();
