@@ -215,20 +215,67 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
 // the "empty" / "tmem_full" barriers of both CTAs, and both CTAs' epilogue warps release
 // an accumulator on its "tmem_empty" barrier.
 constexpr int C2_BN = 256;
-constexpr int C2_STAGES = 6;
 constexpr int C2_HALF_BYTES = 128 * BK * 2;          // 16 KB: 128 rows x 64 bf16
 constexpr int C2_STAGE_BYTES = 2 * C2_HALF_BYTES;    // this CTA's A rows + W rows
 constexpr int C2_TMEM_COLS = 2 * C2_BN;
-constexpr int C2_SMEM_BYTES = C2_STAGES * C2_STAGE_BYTES + 1024 + 256;
+// fp32 residual epilogues stage each 32 x 32 accumulator chunk in shared memory (one
+// [32][33] float tile per epilogue warp) so that their global loads and stores are
+// whole 128-byte rows; that space comes out of the operand ring (5 stages instead of 6).
+constexpr int EPI_STAGE_FLOATS = 32 * 33;
+template <int KIND>
+struct C2Cfg {
+  static constexpr bool STAGED = KIND >= EPI_RESID;
+  static constexpr int STAGES = STAGED ? 5 : 6;
+  static constexpr int EPI_BYTES = STAGED ? 8 * EPI_STAGE_FLOATS * 4 : 0;
+  static constexpr int SMEM_BYTES = STAGES * C2_STAGE_BYTES + EPI_BYTES + 1024 + 256;
+};
+
+// Staged residual epilogue of one warp for one 32 x 32 chunk: rows row0..row0+31 (the
+// warp's TMEM lane quarter), columns col0..col0+31; acc holds the thread's row (lane).
+template <int KIND>
+__device__ __forceinline__ void epi_resid_staged(const GemmEpi& e, float* stg, int lane,
+                                                 int row0, int col0, int M, const float* acc) {
+#pragma unroll
+  for (int j = 0; j < 32; ++j) stg[lane * 33 + j] = acc[j];
+  __syncwarp();
+  const int col = col0 + lane;
+  const float g = e.gate ? e.gate[col] : 1.f;
+  const float b = e.bias ? e.bias[col] : 0.f;
+#pragma unroll 1
+  for (int r0 = 0; r0 < 32; r0 += 8) {
+    float rv[8], bv[8];
+#pragma unroll
+    for (int q = 0; q < 8; ++q) {
+      const int row = row0 + r0 + q;
+      const size_t off = (size_t)row * e.ldo + col;
+      rv[q] = row < M ? e.resid[off] : 0.f;
+      if (KIND == EPI_RESID_DELTA) bv[q] = row < M ? e.base[off] : 0.f;
+    }
+#pragma unroll
+    for (int q = 0; q < 8; ++q) {
+      const int row = row0 + r0 + q;
+      if (row < M) {
+        const size_t off = (size_t)row * e.ldo + col;
+        const float o = rv[q] + g * (stg[(r0 + q) * 33 + lane] + b);
+        if (KIND == EPI_RESID_DELTA) e.delta[off] = __float2bfloat16_rn(o - bv[q]);
+        reinterpret_cast<float*>(e.out)[off] = o;
+      }
+    }
+  }
+  __syncwarp();
+}
 
 template <int KIND>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
     gemm_tc2_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmW,
                     int M, int N, int K, GemmEpi epi, int* err) {
+  using CC = C2Cfg<KIND>;
+  constexpr int C2_STAGES = CC::STAGES;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  uint64_t* full = reinterpret_cast<uint64_t*>(smem + C2_STAGES * C2_STAGE_BYTES);
+  float* epi_stage = reinterpret_cast<float*>(smem + C2_STAGES * C2_STAGE_BYTES);
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + C2_STAGES * C2_STAGE_BYTES + CC::EPI_BYTES);
   uint64_t* empty = full + C2_STAGES;
   uint64_t* tmem_full = empty + C2_STAGES;
   uint64_t* tmem_empty = tmem_full + 2;
@@ -322,17 +369,22 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
       const bool ok = mbar_wait(&tmem_full[acc], acc_phase, err);
       if (!__all_sync(0xffffffffu, ok)) { failed = true; break; }
       tc_fence_after();
-      const int row = m0 + BM * (int)rank + quarter * 32 + lane;
+      const int row0 = m0 + BM * (int)rank + quarter * 32;
+      const int row = row0 + lane;
       const uint32_t taddr = tmem_base + ((uint32_t)(quarter * 32) << 16) + acc * C2_BN;
 #pragma unroll 1
       for (int c = half * (C2_BN / 64); c < (half + 1) * (C2_BN / 64); ++c) {
         uint32_t r[32];
         tmem_ld32(taddr + c * 32, r);
         tmem_ld_wait();
-        if (row < M) {
-          float v[32];
+        float v[32];
 #pragma unroll
-          for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(r[j]);
+        for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(r[j]);
+        if (CC::STAGED) {
+          if (row0 < M)
+            epi_resid_staged<KIND>(epi, epi_stage + (warp - 2) * EPI_STAGE_FLOATS, lane, row0,
+                                   n0 + c * 32, M, v);
+        } else if (row < M) {
           epi_apply32<KIND>(epi, row, n0 + c * 32, v);
         }
       }
@@ -415,6 +467,7 @@ cudaError_t launch2(const GemmArgs& g, int* err, int num_sms, cudaStream_t st) {
   CUtensorMap ma, mw;
   if (!make_map(&ma, g.A, g.M, g.K, g.lda, BM) || !make_map(&mw, g.W, g.N, g.K, g.ldw, 128))
     return cudaErrorInvalidValue;
+  constexpr int C2_SMEM_BYTES = C2Cfg<KIND>::SMEM_BYTES;
   cudaError_t e = cudaFuncSetAttribute(gemm_tc2_kernel<KIND>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, C2_SMEM_BYTES);
   if (e != cudaSuccess) return e;
