@@ -241,18 +241,20 @@ __device__ __forceinline__ void epi_resid_staged(const GemmEpi& e, float* stg, i
   const int col = col0 + lane;
   const float g = e.gate ? e.gate[col] : 1.f;
   const float b = e.bias ? e.bias[col] : 0.f;
+  // all 32 rows' loads in flight before the first store (one memory latency per chunk)
+  constexpr int NB = KIND == EPI_RESID_DELTA ? 16 : 32;
 #pragma unroll 1
-  for (int r0 = 0; r0 < 32; r0 += 8) {
-    float rv[8], bv[8];
+  for (int r0 = 0; r0 < 32; r0 += NB) {
+    float rv[NB], bv[NB];
 #pragma unroll
-    for (int q = 0; q < 8; ++q) {
+    for (int q = 0; q < NB; ++q) {
       const int row = row0 + r0 + q;
       const size_t off = (size_t)row * e.ldo + col;
       rv[q] = row < M ? e.resid[off] : 0.f;
       if (KIND == EPI_RESID_DELTA) bv[q] = row < M ? e.base[off] : 0.f;
     }
 #pragma unroll
-    for (int q = 0; q < 8; ++q) {
+    for (int q = 0; q < NB; ++q) {
       const int row = row0 + r0 + q;
       if (row < M) {
         const size_t off = (size_t)row * e.ldo + col;
