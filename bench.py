@@ -409,7 +409,8 @@ def run_probe(args):
     """A few launches of one kernel on a case sized for an ncu capture (inputs larger
     than L2, a few hundred MB on the device): gemm = the FFN up-projection shape
     (8192 x 1536 -> 8960, GELU epilogue); gemm_resid = FFN down (8192 x 8960 -> 1536,
-    gated residual + contribution write); attn = self-attention over 1560 tokens,
+    gated residual + contribution write); gemm_out = attention output projection
+    (8192 x 1536 -> 1536, gated fp32 residual); attn = self-attention over 1560 tokens,
     4 candidates x 12 heads x 128."""
     import torch
     from paper_2607_04461_gb300 import flashbon as fb
@@ -420,6 +421,12 @@ def run_probe(args):
     rnd = lambda *s, dt=torch.bfloat16: (torch.randn(*s, generator=g) * 0.5).to(dt).cuda()  # noqa
     if args.probe in ("gemm_shapes", "breakdown"):
         call = None
+    elif args.probe == "gemm_out":
+        M, D = 8192, 1536
+        A, W, b = rnd(M, D), rnd(D, D), rnd(D, dt=torch.float32)
+        h, gt = rnd(M, D, dt=torch.float32), rnd(D, dt=torch.float32)
+        out = torch.empty(M, D, dtype=torch.float32, device="cuda")
+        call = lambda: fb.fb_op_gemm(m.handle, M, D, D, A, W, b, 2, out, h, gt)  # noqa
     elif args.probe in ("gemm", "gemm_resid"):
         M, D, F = 8192, 1536, 8960
         if args.probe == "gemm":
@@ -539,8 +546,8 @@ def main():
     ap.add_argument("--variant", choices=list(VARIANTS), default="base",
                     help="base: the draft-pool workload; cfg / sde: the same with guidance "
                          "or SDE steps")
-    ap.add_argument("--probe", choices=["gemm", "gemm_resid", "attn", "attn_mma", "gemm_shapes",
-                                        "breakdown"],
+    ap.add_argument("--probe", choices=["gemm", "gemm_resid", "gemm_out", "attn", "attn_mma",
+                                        "gemm_shapes", "breakdown"],
                     default=None)
     args = ap.parse_args()
     if args.probe:
