@@ -171,7 +171,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       const int acc = it & 1;
       const uint32_t acc_phase = (it >> 1) & 1;
       const int m0 = (tile / n_nt) * BM, n0 = (tile % n_nt) * BN;
-      if (m0 + quarter * 32 + lane < M)
+      // short-K tiles only: over a long mainloop the streamed operands evict the rows
+      if (nk <= 48 && m0 + quarter * 32 + lane < M)
         epi_prefetch<KIND>(epi, m0 + quarter * 32 + lane, n0 + half * (BN / 2), BN / 2);
       // every lane waits; the warp leaves together if any lane gave up, so the
       // .sync.aligned tcgen05.ld below is always executed by the whole warp
@@ -242,7 +243,7 @@ __device__ __forceinline__ void epi_resid_staged(const GemmEpi& e, float* stg, i
   const float g = e.gate ? e.gate[col] : 1.f;
   const float b = e.bias ? e.bias[col] : 0.f;
   // all 32 rows' loads in flight before the first store (one memory latency per chunk)
-  constexpr int NB = KIND == EPI_RESID_DELTA ? 16 : 32;
+  constexpr int NB = 32;
 #pragma unroll 1
   for (int r0 = 0; r0 < 32; r0 += NB) {
     float rv[NB], bv[NB];
@@ -367,7 +368,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
       const uint32_t acc_phase = (it >> 1) & 1;
       const int m0 = (tile / n_nt) * 2 * BM, n0 = (tile % n_nt) * C2_BN;
       const int prow = m0 + BM * (int)rank + quarter * 32 + lane;
-      if (prow < M) epi_prefetch<KIND>(epi, prow, n0 + half * (C2_BN / 2), C2_BN / 2);
+      // short-K tiles only: over a long mainloop the streamed operands evict the rows
+      if (nk <= 48 && prow < M) epi_prefetch<KIND>(epi, prow, n0 + half * (C2_BN / 2), C2_BN / 2);
       const bool ok = mbar_wait(&tmem_full[acc], acc_phase, err);
       if (!__all_sync(0xffffffffu, ok)) { failed = true; break; }
       tc_fence_after();
