@@ -243,7 +243,7 @@ __device__ __forceinline__ void epi_resid_staged(const GemmEpi& e, float* stg, i
   const float g = e.gate ? e.gate[col] : 1.f;
   const float b = e.bias ? e.bias[col] : 0.f;
   // all 32 rows' loads in flight before the first store (one memory latency per chunk)
-  constexpr int NB = 32;
+  constexpr int NB = KIND == EPI_RESID_DELTA ? 16 : 32;  // Delta: 32 would spill
 #pragma unroll 1
   for (int r0 = 0; r0 < 32; r0 += NB) {
     float rv[NB], bv[NB];
