@@ -2,8 +2,10 @@
 // O = softmax(Q K^T / sqrt(128)) V per (batch, head), non-causal, ragged tails masked.
 //
 // One CTA = one 128-query tile of one (batch, head); 6 warps:
-//  * warp 0, one thread: TMA producer. Q once (2 x [128 rows][64 cols] boxes), then
-//    128-key K and V tiles into a 2-deep ring (64 KB per stage), 128-byte swizzle.
+//  * warp 0: TMA producers. Lane 0 loads Q once (2 x [128 rows][64 cols] boxes) and then
+//    128-key K tiles into a 3-slot ring; lane 1 loads the V tiles into a 2-slot ring
+//    (128-byte swizzle). A K slot is released as soon as the S MMA that read it is done,
+//    a V slot when its PV MMA is done, so K tiles load up to two tiles ahead.
 //  * warp 1: TMEM owner (512 columns: S0, S1, O) and, one thread, the MMA issuer:
 //    S_j = Q K_j^T into S[j % 2] (M=128, N=128 keys, K=128, both operands K-major),
 //    then, once the softmax has written P_j, O += P_j V_j (A = P from shared memory,
@@ -24,10 +26,11 @@ namespace {
 constexpr int TB = 128;                    // queries per CTA = keys per KV tile
 constexpr int SUB = TB * 64 * 2;           // 16 KB: 128 rows x 64 bf16 (one swizzle width)
 constexpr int Q_BYTES = 2 * SUB;           // 32 KB
-constexpr int KV_BYTES = 4 * SUB;          // K (2 sub-tiles) + V (2 sub-tiles)
+constexpr int K_BYTES = 2 * SUB;           // one K tile (2 sub-tiles of 64 columns)
+constexpr int V_BYTES = 2 * SUB;           // one V tile
 constexpr int P_BYTES = 2 * SUB;
-constexpr int NSTAGE = 2;
-constexpr int SMEM_BYTES = Q_BYTES + NSTAGE * KV_BYTES + P_BYTES + 1024 + 256;
+constexpr int KSLOT = 3, VSLOT = 2;        // K and V ring depths
+constexpr int SMEM_BYTES = Q_BYTES + KSLOT * K_BYTES + VSLOT * V_BYTES + P_BYTES + 1024 + 256;
 constexpr int THREADS = 192;
 constexpr uint32_t TMEM_COLS = 512;        // S0 [0,128), S1 [128,256), O [256,384)
 constexpr uint32_t O_COL = 256;
@@ -91,16 +94,19 @@ __global__ void __launch_bounds__(THREADS, 1)
   uint8_t* smem = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* Qs = smem;
-  uint8_t* KVs = smem + Q_BYTES;
-  uint8_t* Ps = KVs + NSTAGE * KV_BYTES;
+  uint8_t* Ks = smem + Q_BYTES;
+  uint8_t* Vs = Ks + KSLOT * K_BYTES;
+  uint8_t* Ps = Vs + VSLOT * V_BYTES;
   uint64_t* bars = reinterpret_cast<uint64_t*>(Ps + P_BYTES);
   uint64_t* q_full = bars;
-  uint64_t* kv_full = bars + 1;       // [2]
-  uint64_t* kv_empty = bars + 3;      // [2]
-  uint64_t* s_full = bars + 5;        // [2]
-  uint64_t* p_full = bars + 7;
-  uint64_t* o_done = bars + 8;
-  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(bars + 9);
+  uint64_t* k_full = bars + 1;        // [3]
+  uint64_t* k_empty = bars + 4;       // [3]
+  uint64_t* v_full = bars + 7;        // [2]
+  uint64_t* v_empty = bars + 9;       // [2]
+  uint64_t* s_full = bars + 11;       // [2]
+  uint64_t* p_full = bars + 13;
+  uint64_t* o_done = bars + 14;
+  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(bars + 15);
 
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
   const int qt = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
@@ -112,9 +118,13 @@ __global__ void __launch_bounds__(THREADS, 1)
 
   if (threadIdx.x == 0) {
     mbar_init(q_full, 1);
-    for (int s = 0; s < NSTAGE; ++s) {
-      mbar_init(&kv_full[s], 1);
-      mbar_init(&kv_empty[s], 1);
+    for (int s = 0; s < KSLOT; ++s) {
+      mbar_init(&k_full[s], 1);
+      mbar_init(&k_empty[s], 1);
+    }
+    for (int s = 0; s < 2; ++s) {
+      mbar_init(&v_full[s], 1);
+      mbar_init(&v_empty[s], 1);
       mbar_init(&s_full[s], 1);
     }
     mbar_init(p_full, 4);   // one arrival per softmax warp
@@ -133,22 +143,30 @@ __global__ void __launch_bounds__(THREADS, 1)
   griddep_launch();
 
   if (warp == 0) {
+    // ---------------- TMA producers: lane 0 Q and K, lane 1 V ----------------
+    const int xq = h * 128;
     if (lane == 0) {
-      // ---------------- TMA producer ----------------
-      const int xq = h * 128;
       mbar_expect_tx(q_full, Q_BYTES);
       tma_load_2d(Qs, &tmQ, q_full, xq, q_row0);
       tma_load_2d(Qs + SUB, &tmQ, q_full, xq + 64, q_row0);
       for (int j = 0; j < n_kv; ++j) {
-        const int s = j & 1;
-        if (!mbar_wait(&kv_empty[s], ((j >> 1) & 1) ^ 1u, err)) { failed = true; break; }
-        uint8_t* st = KVs + s * KV_BYTES;
+        const int s = j % KSLOT;
+        if (!mbar_wait(&k_empty[s], ((j / KSLOT) & 1) ^ 1u, err)) { failed = true; break; }
+        uint8_t* st = Ks + s * K_BYTES;
         const int y = kv_row0 + j * TB;
-        mbar_expect_tx(&kv_full[s], KV_BYTES);
-        tma_load_2d(st, &tmK, &kv_full[s], xq, y);
-        tma_load_2d(st + SUB, &tmK, &kv_full[s], xq + 64, y);
-        tma_load_2d(st + 2 * SUB, &tmV, &kv_full[s], xq, y);
-        tma_load_2d(st + 3 * SUB, &tmV, &kv_full[s], xq + 64, y);
+        mbar_expect_tx(&k_full[s], K_BYTES);
+        tma_load_2d(st, &tmK, &k_full[s], xq, y);
+        tma_load_2d(st + SUB, &tmK, &k_full[s], xq + 64, y);
+      }
+    } else if (lane == 1) {
+      for (int j = 0; j < n_kv; ++j) {
+        const int s = j & 1;
+        if (!mbar_wait(&v_empty[s], ((j >> 1) & 1) ^ 1u, err)) { failed = true; break; }
+        uint8_t* st = Vs + s * V_BYTES;
+        const int y = kv_row0 + j * TB;
+        mbar_expect_tx(&v_full[s], V_BYTES);
+        tma_load_2d(st, &tmV, &v_full[s], xq, y);
+        tma_load_2d(st + SUB, &tmV, &v_full[s], xq + 64, y);
       }
     }
   } else if (warp == 1) {
@@ -159,7 +177,7 @@ __global__ void __launch_bounds__(THREADS, 1)
       const uint32_t idesc_pv = idesc_s | (1u << 16);  // B (V) is MN-major
       const uint32_t qa = smem_u32(Qs), pa = smem_u32(Ps);
       auto issue_s = [&](int j) {
-        const uint32_t ka = smem_u32(KVs + (j & 1) * KV_BYTES);
+        const uint32_t ka = smem_u32(Ks + (j % KSLOT) * K_BYTES);
 #pragma unroll
         for (int kk = 0; kk < 8; ++kk) {
           const uint32_t off = (kk >> 2) * SUB + (kk & 3) * 32;
@@ -167,26 +185,28 @@ __global__ void __launch_bounds__(THREADS, 1)
                      kk ? 1u : 0u);
         }
         tc_commit(&s_full[j & 1]);
+        tc_commit(&k_empty[j % KSLOT]);  // K_j is no longer needed once S_j is done
       };
-      if (mbar_wait(q_full, 0, err) && mbar_wait(&kv_full[0], 0, err)) {
+      if (mbar_wait(q_full, 0, err) && mbar_wait(&k_full[0], 0, err)) {
         tc_fence_after();
         issue_s(0);
         for (int j = 0; j < n_kv; ++j) {
           if (j + 1 < n_kv) {
-            if (!mbar_wait(&kv_full[(j + 1) & 1], ((j + 1) >> 1) & 1, err)) { failed = true; break; }
+            if (!mbar_wait(&k_full[(j + 1) % KSLOT], ((j + 1) / KSLOT) & 1, err)) { failed = true; break; }
             tc_fence_after();
             issue_s(j + 1);
           }
           if (!mbar_wait(p_full, j & 1, err)) { failed = true; break; }
+          if (!mbar_wait(&v_full[j & 1], (j >> 1) & 1, err)) { failed = true; break; }
           tc_fence_after();
-          const uint32_t va = smem_u32(KVs + (j & 1) * KV_BYTES + 2 * SUB);
+          const uint32_t va = smem_u32(Vs + (j & 1) * V_BYTES);
 #pragma unroll
           for (int kk = 0; kk < 8; ++kk) {
             const uint32_t off = (kk >> 2) * SUB + (kk & 3) * 32;
             tc_mma_f16(tmem + O_COL, desc_k_sw128(pa + off), desc_mn_sw128(va + kk * 2048, SUB),
                        idesc_pv, (j | kk) ? 1u : 0u);
           }
-          tc_commit(&kv_empty[j & 1]);
+          tc_commit(&v_empty[j & 1]);
           tc_commit(o_done);
         }
       } else {
@@ -318,7 +338,7 @@ __global__ void __launch_bounds__(THREADS, 1)
 // after PV_A(j) has read it, and the commit that announces S_g(j+1) also covers PV_g(j)
 // (the softmax may then rescale O_g).
 constexpr int THREADS2 = 320;
-constexpr int SMEM2_BYTES = 2 * Q_BYTES + NSTAGE * KV_BYTES + 1024 + 256;
+constexpr int SMEM2_BYTES = 2 * Q_BYTES + KSLOT * K_BYTES + VSLOT * V_BYTES + 1024 + 256;
 
 __device__ __forceinline__ void tc_mma_f16_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t bdesc,
                                               uint32_t idesc, uint32_t accumulate) {
@@ -337,15 +357,18 @@ __global__ void __launch_bounds__(THREADS2, 1)
   uint8_t* smem = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* Qs = smem;                  // [2 tiles][2 sub-tiles]
-  uint8_t* KVs = smem + 2 * Q_BYTES;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(KVs + NSTAGE * KV_BYTES);
+  uint8_t* Ks = smem + 2 * Q_BYTES;
+  uint8_t* Vs = Ks + KSLOT * K_BYTES;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(Vs + VSLOT * V_BYTES);
   uint64_t* q_full = bars;
-  uint64_t* kv_full = bars + 1;        // [2]
-  uint64_t* kv_empty = bars + 3;       // [2]
-  uint64_t* s_full = bars + 5;         // [2 groups]
-  uint64_t* p_full = bars + 7;         // [2 groups]
-  uint64_t* o_done = bars + 9;
-  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(bars + 10);
+  uint64_t* k_full = bars + 1;         // [3]
+  uint64_t* k_empty = bars + 4;        // [3]
+  uint64_t* v_full = bars + 7;         // [2]
+  uint64_t* v_empty = bars + 9;        // [2]
+  uint64_t* s_full = bars + 11;        // [2 groups]
+  uint64_t* p_full = bars + 13;        // [2 groups]
+  uint64_t* o_done = bars + 15;
+  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(bars + 16);
 
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
   const int qb = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
@@ -357,9 +380,13 @@ __global__ void __launch_bounds__(THREADS2, 1)
 
   if (threadIdx.x == 0) {
     mbar_init(q_full, 1);
+    for (int s = 0; s < KSLOT; ++s) {
+      mbar_init(&k_full[s], 1);
+      mbar_init(&k_empty[s], 1);
+    }
     for (int s = 0; s < 2; ++s) {
-      mbar_init(&kv_full[s], 1);
-      mbar_init(&kv_empty[s], 1);
+      mbar_init(&v_full[s], 1);
+      mbar_init(&v_empty[s], 1);
       mbar_init(&s_full[s], 1);
       mbar_init(&p_full[s], 4);
     }
@@ -378,23 +405,32 @@ __global__ void __launch_bounds__(THREADS2, 1)
   griddep_launch();
 
   if (warp == 0) {
+    // ---------------- TMA producers: lane 0 Q and K, lane 1 V ----------------
+    const int xq = h * 128;
     if (lane == 0) {
-      const int xq = h * 128;
       mbar_expect_tx(q_full, 2 * Q_BYTES);
       for (int g = 0; g < 2; ++g) {
         tma_load_2d(Qs + g * Q_BYTES, &tmQ, q_full, xq, q_row0 + g * TB);
         tma_load_2d(Qs + g * Q_BYTES + SUB, &tmQ, q_full, xq + 64, q_row0 + g * TB);
       }
       for (int j = 0; j < n_kv; ++j) {
-        const int s = j & 1;
-        if (!mbar_wait(&kv_empty[s], ((j >> 1) & 1) ^ 1u, err)) { failed = true; break; }
-        uint8_t* st = KVs + s * KV_BYTES;
+        const int s = j % KSLOT;
+        if (!mbar_wait(&k_empty[s], ((j / KSLOT) & 1) ^ 1u, err)) { failed = true; break; }
+        uint8_t* st = Ks + s * K_BYTES;
         const int y = kv_row0 + j * TB;
-        mbar_expect_tx(&kv_full[s], KV_BYTES);
-        tma_load_2d(st, &tmK, &kv_full[s], xq, y);
-        tma_load_2d(st + SUB, &tmK, &kv_full[s], xq + 64, y);
-        tma_load_2d(st + 2 * SUB, &tmV, &kv_full[s], xq, y);
-        tma_load_2d(st + 3 * SUB, &tmV, &kv_full[s], xq + 64, y);
+        mbar_expect_tx(&k_full[s], K_BYTES);
+        tma_load_2d(st, &tmK, &k_full[s], xq, y);
+        tma_load_2d(st + SUB, &tmK, &k_full[s], xq + 64, y);
+      }
+    } else if (lane == 1) {
+      for (int j = 0; j < n_kv; ++j) {
+        const int s = j & 1;
+        if (!mbar_wait(&v_empty[s], ((j >> 1) & 1) ^ 1u, err)) { failed = true; break; }
+        uint8_t* st = Vs + s * V_BYTES;
+        const int y = kv_row0 + j * TB;
+        mbar_expect_tx(&v_full[s], V_BYTES);
+        tma_load_2d(st, &tmV, &v_full[s], xq, y);
+        tma_load_2d(st + SUB, &tmV, &v_full[s], xq + 64, y);
       }
     }
   } else if (warp == 1) {
@@ -404,7 +440,7 @@ __global__ void __launch_bounds__(THREADS2, 1)
       const uint32_t idesc_pv = idesc_s | (1u << 16);
       const uint32_t qa = smem_u32(Qs);
       auto issue_s = [&](int g, int j) {
-        const uint32_t ka = smem_u32(KVs + (j & 1) * KV_BYTES);
+        const uint32_t ka = smem_u32(Ks + (j % KSLOT) * K_BYTES);
         const uint32_t qg = qa + g * Q_BYTES;
 #pragma unroll
         for (int kk = 0; kk < 8; ++kk) {
@@ -413,15 +449,16 @@ __global__ void __launch_bounds__(THREADS2, 1)
                      kk ? 1u : 0u);
         }
         tc_commit(&s_full[g]);
+        if (g == 1) tc_commit(&k_empty[j % KSLOT]);  // both tiles' S_j done: K_j is free
       };
       auto issue_pv = [&](int g, int j) {
-        const uint32_t va = smem_u32(KVs + (j & 1) * KV_BYTES + 2 * SUB);
+        const uint32_t va = smem_u32(Vs + (j & 1) * V_BYTES);
 #pragma unroll
         for (int kk = 0; kk < 8; ++kk)
           tc_mma_f16_ts(tmem + O_COL + g * TB, tmem + g * TB + kk * 8,
                         desc_mn_sw128(va + kk * 2048, SUB), idesc_pv, (j | kk) ? 1u : 0u);
       };
-      bool ok = mbar_wait(q_full, 0, err) && mbar_wait(&kv_full[0], 0, err);
+      bool ok = mbar_wait(q_full, 0, err) && mbar_wait(&k_full[0], 0, err);
       if (ok) {
         tc_fence_after();
         issue_s(0, 0);
@@ -429,17 +466,18 @@ __global__ void __launch_bounds__(THREADS2, 1)
         for (int j = 0; j < n_kv && ok; ++j) {
           const bool more = j + 1 < n_kv;
           if (!(ok = mbar_wait(&p_full[0], j & 1, err))) break;
+          if (!(ok = mbar_wait(&v_full[j & 1], (j >> 1) & 1, err))) break;
           tc_fence_after();
           issue_pv(0, j);
           if (more) {
-            if (!(ok = mbar_wait(&kv_full[(j + 1) & 1], ((j + 1) >> 1) & 1, err))) break;
+            if (!(ok = mbar_wait(&k_full[(j + 1) % KSLOT], ((j + 1) / KSLOT) & 1, err))) break;
             tc_fence_after();
             issue_s(0, j + 1);
           }
           if (!(ok = mbar_wait(&p_full[1], j & 1, err))) break;
           tc_fence_after();
           issue_pv(1, j);
-          tc_commit(&kv_empty[j & 1]);
+          tc_commit(&v_empty[j & 1]);
           if (more) issue_s(1, j + 1);
         }
         if (ok) tc_commit(o_done);
