@@ -97,6 +97,15 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_holder;
+  // The weights do not depend on the previous kernel: the producer starts loading the W
+  // tiles of its first tile's first stages before waiting for its predecessor.
+  const int pre = (warp == 0 && lane == 0 && (int)blockIdx.x < n_tiles)
+                      ? (nk < C::STAGES ? nk : C::STAGES) : 0;
+  for (int kb = 0; kb < pre; ++kb) {
+    uint8_t* sa = smem + kb * C::STAGE_BYTES;
+    mbar_expect_tx(&full[kb], C::STAGE_BYTES);
+    tma_load_2d(sa + C::A_BYTES, &tmW, &full[kb], kb * BK, ((int)blockIdx.x % n_nt) * BN);
+  }
   griddep_wait();  // inputs written by the previous kernel are visible from here on
   griddep_launch();
 
@@ -112,11 +121,15 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       for (int tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x) {
         const int m0 = (tile / n_nt) * BM, n0 = (tile % n_nt) * BN;
         for (int kb = 0; kb < nk; ++kb) {
-          if (!mbar_wait(&empty[stage], phase ^ 1u, err)) { ok = false; break; }
           uint8_t* sa = smem + stage * C::STAGE_BYTES;
-          mbar_expect_tx(&full[stage], C::STAGE_BYTES);
-          tma_load_2d(sa, &tmA, &full[stage], kb * BK, m0);
-          tma_load_2d(sa + C::A_BYTES, &tmW, &full[stage], kb * BK, n0);
+          if (tile == (int)blockIdx.x && kb < pre) {
+            tma_load_2d(sa, &tmA, &full[stage], kb * BK, m0);  // W already requested
+          } else {
+            if (!mbar_wait(&empty[stage], phase ^ 1u, err)) { ok = false; break; }
+            mbar_expect_tx(&full[stage], C::STAGE_BYTES);
+            tma_load_2d(sa, &tmA, &full[stage], kb * BK, m0);
+            tma_load_2d(sa + C::A_BYTES, &tmW, &full[stage], kb * BK, n0);
+          }
           ++issued[stage];
           if (++stage == C::STAGES) { stage = 0; phase ^= 1u; }
         }
@@ -309,6 +322,15 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
   cluster_sync();  // both CTAs' barriers initialised, TMEM allocated
   tc_fence_after();
   const uint32_t tmem_base = *tmem_holder;
+  // As in the 1-SM kernel: W tiles of the first tile's first stages before the wait.
+  const int pre = (warp == 0 && lane == 0 && cluster < n_tiles)
+                      ? (nk < C2_STAGES ? nk : C2_STAGES) : 0;
+  for (int kb = 0; kb < pre; ++kb) {
+    uint8_t* sa = smem + kb * C2_STAGE_BYTES;
+    if (rank == 0) mbar_expect_tx(&full[kb], 2 * C2_STAGE_BYTES);
+    tma_load_2d_cg2(sa + C2_HALF_BYTES, &tmW, mapa_shared(smem_u32(&full[kb]), 0), kb * BK,
+                    (cluster % n_nt) * C2_BN + 128 * (int)rank);
+  }
   griddep_wait();
   griddep_launch();
 
@@ -320,10 +342,15 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
       for (int tile = cluster; tile < n_tiles && !failed; tile += n_clusters) {
         const int m0 = (tile / n_nt) * 2 * BM, n0 = (tile % n_nt) * C2_BN;
         for (int kb = 0; kb < nk; ++kb) {
-          if (!mbar_wait(&empty[stage], phase ^ 1u, err)) { failed = true; break; }
           uint8_t* sa = smem + stage * C2_STAGE_BYTES;
-          if (rank == 0) mbar_expect_tx(&full[stage], 2 * C2_STAGE_BYTES);
           const uint32_t fb = mapa_shared(smem_u32(&full[stage]), 0);
+          if (tile == cluster && kb < pre) {  // W already requested before the wait
+            tma_load_2d_cg2(sa, &tmA, fb, kb * BK, m0 + BM * (int)rank);
+            if (++stage == C2_STAGES) { stage = 0; phase ^= 1u; }
+            continue;
+          }
+          if (!mbar_wait(&empty[stage], phase ^ 1u, err)) { failed = true; break; }
+          if (rank == 0) mbar_expect_tx(&full[stage], 2 * C2_STAGE_BYTES);
           tma_load_2d_cg2(sa, &tmA, fb, kb * BK, m0 + BM * (int)rank);
           tma_load_2d_cg2(sa + C2_HALF_BYTES, &tmW, fb, kb * BK, n0 + 128 * (int)rank);
           if (++stage == C2_STAGES) { stage = 0; phase ^= 1u; }

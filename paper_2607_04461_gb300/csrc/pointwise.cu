@@ -214,7 +214,7 @@ __global__ void __launch_bounds__(256) patch_embed_kernel(const float* __restric
 // chunks of 64. Thread -> output o = tid % PD and TPT = 32 PD / 256 consecutive tokens.
 // With guidance each thread also accumulates the unconditional row of its tokens.
 constexpr int HE_TOK = 32, HE_KC = 64;
-template <int PD>
+template <int PD, bool GUIDED>
 __global__ void __launch_bounds__(256) head_euler_kernel(const bf16* __restrict__ a, int n,
                                                          int C, int H, int W, int p,
                                                          const bf16* __restrict__ Wh,
@@ -226,7 +226,7 @@ __global__ void __launch_bounds__(256) head_euler_kernel(const bf16* __restrict_
   __shared__ float as[2][HE_TOK][HE_KC + 1];
   __shared__ float ws[PD][HE_KC + 1];
   const int gw = W / p, P = (H / p) * gw, M = n * P;
-  const bool guided = hs.uncond_rows > 0;
+  constexpr bool guided = GUIDED;
   const int tok0 = blockIdx.x * HE_TOK;
   const int o = threadIdx.x % PD, grp = threadIdx.x / PD;
   float acc[TPT], accu[TPT];
@@ -234,7 +234,7 @@ __global__ void __launch_bounds__(256) head_euler_kernel(const bf16* __restrict_
   for (int i = 0; i < TPT; ++i) acc[i] = accu[i] = 0.f;
   for (int k0 = 0; k0 < D; k0 += HE_KC) {
     __syncthreads();
-    for (int i = threadIdx.x; i < 2 * HE_TOK * HE_KC / 8; i += 256) {
+    for (int i = threadIdx.x; i < (GUIDED ? 2 : 1) * HE_TOK * HE_KC / 8; i += 256) {
       const int u = i / (HE_TOK * HE_KC / 8), rem = i % (HE_TOK * HE_KC / 8);
       const int t = rem / (HE_KC / 8), kc = (rem % (HE_KC / 8)) * 8;
       float v[8] = {0, 0, 0, 0, 0, 0, 0, 0};
@@ -257,7 +257,7 @@ __global__ void __launch_bounds__(256) head_euler_kernel(const bf16* __restrict_
 #pragma unroll
       for (int i = 0; i < TPT; ++i) {
         acc[i] += wv * as[0][grp * TPT + i][k];
-        accu[i] += wv * as[1][grp * TPT + i][k];
+        if (GUIDED) accu[i] += wv * as[1][grp * TPT + i][k];
       }
     }
   }
@@ -415,13 +415,20 @@ cudaError_t head_euler(const bf16* a, int n, int C, int H, int W, int p, const b
   if (M == 0) return cudaSuccess;
   if (D % 8) return cudaErrorInvalidValue;
   const dim3 grid((M + HE_TOK - 1) / HE_TOK);
+#define HE(PD)                                                                              \
+  (hs.uncond_rows > 0                                                                      \
+       ? launch_k(head_euler_kernel<PD, true>, grid, dim3(256), 0, st, a, n, C, H, W, p, Wh, \
+                  bh, D, hs, z)                                                            \
+       : launch_k(head_euler_kernel<PD, false>, grid, dim3(256), 0, st, a, n, C, H, W, p,   \
+                  Wh, bh, D, hs, z))
   switch (PD) {
-    case 8: return launch_k(head_euler_kernel<8>, grid, dim3(256), 0, st, a, n, C, H, W, p, Wh, bh, D, hs, z);
-    case 16: return launch_k(head_euler_kernel<16>, grid, dim3(256), 0, st, a, n, C, H, W, p, Wh, bh, D, hs, z);
-    case 32: return launch_k(head_euler_kernel<32>, grid, dim3(256), 0, st, a, n, C, H, W, p, Wh, bh, D, hs, z);
-    case 64: return launch_k(head_euler_kernel<64>, grid, dim3(256), 0, st, a, n, C, H, W, p, Wh, bh, D, hs, z);
+    case 8: return HE(8);
+    case 16: return HE(16);
+    case 32: return HE(32);
+    case 64: return HE(64);
     default: return cudaErrorInvalidValue;
   }
+#undef HE
 }
 
 cudaError_t gemv(const bf16* W, const float* b, const float* x, float* y, int O, int K,
