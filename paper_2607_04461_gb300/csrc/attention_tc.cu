@@ -225,21 +225,28 @@ __global__ void __launch_bounds__(THREADS, 1)
       if (!__all_sync(0xffffffffu, ok)) { failed = true; break; }
       tc_fence_after();
       float s[128];
+      {
+        // all four loads in flight, one wait; scores stay unscaled (the scale is > 0, so the
+        // row max commutes with it and is scaled once)
+        uint32_t u[128];
 #pragma unroll
-      for (int c = 0; c < 4; ++c) {
-        uint32_t u[32];
-        tmem_ld32(lane_base + (j & 1) * TB + c * 32, u);
+        for (int c = 0; c < 4; ++c) tmem_ld32(lane_base + (j & 1) * TB + c * 32, u + c * 32);
         tmem_ld_wait();
 #pragma unroll
-        for (int i = 0; i < 32; ++i) s[c * 32 + i] = __uint_as_float(u[i]) * p.scale_log2;
+        for (int c = 0; c < 4; ++c) reg_fence32(u + c * 32);
+#pragma unroll
+        for (int i = 0; i < 128; ++i) s[i] = __uint_as_float(u[i]);
       }
       const int valid = p.Lkv - j * TB;  // keys of this tile that exist
+      if (valid < TB) {
+#pragma unroll
+        for (int i = 0; i < 128; ++i)
+          if (i >= valid) s[i] = -INFINITY;
+      }
       float mx = -INFINITY;
 #pragma unroll
-      for (int i = 0; i < 128; ++i) {
-        if (i >= valid) s[i] = -INFINITY;
-        mx = fmaxf(mx, s[i]);
-      }
+      for (int i = 0; i < 128; ++i) mx = fmaxf(mx, s[i]);
+      mx *= p.scale_log2;
       if (j > 0) {
         // PV_{j-1} must be done before P is overwritten and before O is touched
         const bool ok2 = mbar_wait(o_done, (j - 1) & 1, err);
@@ -258,6 +265,7 @@ __global__ void __launch_bounds__(THREADS, 1)
           uint32_t u[32];
           tmem_ld32(lane_base + O_COL + c * 32, u);
           tmem_ld_wait();
+          reg_fence32(u);
 #pragma unroll
           for (int i = 0; i < 32; ++i) u[i] = __float_as_uint(__uint_as_float(u[i]) * alpha);
           tmem_st32(lane_base + O_COL + c * 32, u);
@@ -270,7 +278,7 @@ __global__ void __launch_bounds__(THREADS, 1)
         float e[8];
 #pragma unroll
         for (int q = 0; q < 8; ++q) {
-          e[q] = ex2(s[ch * 8 + q] - m_used);
+          e[q] = ex2(fmaf(s[ch * 8 + q], p.scale_log2, -m_used));
           lsum += e[q];
         }
         uint4 v;
@@ -299,6 +307,7 @@ __global__ void __launch_bounds__(THREADS, 1)
           uint32_t u[32];
           tmem_ld32(lane_base + O_COL + c * 32, u);
           tmem_ld_wait();
+          reg_fence32(u);
           if (qrow < p.Lq) {
 #pragma unroll
             for (int g = 0; g < 4; ++g) {
@@ -497,21 +506,28 @@ __global__ void __launch_bounds__(THREADS2, 1)
       if (!__all_sync(0xffffffffu, ok)) { failed = true; break; }
       tc_fence_after();
       float s[128];
+      {
+        // all four loads in flight, one wait; scores stay unscaled (the scale is > 0, so the
+        // row max commutes with it and is scaled once)
+        uint32_t u[128];
 #pragma unroll
-      for (int c = 0; c < 4; ++c) {
-        uint32_t u[32];
-        tmem_ld32(lane_base + s_col + c * 32, u);
+        for (int c = 0; c < 4; ++c) tmem_ld32(lane_base + s_col + c * 32, u + c * 32);
         tmem_ld_wait();
 #pragma unroll
-        for (int i = 0; i < 32; ++i) s[c * 32 + i] = __uint_as_float(u[i]) * p.scale_log2;
+        for (int c = 0; c < 4; ++c) reg_fence32(u + c * 32);
+#pragma unroll
+        for (int i = 0; i < 128; ++i) s[i] = __uint_as_float(u[i]);
       }
-      const int valid = p.Lkv - j * TB;
+      const int valid = p.Lkv - j * TB;  // keys of this tile that exist
+      if (valid < TB) {
+#pragma unroll
+        for (int i = 0; i < 128; ++i)
+          if (i >= valid) s[i] = -INFINITY;
+      }
       float mx = -INFINITY;
 #pragma unroll
-      for (int i = 0; i < 128; ++i) {
-        if (i >= valid) s[i] = -INFINITY;
-        mx = fmaxf(mx, s[i]);
-      }
+      for (int i = 0; i < 128; ++i) mx = fmaxf(mx, s[i]);
+      mx *= p.scale_log2;
       if (j == 0) {
         m_used = mx;
       } else if (__any_sync(0xffffffffu, mx > m_used + 8.f)) {
@@ -524,6 +540,7 @@ __global__ void __launch_bounds__(THREADS2, 1)
           uint32_t u[32];
           tmem_ld32(lane_base + o_col + c * 32, u);
           tmem_ld_wait();
+          reg_fence32(u);
 #pragma unroll
           for (int i = 0; i < 32; ++i) u[i] = __float_as_uint(__uint_as_float(u[i]) * alpha);
           tmem_st32(lane_base + o_col + c * 32, u);
@@ -535,8 +552,8 @@ __global__ void __launch_bounds__(THREADS2, 1)
         uint32_t u[32];
 #pragma unroll
         for (int i = 0; i < 32; ++i) {
-          const float e0 = ex2(s[c * 64 + 2 * i] - m_used);
-          const float e1 = ex2(s[c * 64 + 2 * i + 1] - m_used);
+          const float e0 = ex2(fmaf(s[c * 64 + 2 * i], p.scale_log2, -m_used));
+          const float e1 = ex2(fmaf(s[c * 64 + 2 * i + 1], p.scale_log2, -m_used));
           lsum += e0 + e1;
           u[i] = pack_bf16x2(e0, e1);
         }
@@ -560,6 +577,7 @@ __global__ void __launch_bounds__(THREADS2, 1)
           uint32_t u[32];
           tmem_ld32(lane_base + o_col + c * 32, u);
           tmem_ld_wait();
+          reg_fence32(u);
           if (qrow < p.Lq) {
 #pragma unroll
             for (int q = 0; q < 4; ++q) {
