@@ -419,8 +419,21 @@ def run_probe(args):
     m = fb.Model(cfg, synth.make_weights(cfg))
     g = torch.Generator().manual_seed(0)
     rnd = lambda *s, dt=torch.bfloat16: (torch.randn(*s, generator=g) * 0.5).to(dt).cuda()  # noqa
-    if args.probe in ("gemm_shapes", "breakdown"):
+    if args.probe in ("gemm_shapes", "attn_shapes", "breakdown"):
         call = None
+    elif args.probe in ("gemm_refine_out", "gemm_refine_down"):
+        # the refine pass's attention output projection / FFN down-projection (one
+        # candidate, 1560 rows), once over whole tiles (impl 3) and once with the
+        # stream-K split (impl 4) per step
+        M, D = 1560, 1536
+        K = D if args.probe == "gemm_refine_out" else 8960
+        A, W, b = rnd(M, K), rnd(D, K), rnd(D, dt=torch.float32)
+        h, gt = rnd(M, D, dt=torch.float32), rnd(D, dt=torch.float32)
+        out = torch.empty(M, D, dtype=torch.float32, device="cuda")
+
+        def call():
+            for impl in (3, 4):
+                fb.fb_op_gemm(m.handle, M, D, K, A, W, b, 2, out, h, gt, None, None, impl)
     elif args.probe == "gemm_out":
         M, D = 8192, 1536
         A, W, b = rnd(M, D), rnd(D, D), rnd(D, dt=torch.float32)
@@ -447,6 +460,8 @@ def run_probe(args):
                                           1 if args.probe == "attn_mma" else 0)
     if args.probe == "gemm_shapes":
         return probe_gemm_shapes(m, rnd, args)
+    if args.probe == "attn_shapes":
+        return probe_attn_shapes(m, rnd, args)
     if args.probe == "breakdown":
         m.close()
         return probe_breakdown(args)
@@ -477,22 +492,76 @@ def probe_gemm_shapes(m, rnd, args):
             out = torch.empty(M, N, dtype=torch.bfloat16 if epi < 2 else torch.float32, device="cuda")
             r = rnd(M, N, dt=torch.float32) if epi >= 2 else None
             dl = torch.empty(M, N, dtype=torch.bfloat16, device="cuda") if epi == 3 else None
-            for impl in (0, 2):
+            for impl, tag in ((0, "auto"), (2, "1sm"), (3, "2sm_tiles"), (4, "2sm_streamk")):
                 f = lambda: fb.fb_op_gemm(m.handle, M, N, K, A, W, b, epi, out, r, b if epi >= 2 else None,  # noqa
                                           r if epi == 3 else None, dl, impl)
-                f()
+                try:
+                    f()
+                except fb.FlashBonError:
+                    continue   # stream-K needs enough K blocks per SM pair
                 fb.fb_set_op_repeat(m.handle, reps)
                 m.reset_stats()
                 m.set_timing(1 << fb.K["gemm_tc"])
                 f()
                 m.set_timing(0)
-                fb.fb_set_op_repeat(m.handle, 1)
                 st = m.stats()["gemm_tc"]
                 us = st["ms"] * 1e3 / st["launches"]
-                res[f"M{M}/{name}/{'auto' if impl == 0 else '1sm'}"] = {
-                    "us": round(us, 2), "tflops": round(2 * M * N * K / us / 1e6, 1)}
+                # back to back without per-launch events (chained as in the model)
+                fb.fb_set_op_repeat(m.handle, 10 * reps)
+                t0 = time.perf_counter()
+                f()
+                chain_us = (time.perf_counter() - t0) * 1e6 / (10 * reps)
+                fb.fb_set_op_repeat(m.handle, 1)
+                res[f"M{M}/{name}/{tag}"] = {
+                    "us": round(us, 2), "tflops": round(2 * M * N * K / us / 1e6, 1),
+                    "chained_us": round(chain_us, 2)}
             del A, W, out, r, dl
     print(json.dumps({"probe": "gemm_shapes", "res": res}))
+    return 0
+
+
+def probe_attn_shapes(m, rnd, args):
+    """Per-launch and back-to-back time of the block's attention shapes at the draft
+    (N=32) and refine (N=1) batch sizes for the tcgen05 kernel with 128- and 256-query
+    CTAs."""
+    import torch
+    from paper_2607_04461_gb300 import flashbon as fb
+    H, dh, P, T = 12, 128, 1560, 512
+    D = H * dh
+    res = {}
+    reps = max(5, args.steps)
+    for n in (32, 1):
+        qkv = rnd(n * P, 3 * D)
+        kv = rnd(T, 2 * D)
+        o = torch.empty(n * P, D, dtype=torch.bfloat16, device="cuda")
+        base = qkv.data_ptr()
+        cases = {
+            "self": lambda impl: fb.fb_op_attention(m.handle, base, 3 * D, base + 2 * D, 3 * D,
+                                                    base + 4 * D, 3 * D, o, D, n, P, P, P, H,
+                                                    dh, impl),
+            "cross": lambda impl: fb.fb_op_attention(m.handle, base, 3 * D, kv.data_ptr(),
+                                                     2 * D, kv.data_ptr() + 2 * D, 2 * D, o, D,
+                                                     n, P, T, 0, H, dh, impl)}
+        for name, f in cases.items():
+            flops = 4.0 * n * H * P * (P if name == "self" else T) * dh
+            for impl, tag in ((0, "auto"), (2, "q128"), (3, "q256")):
+                f(impl)
+                fb.fb_set_op_repeat(m.handle, reps)
+                m.reset_stats()
+                m.set_timing(1 << fb.K["attn_self"])
+                f(impl)
+                m.set_timing(0)
+                st = m.stats()["attn_self"]
+                us = st["ms"] * 1e3 / st["launches"]
+                fb.fb_set_op_repeat(m.handle, 10 * reps)
+                t0 = time.perf_counter()
+                f(impl)
+                chain_us = (time.perf_counter() - t0) * 1e6 / (10 * reps)
+                fb.fb_set_op_repeat(m.handle, 1)
+                res[f"N{n}/{name}/{tag}"] = {"us": round(us, 2), "chained_us": round(chain_us, 2),
+                                             "tflops": round(flops / chain_us / 1e6, 1)}
+        del qkv, kv, o
+    print(json.dumps({"probe": "attn_shapes", "res": res}))
     return 0
 
 
@@ -546,8 +615,9 @@ def main():
     ap.add_argument("--variant", choices=list(VARIANTS), default="base",
                     help="base: the draft-pool workload; cfg / sde: the same with guidance "
                          "or SDE steps")
-    ap.add_argument("--probe", choices=["gemm", "gemm_resid", "gemm_out", "attn", "attn_mma",
-                                        "gemm_shapes", "breakdown"],
+    ap.add_argument("--probe", choices=["gemm", "gemm_resid", "gemm_out", "gemm_refine_out",
+                                        "gemm_refine_down", "attn", "attn_mma", "gemm_shapes",
+                                        "attn_shapes", "breakdown"],
                     default=None)
     args = ap.parse_args()
     if args.probe:

@@ -221,7 +221,13 @@ const char* fb_kernel_name(int kind);
  * A, W bf16 row-major, leading dimensions K; out / resid / base / delta leading
  * dimension N. impl: 0 = automatic (tcgen05 when N % 128 == 0 and K % 64 == 0: the
  * 2-SM cta_group::2 kernel when N % 256 == 0, else the 1-SM kernel), 1 = force the
- * CUDA-core kernel, 2 = force the 1-SM tcgen05 kernel (same shape rules). */
+ * CUDA-core kernel, 2 = force the 1-SM tcgen05 kernel (same shape rules), 3 = the 2-SM
+ * kernel over whole 256 x 256 tiles only, 4 = the 2-SM kernel with the stream-K split:
+ * every SM pair takes an equal share of the (tile, 64-wide K block) units and tiles cut
+ * between pairs are summed from fp32 partials in the model's workspace, in K order (so
+ * the result does not depend on timing). impl 4 needs N % 256 == 0 and at least 4 K
+ * blocks per SM pair (ceil(M / 256) * N / 256 * K / 64 >= 4 * pairs), else FB_ECUDA;
+ * impl 0 uses whole tiles. */
 /* fb_set_op_repeat: fb_op_gemm / fb_op_attention launch their kernel n >= 1 times back
  * to back (default 1), for timing a kernel without a stream synchronisation per launch. */
 fb_status fb_set_op_repeat(fb_model* m, int n);
@@ -233,7 +239,8 @@ fb_status fb_op_gemm(fb_model* m, int M, int N, int K, const void* A, const void
  * h*head_dim; likewise K, V (kv_batch_rows = 0 shares one K/V across the batch,
  * otherwise the row offset between batches); O row stride ldo. impl: 0 = automatic
  * (the tcgen05 kernel for head_dim 128, the mma.sync kernel for 64), 1 = force the
- * mma.sync kernel. */
+ * mma.sync kernel, 2 / 3 = force the tcgen05 kernel with 128- / 256-query CTAs
+ * (head_dim 128 only, else FB_EINVAL). */
 fb_status fb_op_attention(fb_model* m, const void* Q, int ldq, const void* K, int ldk,
                           const void* V, int ldv, void* O, int ldo, int batch, int Lq,
                           int Lkv, int kv_batch_rows, int heads, int head_dim, int impl);

@@ -169,6 +169,11 @@ struct fb_model {
   size_t anchor_elems = 0;
   int* derr = nullptr;
   int* herr = nullptr;  // pinned
+  // stream-K workspace of the 2-SM GEMM: partial accumulators and per-tile counters
+  // (zero between launches; reset after a device error)
+  float* sk_ws = nullptr;
+  int* sk_ctr = nullptr;
+  int sk_clusters = 0;
   // statistics
   unsigned timing_mask = 0;
   int op_repeat = 1;
@@ -264,6 +269,13 @@ fb_status end_call(fb_model* m) {
   CK(cudaMemcpyAsync(m->herr, m->derr, sizeof(int), cudaMemcpyDeviceToHost, m->st));
   CK(cudaStreamSynchronize(m->st));
   collect_timings(m);
+  if (*m->herr != 0 && m->sk_ctr) {
+    // a kernel that gave up may have left stream-K counters counted in
+    fb_stream_op_not_kernel();
+    CK(cudaMemsetAsync(m->sk_ctr, 0, (size_t)m->sk_clusters * SK_CTR_PER_CLUSTER * sizeof(int),
+                       m->st));
+    CK(cudaStreamSynchronize(m->st));
+  }
   if (*m->herr == FB_DEVERR_WAIT_TIMEOUT)
     return fail(FB_ECUDA, "device wait timed out (a kernel gave up after its time limit)");
   if (*m->herr != 0) return fail(FB_ECUDA, "device error %d", *m->herr);
@@ -271,8 +283,14 @@ fb_status end_call(fb_model* m) {
 }
 
 // ---- kernel wrappers with statistics ------------------------------------------------
-// impl: 0 automatic, 1 CUDA-core kernel, 2 the 1-SM tcgen05 kernel
-fb_status run_gemm(fb_model* m, const GemmArgs& g, int impl = 0) {
+// impl: 0 automatic, 1 CUDA-core kernel, 2 the 1-SM tcgen05 kernel, 3 the 2-SM kernel
+// over whole tiles, 4 the 2-SM kernel with the stream-K split
+fb_status run_gemm(fb_model* m, const GemmArgs& g0, int impl = 0) {
+  GemmArgs g = g0;
+  g.sk_ws = m->sk_ws;
+  g.sk_ctr = m->sk_ctr;
+  g.sk_clusters = m->sk_clusters;
+  g.sk_mode = impl == 3 ? 1 : impl == 4 ? 2 : 0;
   const double flops = 2.0 * g.M * (double)g.N * g.K;
   double bytes = 2.0 * ((double)g.M * g.K + (double)g.N * g.K);
   bytes += (g.kind <= EPI_GELU_BF16) ? 2.0 * g.M * g.N : 8.0 * g.M * g.N;
@@ -300,13 +318,17 @@ GemmArgs gemm_args(int M, int N, int K, const bf16* A, const bf16* W, const floa
   return g;
 }
 
-// impl: 0 automatic (tcgen05 for head_dim 128), 1 the mma.sync kernel
-fb_status run_attn(fb_model* m, const AttnArgs& a, int kind, int impl = 0) {
+// impl: 0 automatic (tcgen05 for head_dim 128), 1 the mma.sync kernel, 2 / 3 the tcgen05
+// kernel with 128- / 256-query CTAs
+fb_status run_attn(fb_model* m, const AttnArgs& a0, int kind, int impl = 0) {
+  AttnArgs a = a0;
+  a.tc_variant = impl >= 2 ? impl - 1 : 0;
   const double flops = 4.0 * a.batch * a.heads * (double)a.Lq * a.Lkv * a.head_dim;
   const double kvb = (a.kv_batch_rows ? a.batch : 1) * 2.0 * a.Lkv * a.heads * a.head_dim * 2;
   const double bytes = 2.0 * a.batch * a.Lq * (double)a.heads * a.head_dim * 2 + kvb;
   KTimer t(m, kind, flops, bytes);
-  if (impl == 0 && attention_tc_supported(a)) CK(attention_tc(a, m->derr, m->st));
+  if (impl != 1 && attention_tc_supported(a)) CK(attention_tc(a, m->derr, m->st));
+  else if (impl >= 2) return fail(FB_EINVAL, "the tcgen05 attention kernel needs head_dim 128");
   else CK(attention(a, m->st));
   return FB_OK;
 }
@@ -845,6 +867,13 @@ fb_status fb_init_model(const fb_cfg* cfg, const float* weights_host, fb_model**
       (s = dalloc_t(m, &m->rope, (size_t)m->P * c.head_dim / 2)) ||
       (s = dalloc_t(m, &m->zbuf, zn)) || (s = dalloc_t(m, &m->derr, 1)))
     return bail(s);
+  m->sk_clusters = m->num_sms / 2;
+  if ((s = dalloc_t(m, &m->sk_ws, (size_t)m->sk_clusters * SK_WS_FLOATS_PER_CLUSTER)) ||
+      (s = dalloc_t(m, &m->sk_ctr, (size_t)m->sk_clusters * SK_CTR_PER_CLUSTER)))
+    return bail(s);
+  if (cudaMemset(m->sk_ctr, 0, (size_t)m->sk_clusters * SK_CTR_PER_CLUSTER * sizeof(int)) !=
+      cudaSuccess)
+    return bail(fail(FB_ECUDA, "cudaMemset failed"));
   // RoPE table: pair j of a head rotates by the token's row (j < head_dim/4) or column,
   // with frequency theta^(-2 j' / (head_dim/2)), j' = j mod head_dim/4.
   {
@@ -995,7 +1024,7 @@ fb_status fb_op_gemm(fb_model* m, int M, int N, int K, const void* A, const void
   g.epi.base = base;
   g.epi.delta = (bf16*)delta;
   CKS(begin_call(m));
-  if (impl < 0 || impl > 2) return fail(FB_EINVAL, "impl must be 0, 1 or 2");
+  if (impl < 0 || impl > 4) return fail(FB_EINVAL, "impl must be 0 .. 4");
   for (int r = 0; r < m->op_repeat; ++r) CKS(run_gemm(m, g, impl));
   return end_call(m);
 }
@@ -1004,7 +1033,7 @@ fb_status fb_op_attention(fb_model* m, const void* Q, int ldq, const void* K, in
                           const void* V, int ldv, void* O, int ldo, int batch, int Lq, int Lkv,
                           int kv_batch_rows, int heads, int head_dim, int impl) {
   if (!m || !Q || !K || !V || !O) return fail(FB_EINVAL, "null argument");
-  if (impl < 0 || impl > 1) return fail(FB_EINVAL, "impl must be 0 or 1");
+  if (impl < 0 || impl > 3) return fail(FB_EINVAL, "impl must be 0 .. 3");
   if (batch < 1 || Lq < 1 || Lkv < 1 || heads < 1 || (head_dim != 64 && head_dim != 128))
     return fail(FB_EINVAL, "bad sizes");
   AttnArgs a{};

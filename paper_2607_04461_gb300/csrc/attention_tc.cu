@@ -659,10 +659,13 @@ cudaError_t attention_tc(const AttnArgs& a, int* err, cudaStream_t st) {
   p.ldo = a.ldo;
   p.scale_log2 = 1.4426950408889634f / sqrtf(128.f);
   p.err = err;
-  // 256-query CTAs share each K/V tile between two query tiles; with fewer than two
-  // such CTAs per SM the 128-query kernel keeps more SMs busy.
-  const long ctas2 = (long)((a.Lq + 2 * TB - 1) / (2 * TB)) * a.heads * a.batch;
-  if (ctas2 >= 2L * sms) {
+  // 256-query CTAs share each K/V tile between two query tiles and overlap one tile's
+  // softmax with the other's MMAs; the 128-query kernel only where all of its CTAs fit
+  // in one wave (one CTA per SM), which then finishes sooner (e.g. 1 x 1560 queries x 12
+  // heads: 156 CTAs of 128 > 152 SMs, 256-query CTAs 18 % faster).
+  const long ctas1 = (long)((a.Lq + TB - 1) / TB) * a.heads * a.batch;
+  const bool two = a.tc_variant == 2 || (a.tc_variant == 0 && ctas1 > sms);
+  if (two) {
     cudaError_t e = cudaFuncSetAttribute(attn_tc2_kernel,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM2_BYTES);
     if (e != cudaSuccess) return e;

@@ -19,6 +19,7 @@
 // Every mbarrier wait is bounded (mbar_wait): on timeout the kernel records the error,
 // stops issuing work, waits (bounded) for its own TMA loads, frees TMEM and returns.
 #include <cudaTypedefs.h>
+#include <string.h>
 
 #include "kernels.h"
 
@@ -233,17 +234,34 @@ constexpr int C2_BN = 256;
 constexpr int C2_HALF_BYTES = 128 * BK * 2;          // 16 KB: 128 rows x 64 bf16
 constexpr int C2_STAGE_BYTES = 2 * C2_HALF_BYTES;    // this CTA's A rows + W rows
 constexpr int C2_TMEM_COLS = 2 * C2_BN;
-// fp32 residual epilogues stage each 32 x 32 accumulator chunk in shared memory (one
-// [32][33] float tile per epilogue warp) so that their global loads and stores are
-// whole 128-byte rows; that space comes out of the operand ring (5 stages instead of 6).
+// Epilogues. bf16 outputs and the fp32 gated residual go through shared memory and TMA:
+// each epilogue warp owns two 32 x 32 tiles (bf16 64-byte rows with the 64-byte swizzle,
+// or fp32 128-byte rows with the 128-byte swizzle, so that one row per lane is read and
+// written at full shared-memory bandwidth), writes its results there and stores them with
+// a TMA bulk store that runs while it computes the next chunk; the fp32 residual tiles of
+// a chunk are loaded by TMA into the same tile, two chunks ahead, the first two before
+// the accumulator is ready. The residual + contribution epilogue (Delta) stages each
+// chunk in a [32][33] float tile per warp and moves whole 128-byte rows with plain loads
+// and stores. The epilogue space comes out of the operand ring where needed.
 constexpr int EPI_STAGE_FLOATS = 32 * 33;
 template <int KIND>
 struct C2Cfg {
-  static constexpr bool STAGED = KIND >= EPI_RESID;
-  static constexpr int STAGES = STAGED ? 5 : 6;
-  static constexpr int EPI_BYTES = STAGED ? 8 * EPI_STAGE_FLOATS * 4 : 0;
-  static constexpr int SMEM_BYTES = STAGES * C2_STAGE_BYTES + EPI_BYTES + 1024 + 256;
+  static constexpr bool TMA_EPI = KIND != EPI_RESID_DELTA;
+  static constexpr bool STAGED = KIND == EPI_RESID_DELTA;
+  static constexpr int STAGES = KIND == EPI_BF16 || KIND == EPI_GELU_BF16 ? 6 : 5;
+  static constexpr int TILE_BYTES = KIND == EPI_RESID ? 32 * 32 * 4 : 32 * 32 * 2;
+  static constexpr int EPI_BYTES = TMA_EPI ? 8 * 2 * TILE_BYTES : 8 * EPI_STAGE_FLOATS * 4;
+  static constexpr int SMEM_BYTES = STAGES * C2_STAGE_BYTES + EPI_BYTES + 1024 + 512;
 };
+static_assert(C2Cfg<EPI_BF16>::SMEM_BYTES <= 232448 && C2Cfg<EPI_RESID>::SMEM_BYTES <= 232448 &&
+                  C2Cfg<EPI_RESID_DELTA>::SMEM_BYTES <= 232448,
+              "2-SM GEMM shared memory");
+
+// byte offset of row r, 16-byte column chunk q in a TMA tile of 128-byte rows (128-byte
+// swizzle: chunk bits 4-6 of the address XOR bits 7-9) or 64-byte rows (64-byte swizzle:
+// bits 4-5 XOR bits 7-8); tiles start on 1024-byte boundaries
+__device__ __forceinline__ uint32_t swz128(int r, int q) { return r * 128 + ((q ^ (r & 7)) << 4); }
+__device__ __forceinline__ uint32_t swz64(int r, int q) { return r * 64 + ((q ^ ((r >> 1) & 3)) << 4); }
 
 // Staged residual epilogue of one warp for one 32 x 32 chunk: rows row0..row0+31 (the
 // warp's TMEM lane quarter), columns col0..col0+31; acc holds the thread's row (lane).
@@ -282,21 +300,79 @@ __device__ __forceinline__ void epi_resid_staged(const GemmEpi& e, float* stg, i
   __syncwarp();
 }
 
+// ---- work split of the 2-SM kernel --------------------------------------------------
+// Data-parallel: cluster c computes whole tiles c, c + G, c + 2G, ... (G clusters).
+// Stream-K: the U = tiles x nk (tile, K-block) units, tile-major, are cut into G
+// contiguous ranges of floor(c U / G) .. floor((c + 1) U / G); a cluster walks its range
+// as segments (one tile, K-blocks kb0..kb1). A tile cut between clusters c_lo..c_hi gets
+// one fp32 partial accumulator per contributor; each epilogue warp writes its part of the
+// partial to the workspace and counts itself on the tile's counter, and the last of the
+// contributors' warps to arrive adds the partials in contributor (= K) order, so the sum
+// does not depend on arrival order, runs the epilogue and resets the counter to zero.
+// With U >= G every range is non-empty, so c_hi - c_lo + 1 clusters contribute.
+struct Seg {
+  int tile, kb0, kb1;
+};
+struct WorkIter {
+  long long u, u1;
+  int tile, n_tiles, nk, G;
+  bool sk;
+  __device__ WorkIter(bool sk_, int c, int G_, int n_tiles_, int nk_)
+      : tile(c), n_tiles(n_tiles_), nk(nk_), G(G_), sk(sk_) {
+    const long long U = (long long)n_tiles_ * nk_;
+    u = (long long)c * U / G_;
+    u1 = (long long)(c + 1) * U / G_;
+  }
+  __device__ bool next(Seg& g) {
+    if (!sk) {
+      if (tile >= n_tiles) return false;
+      g.tile = tile;
+      g.kb0 = 0;
+      g.kb1 = nk;
+      tile += G;
+      return true;
+    }
+    if (u >= u1) return false;
+    g.tile = (int)(u / nk);
+    g.kb0 = (int)(u % nk);
+    const long long rest = u1 - u;
+    g.kb1 = rest < nk - g.kb0 ? g.kb0 + (int)rest : nk;
+    u += g.kb1 - g.kb0;
+    return true;
+  }
+};
+// the cluster whose stream-K range holds unit u
+__device__ __forceinline__ int sk_owner(long long u, long long U, int G) {
+  return (int)(((u + 1) * G - 1) / U);
+}
+// Workspace slot of cluster c's segment of `tile`: 2c for the first segment of its range,
+// 2c + 1 for the last (a range meets at most two cut tiles). Per slot and CTA of the pair,
+// 8 epilogue warps x 4096 floats: [chunk 4][j/4 8][lane 32][4], 32 rows x 128 columns.
+__device__ __forceinline__ float* sk_part(float* ws, int c, int tile, long long U, int G, int nk,
+                                          int rank, int we) {
+  const int first_tile = (int)(((long long)c * U / G) / nk);
+  const int slot = 2 * c + (tile == first_tile ? 0 : 1);
+  return ws + ((size_t)(slot * 2 + rank) * 8 + we) * 4096;
+}
+
 template <int KIND>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
     gemm_tc2_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmW,
-                    int M, int N, int K, GemmEpi epi, int* err) {
+                    const __grid_constant__ CUtensorMap tmO, const __grid_constant__ CUtensorMap tmR,
+                    int M, int N, int K, GemmEpi epi, SkArgs sk, int* err) {
   using CC = C2Cfg<KIND>;
   constexpr int C2_STAGES = CC::STAGES;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  float* epi_stage = reinterpret_cast<float*>(smem + C2_STAGES * C2_STAGE_BYTES);
-  uint64_t* full = reinterpret_cast<uint64_t*>(smem + C2_STAGES * C2_STAGE_BYTES + CC::EPI_BYTES);
+  uint8_t* epi_smem = smem + C2_STAGES * C2_STAGE_BYTES;
+  float* epi_stage = reinterpret_cast<float*>(epi_smem);
+  uint64_t* full = reinterpret_cast<uint64_t*>(epi_smem + CC::EPI_BYTES);
   uint64_t* empty = full + C2_STAGES;
   uint64_t* tmem_full = empty + C2_STAGES;
   uint64_t* tmem_empty = tmem_full + 2;
-  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(tmem_empty + 2);
+  uint64_t* rload = tmem_empty + 2;  // residual tile loads: 2 per epilogue warp
+  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(rload + 16);
 
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
   const uint32_t rank = cluster_ctarank();
@@ -314,23 +390,35 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
       mbar_init(&tmem_full[a], 1);
       mbar_init(&tmem_empty[a], 16);  // 8 epilogue warps x 2 CTAs
     }
+    for (int b = 0; b < 16; ++b) mbar_init(&rload[b], 1);
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     tma_prefetch_desc(&tmA);
     tma_prefetch_desc(&tmW);
+    if (CC::TMA_EPI) tma_prefetch_desc(&tmO);
+    if (KIND == EPI_RESID) tma_prefetch_desc(&tmR);
   }
   if (warp == 1) tmem_alloc_cg2(tmem_holder, C2_TMEM_COLS);
   tc_fence_before();
   cluster_sync();  // both CTAs' barriers initialised, TMEM allocated
   tc_fence_after();
   const uint32_t tmem_base = *tmem_holder;
-  // As in the 1-SM kernel: W tiles of the first tile's first stages before the wait.
-  const int pre = (warp == 0 && lane == 0 && cluster < n_tiles)
-                      ? (nk < C2_STAGES ? nk : C2_STAGES) : 0;
-  for (int kb = 0; kb < pre; ++kb) {
-    uint8_t* sa = smem + kb * C2_STAGE_BYTES;
-    if (rank == 0) mbar_expect_tx(&full[kb], 2 * C2_STAGE_BYTES);
-    tma_load_2d_cg2(sa + C2_HALF_BYTES, &tmW, mapa_shared(smem_u32(&full[kb]), 0), kb * BK,
-                    (cluster % n_nt) * C2_BN + 128 * (int)rank);
+  const bool use_sk = sk.on != 0;
+  const long long U = (long long)n_tiles * nk;
+  // As in the 1-SM kernel: W tiles of the first segment's first stages before the wait.
+  Seg first{0, 0, 0};
+  int pre = 0;
+  if (warp == 0 && lane == 0) {
+    WorkIter w0(use_sk, cluster, n_clusters, n_tiles, nk);
+    if (w0.next(first)) {
+      const int len = first.kb1 - first.kb0;
+      pre = len < C2_STAGES ? len : C2_STAGES;
+    }
+  }
+  for (int i = 0; i < pre; ++i) {
+    uint8_t* sa = smem + i * C2_STAGE_BYTES;
+    if (rank == 0) mbar_expect_tx(&full[i], 2 * C2_STAGE_BYTES);
+    tma_load_2d_cg2(sa + C2_HALF_BYTES, &tmW, mapa_shared(smem_u32(&full[i]), 0),
+                    (first.kb0 + i) * BK, (first.tile % n_nt) * C2_BN + 128 * (int)rank);
   }
   griddep_wait();
   griddep_launch();
@@ -340,12 +428,14 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
       // ---------------- TMA producer (both CTAs) ----------------
       int stage = 0;
       uint32_t phase = 0;
-      for (int tile = cluster; tile < n_tiles && !failed; tile += n_clusters) {
-        const int m0 = (tile / n_nt) * 2 * BM, n0 = (tile % n_nt) * C2_BN;
-        for (int kb = 0; kb < nk; ++kb) {
+      WorkIter wi(use_sk, cluster, n_clusters, n_tiles, nk);
+      Seg sg;
+      for (int it = 0; !failed && wi.next(sg); ++it) {
+        const int m0 = (sg.tile / n_nt) * 2 * BM, n0 = (sg.tile % n_nt) * C2_BN;
+        for (int kb = sg.kb0; kb < sg.kb1; ++kb) {
           uint8_t* sa = smem + stage * C2_STAGE_BYTES;
           const uint32_t fb = mapa_shared(smem_u32(&full[stage]), 0);
-          if (tile == cluster && kb < pre) {  // W already requested before the wait
+          if (it == 0 && kb - sg.kb0 < pre) {  // W already requested before the wait
             tma_load_2d_cg2(sa, &tmA, fb, kb * BK, m0 + BM * (int)rank);
             if (++stage == C2_STAGES) { stage = 0; phase ^= 1u; }
             continue;
@@ -365,21 +455,23 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
                              ((uint32_t)(C2_BN >> 3) << 17) | ((uint32_t)((2 * BM) >> 4) << 24);
       int stage = 0;
       uint32_t phase = 0;
-      int it = 0;
-      for (int tile = cluster; tile < n_tiles && !failed; tile += n_clusters, ++it) {
+      WorkIter wi(use_sk, cluster, n_clusters, n_tiles, nk);
+      Seg sg;
+      for (int it = 0; !failed && wi.next(sg); ++it) {
         const int acc = it & 1;
         const uint32_t acc_phase = (it >> 1) & 1;
         if (!mbar_wait(&tmem_empty[acc], acc_phase ^ 1u, err)) { failed = true; break; }
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + acc * C2_BN;
-        for (int kb = 0; kb < nk; ++kb) {
+        for (int kb = sg.kb0; kb < sg.kb1; ++kb) {
           if (!mbar_wait(&full[stage], phase, err)) { failed = true; break; }
           tc_fence_after();
           const uint32_t sa = smem_u32(smem + stage * C2_STAGE_BYTES);
           const uint64_t adesc = sdesc_sw128(sa), bdesc = sdesc_sw128(sa + C2_HALF_BYTES);
 #pragma unroll
           for (int k = 0; k < BK / 16; ++k)
-            tc_mma_f16_cg2(d_tmem, adesc + 2 * k, bdesc + 2 * k, idesc, (kb | k) ? 1u : 0u);
+            tc_mma_f16_cg2(d_tmem, adesc + 2 * k, bdesc + 2 * k, idesc,
+                           (kb > sg.kb0 || k > 0) ? 1u : 0u);
           tc_commit_mc(&empty[stage], 0x3);
           if (++stage == C2_STAGES) { stage = 0; phase ^= 1u; }
         }
@@ -388,38 +480,195 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
     }
   } else {
     // ---------------- epilogue (warps 2..9 of both CTAs) ----------------
-    const int quarter = warp & 3, half = (warp - 2) >> 2;
+    const int quarter = warp & 3, half = (warp - 2) >> 2, we = warp - 2;
     const uint32_t te_remote = mapa_shared(smem_u32(&tmem_empty[0]), 0);
-    int it = 0;
-    for (int tile = cluster; tile < n_tiles; tile += n_clusters, ++it) {
+    uint8_t* wtiles = epi_smem + we * 2 * CC::TILE_BYTES;  // this warp's two TMA tiles
+    uint32_t rl_phase = 0;                                 // bit b: parity of tile b's load
+    WorkIter wi(use_sk, cluster, n_clusters, n_tiles, nk);
+    Seg sg;
+    for (int it = 0; wi.next(sg); ++it) {
       const int acc = it & 1;
       const uint32_t acc_phase = (it >> 1) & 1;
+      const int tile = sg.tile;
+      const bool whole = sg.kb0 == 0 && sg.kb1 == nk;
       const int m0 = (tile / n_nt) * 2 * BM, n0 = (tile % n_nt) * C2_BN;
       const int prow = m0 + BM * (int)rank + quarter * 32 + lane;
-      // short-K tiles only: over a long mainloop the streamed operands evict the rows
-      if (nk <= 48 && prow < M) epi_prefetch<KIND>(epi, prow, n0 + half * (C2_BN / 2), C2_BN / 2);
+      const int row0 = m0 + BM * (int)rank + quarter * 32;
+      // residual chunk cc of this warp's rows into tile cc % 2 (one lane)
+      auto rload_issue = [&](int cc) {
+        const int b = cc & 1;
+        mbar_expect_tx(&rload[2 * we + b], CC::TILE_BYTES);
+        tma_load_2d(wtiles + b * CC::TILE_BYTES, &tmR, &rload[2 * we + b],
+                    n0 + (half * 4 + cc) * 32, row0);
+      };
+      // whole tiles: the first two residual chunks load while the mainloop runs
+      const bool early = KIND == EPI_RESID && whole && row0 < M;
+      if (early) {
+        if (lane == 0) {
+          bulk_wait_read<0>();
+          rload_issue(0);
+          rload_issue(1);
+        }
+        __syncwarp();
+      }
+      // Delta epilogue, short-K tiles only: the rows into L2 (over a long mainloop the
+      // streamed operands would evict them)
+      if (CC::STAGED && whole && nk <= 48 && prow < M)
+        epi_prefetch<KIND>(epi, prow, n0 + half * (C2_BN / 2), C2_BN / 2);
       const bool ok = mbar_wait(&tmem_full[acc], acc_phase, err);
       if (!__all_sync(0xffffffffu, ok)) { failed = true; break; }
       tc_fence_after();
-      const int row0 = m0 + BM * (int)rank + quarter * 32;
-      const int row = row0 + lane;
       const uint32_t taddr = tmem_base + ((uint32_t)(quarter * 32) << 16) + acc * C2_BN;
+      bool finish = whole;
+      int c_lo = 0, n_c = 1;
+      if (!whole) {
+        // a cut tile: publish this warp's partial, then count in on the tile's counter
+        c_lo = sk_owner((long long)tile * nk, U, n_clusters);
+        n_c = sk_owner((long long)(tile + 1) * nk - 1, U, n_clusters) - c_lo + 1;
+        float* part = sk_part(sk.ws, cluster, tile, U, n_clusters, nk, (int)rank, we);
 #pragma unroll 1
-      for (int c = half * (C2_BN / 64); c < (half + 1) * (C2_BN / 64); ++c) {
-        uint32_t r[32];
-        tmem_ld32(taddr + c * 32, r);
-        tmem_ld_wait();
-        reg_fence32(r);
-        float v[32];
+        for (int cc = 0; cc < 4; ++cc) {
+          uint32_t r[32];
+          tmem_ld32(taddr + (half * 4 + cc) * 32, r);
+          tmem_ld_wait();
+          reg_fence32(r);
+          float4* dst = reinterpret_cast<float4*>(part + cc * 1024) + lane;
 #pragma unroll
-        for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(r[j]);
-        if (CC::STAGED) {
-          if (row0 < M)
-            epi_resid_staged<KIND>(epi, epi_stage + (warp - 2) * EPI_STAGE_FLOATS, lane, row0,
-                                   n0 + c * 32, M, v);
-        } else if (row < M) {
-          epi_apply32<KIND>(epi, row, n0 + c * 32, v);
+          for (int j4 = 0; j4 < 8; ++j4)
+            dst[j4 * 32] = make_float4(__uint_as_float(r[4 * j4]), __uint_as_float(r[4 * j4 + 1]),
+                                       __uint_as_float(r[4 * j4 + 2]),
+                                       __uint_as_float(r[4 * j4 + 3]));
         }
+        __threadfence();
+        __syncwarp();
+        int* ctr = sk.ctr + ((size_t)c_lo * 2 + rank) * 8 + we;
+        int old = 0;
+        if (lane == 0) old = atomicAdd(ctr, 1);
+        old = __shfl_sync(0xffffffffu, old, 0);
+        finish = old == n_c - 1;
+        if (finish) {
+          __threadfence();
+          if (lane == 0) *ctr = 0;  // every contributor has counted in: ready for reuse
+        }
+      }
+      if (finish && row0 < M) {
+        if (KIND == EPI_RESID && !early) {
+          if (lane == 0) {
+            bulk_wait_read<0>();
+            for (int cc = 0; cc < 2; ++cc) rload_issue(cc);
+          }
+          __syncwarp();
+        }
+#pragma unroll 1
+        for (int cc = 0; cc < 4; ++cc) {
+          const int c = half * 4 + cc;
+          float v[32];
+          if (whole) {
+            uint32_t r[32];
+            tmem_ld32(taddr + c * 32, r);
+            tmem_ld_wait();
+            reg_fence32(r);
+#pragma unroll
+            for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(r[j]);
+          } else {
+            // the contributors' partials summed in K order, this cluster's from TMEM
+#pragma unroll
+            for (int j = 0; j < 32; ++j) v[j] = 0.f;
+#pragma unroll 1
+            for (int q = 0; q < n_c; ++q) {
+              const int cq = c_lo + q;
+              if (cq == cluster) {
+                uint32_t r[32];
+                tmem_ld32(taddr + c * 32, r);
+                tmem_ld_wait();
+                reg_fence32(r);
+#pragma unroll
+                for (int j = 0; j < 32; ++j) v[j] += __uint_as_float(r[j]);
+              } else {
+                const float4* src = reinterpret_cast<const float4*>(
+                                        sk_part(sk.ws, cq, tile, U, n_clusters, nk, (int)rank, we) +
+                                        cc * 1024) + lane;
+#pragma unroll
+                for (int j4 = 0; j4 < 8; ++j4) {
+                  const float4 f = __ldcg(src + j4 * 32);
+                  v[4 * j4] += f.x;
+                  v[4 * j4 + 1] += f.y;
+                  v[4 * j4 + 2] += f.z;
+                  v[4 * j4 + 3] += f.w;
+                }
+              }
+            }
+          }
+          const int col0 = n0 + c * 32;
+          if (CC::STAGED) {
+            epi_resid_staged<KIND>(epi, epi_stage + we * EPI_STAGE_FLOATS, lane, row0, col0, M, v);
+            continue;
+          }
+          const int b = cc & 1;
+          uint8_t* tile_b = wtiles + b * CC::TILE_BYTES;
+          float bv[32];
+#pragma unroll
+          for (int j = 0; j < 32; j += 8) {
+            if (epi.bias) load_f32x8(epi.bias + col0 + j, bv + j);
+            else {
+#pragma unroll
+              for (int q = 0; q < 8; ++q) bv[j + q] = 0.f;
+            }
+          }
+          if (KIND == EPI_RESID) {
+            float gv[32];
+#pragma unroll
+            for (int j = 0; j < 32; j += 8) {
+              if (epi.gate) load_f32x8(epi.gate + col0 + j, gv + j);
+              else {
+#pragma unroll
+                for (int q = 0; q < 8; ++q) gv[j + q] = 1.f;
+              }
+            }
+            const bool lok = mbar_wait(&rload[2 * we + b], (rl_phase >> b) & 1u, err);
+            rl_phase ^= 1u << b;
+            if (!__all_sync(0xffffffffu, lok)) { failed = true; break; }
+#pragma unroll
+            for (int j4 = 0; j4 < 8; ++j4) {
+              float4* p4 = reinterpret_cast<float4*>(tile_b + swz128(lane, j4));
+              float4 o = *p4;
+              o.x += gv[4 * j4] * (v[4 * j4] + bv[4 * j4]);
+              o.y += gv[4 * j4 + 1] * (v[4 * j4 + 1] + bv[4 * j4 + 1]);
+              o.z += gv[4 * j4 + 2] * (v[4 * j4 + 2] + bv[4 * j4 + 2]);
+              o.w += gv[4 * j4 + 3] * (v[4 * j4 + 3] + bv[4 * j4 + 3]);
+              *p4 = o;
+            }
+          } else {
+            // the store issued from this tile two chunks ago has left shared memory (the
+            // one outstanding group allowed is the other tile's, one chunk ago)
+            if (lane == 0) bulk_wait_read<1>();
+            __syncwarp();
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+              float y[8];
+#pragma unroll
+              for (int i = 0; i < 8; ++i) {
+                y[i] = v[8 * q + i] + bv[8 * q + i];
+                if (KIND == EPI_GELU_BF16) y[i] = gelu_tanh_f(y[i]);
+              }
+              *reinterpret_cast<uint4*>(tile_b + swz64(lane, q)) =
+                  make_uint4(pack_bf16x2(y[0], y[1]), pack_bf16x2(y[2], y[3]),
+                             pack_bf16x2(y[4], y[5]), pack_bf16x2(y[6], y[7]));
+            }
+          }
+          fence_proxy_async_smem();
+          __syncwarp();
+          if (lane == 0) {
+            tma_store_2d(&tmO, smem_u32(tile_b), col0, row0);
+            bulk_commit();
+            if (KIND == EPI_RESID && cc + 2 < 4) {
+              bulk_wait_read<0>();  // the tile is free again: next residual chunk into it
+              rload_issue(cc + 2);
+            }
+          }
+          __syncwarp();
+        }
+        if (failed) break;
       }
       tc_fence_before();
       __syncwarp();
@@ -427,6 +676,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
     }
   }
 
+  if (CC::TMA_EPI && warp >= 2 && lane == 0) bulk_wait<0>();  // own TMA stores complete
   if (failed || *(volatile int*)err != 0) {
     // After a timeout, give TMA loads that may still be in flight time to land before
     // the shared memory they target is released (they complete within microseconds).
@@ -495,10 +745,35 @@ cudaError_t dispatch_kind(const GemmArgs& g, int* err, int num_sms, cudaStream_t
   return cudaErrorInvalidValue;
 }
 
+// 2-D map over an epilogue matrix [rows][cols] (row stride ld elements) with 32 x 32
+// boxes: fp32 with the 128-byte swizzle, bf16 with the 64-byte swizzle.
+bool make_epi_map(CUtensorMap* map, const void* ptr, bool f32, int rows, int cols, int ld) {
+  auto enc = get_encode();
+  if (!enc) return false;
+  const size_t es = f32 ? 4 : 2;
+  cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
+  cuuint64_t strides[1] = {(cuuint64_t)ld * es};
+  cuuint32_t box[2] = {32, 32};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = enc(map, f32 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16,
+                   2, const_cast<void*>(ptr), dims, strides, box, estr,
+                   CU_TENSOR_MAP_INTERLEAVE_NONE,
+                   f32 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_64B,
+                   CU_TENSOR_MAP_L2_PROMOTION_L2_128B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
 template <int KIND>
 cudaError_t launch2(const GemmArgs& g, int* err, int num_sms, cudaStream_t st) {
-  CUtensorMap ma, mw;
+  CUtensorMap ma, mw, mo, mr;
+  memset(&mo, 0, sizeof(mo));
+  memset(&mr, 0, sizeof(mr));
   if (!make_map(&ma, g.A, g.M, g.K, g.lda, BM) || !make_map(&mw, g.W, g.N, g.K, g.ldw, 128))
+    return cudaErrorInvalidValue;
+  if (C2Cfg<KIND>::TMA_EPI &&
+      !make_epi_map(&mo, g.epi.out, KIND == EPI_RESID, g.M, g.N, g.epi.ldo))
+    return cudaErrorInvalidValue;
+  if (KIND == EPI_RESID && !make_epi_map(&mr, g.epi.resid, true, g.M, g.N, g.epi.ldo))
     return cudaErrorInvalidValue;
   constexpr int C2_SMEM_BYTES = C2Cfg<KIND>::SMEM_BYTES;
   cudaError_t e = cudaFuncSetAttribute(gemm_tc2_kernel<KIND>,
@@ -520,9 +795,21 @@ cudaError_t launch2(const GemmArgs& g, int* err, int num_sms, cudaStream_t st) {
     mc = n < num_sms / 2 ? n : num_sms / 2;
   }
   const int tiles = ((g.M + 2 * BM - 1) / (2 * BM)) * (g.N / C2_BN);
-  const int clusters = tiles < mc ? tiles : mc;
+  const int nk = g.K / BK;
+  SkArgs sk{0, g.sk_ws, g.sk_ctr};
+  // Stream-K only on request (sk_mode 2): with every SM busy the mainloop's K blocks
+  // take longer and the partial write-back and sum of a cut tile cost more than the
+  // idle pairs of a short last wave save (measured at 1560 x 1536 x {1536, 8960}).
+  const long long U = (long long)tiles * nk;
+  const bool sk_ok = g.sk_ws && g.sk_ctr && mc <= g.sk_clusters && U >= 4LL * mc;
+  if (g.sk_mode == 2) {
+    if (!sk_ok) return cudaErrorInvalidValue;
+    sk.on = 1;
+  }
+  (void)nk;
+  const int clusters = sk.on ? mc : (tiles < mc ? tiles : mc);
   return launch_k(gemm_tc2_kernel<KIND>, dim3(2 * clusters), dim3(NUM_THREADS), C2_SMEM_BYTES, st,
-                  ma, mw, g.M, g.N, g.K, g.epi, err);
+                  ma, mw, mo, mr, g.M, g.N, g.K, g.epi, sk, err);
 }
 
 cudaError_t dispatch2(const GemmArgs& g, int* err, int num_sms, cudaStream_t st) {
@@ -540,7 +827,9 @@ cudaError_t dispatch2(const GemmArgs& g, int* err, int num_sms, cudaStream_t st)
 bool gemm_tc_supported(const GemmArgs& g) {
   auto al16 = [](const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15) == 0; };
   return g.M >= 1 && g.N % 128 == 0 && g.K % BK == 0 && g.K >= BK && g.lda % 8 == 0 &&
-         g.ldw % 8 == 0 && g.epi.ldo % 8 == 0 && al16(g.A) && al16(g.W) && al16(g.epi.out);
+         g.ldw % 8 == 0 && g.epi.ldo % 8 == 0 && al16(g.A) && al16(g.W) && al16(g.epi.out) &&
+         (g.kind < EPI_RESID || al16(g.epi.resid)) &&
+         (g.kind != EPI_RESID_DELTA || (al16(g.epi.base) && al16(g.epi.delta)));
 }
 
 cudaError_t gemm_tc(const GemmArgs& g, int* err, int num_sms, cudaStream_t st, bool force_1sm) {
@@ -548,6 +837,7 @@ cudaError_t gemm_tc(const GemmArgs& g, int* err, int num_sms, cudaStream_t st, b
   // 2-SM 256 x 256 tiles whenever N allows; otherwise 1-SM 128 x BN tiles, BN = 256
   // when that still gives every SM a tile.
   if (g.N % C2_BN == 0 && !force_1sm && num_sms >= 2) return dispatch2(g, err, num_sms, st);
+  if (g.sk_mode == 2) return cudaErrorInvalidValue;  // stream-K exists in the 2-SM kernel only
   const int mt = (g.M + BM - 1) / BM;
   if (g.N % 256 == 0 && mt * (g.N / 256) >= num_sms) return dispatch_kind<256>(g, err, num_sms, st);
   return dispatch_kind<128>(g, err, num_sms, st);

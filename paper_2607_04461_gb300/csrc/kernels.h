@@ -16,7 +16,17 @@ struct GemmArgs {
   int ldw;
   int kind;       // EPI_*
   GemmEpi epi;
+  // Stream-K workspace of the 2-SM kernel (null: data-parallel tiles only): room for
+  // sk_clusters clusters (sk_clusters * 131072 floats) and sk_clusters * 16 counters that
+  // start at zero and are left at zero. sk_mode: 0 automatic, 1 never, 2 always.
+  float* sk_ws;
+  int* sk_ctr;
+  int sk_clusters;
+  int sk_mode;
 };
+// floats and counters of the stream-K workspace per cluster
+constexpr size_t SK_WS_FLOATS_PER_CLUSTER = 2 * 2 * 8 * 4096;
+constexpr int SK_CTR_PER_CLUSTER = 16;
 // tcgen05 path: requires N % 128 == 0, K % 64 == 0, 16-byte aligned rows. Uses the
 // 2-SM (cta_group::2) kernel when N % 256 == 0 unless force_1sm.
 bool gemm_tc_supported(const GemmArgs& g);
@@ -33,6 +43,7 @@ struct AttnArgs {
   int batch, Lq, Lkv;
   int kv_batch_rows;       // row offset of batch b's K/V (0 = shared)
   int heads, head_dim;
+  int tc_variant;          // tcgen05 kernel: 0 automatic, 1 128-query CTAs, 2 256-query CTAs
 };
 // mma.sync (warp-level) kernel: head_dim 64 or 128.
 cudaError_t attention(const AttnArgs& a, cudaStream_t st);

@@ -59,6 +59,60 @@ def test_gemm_tc_2sm_ragged_rows(model, M):
     _gemm_case(model, M, 512, 128, 0, impl=0)
 
 
+# Stream-K shapes: the refine pass's one-candidate projections (1560 rows), a few tiles
+# over a long K (13 pairs per tile), and two tiles over K = 9728 (about 38 pairs each).
+SK_SHAPES = [(1560, 1536, 1536), (1560, 1536, 8960), (1560, 8960, 1536), (1560, 4608, 1536),
+             (513, 512, 8960), (300, 256, 9728)]
+
+
+@pytest.mark.parametrize("M,N,K", SK_SHAPES)
+@pytest.mark.parametrize("epi", [0, 1, 2, 3])
+def test_gemm_tc_stream_k_forced(model, M, N, K, epi):
+    _gemm_case(model, M, N, K, epi, impl=4)
+
+
+@pytest.mark.parametrize("M,N,K", SK_SHAPES[:2] + SK_SHAPES[-1:])
+def test_gemm_stream_k_is_deterministic_and_matches_whole_tiles(model, M, N, K):
+    """Cut tiles are summed in K order, so two runs agree bit for bit; whole-tile runs
+    (impl 3) differ only by the fp32 summation order."""
+    A = randn((M, K), 21)
+    W = randn((N, K), 22, scale=K ** -0.5)
+    resid = randn((M, N), 23, dtype=torch.float32)
+    outs = []
+    for impl in (4, 4, 3):
+        out = torch.empty((M, N), dtype=torch.float32, device="cuda")
+        fb.fb_op_gemm(model.handle, M, N, K, A, W, None, 2, out, resid, None, None, None, impl)
+        outs.append(out)
+    torch.cuda.synchronize()
+    assert torch.equal(outs[0], outs[1])
+    assert rel_max(f64(outs[0]), f64(outs[2])) <= 1e-5
+
+
+def test_gemm_stream_k_in_place_residual(model):
+    M, N, K = 1560, 1536, 8960
+    A, W = randn((M, K), 31), randn((N, K), 32, scale=K ** -0.5)
+    h = randn((M, N), 33, dtype=torch.float32)
+    h0 = f64(h)
+    gate = randn((N,), 34, dtype=torch.float32)
+    delta = torch.empty((M, N), dtype=torch.bfloat16, device="cuda")
+    fb.fb_op_gemm(model.handle, M, N, K, A, W, None, 3, h, h, gate, h, delta, 4)
+    torch.cuda.synchronize()
+    want = h0 + f64(gate) * O.linear(f64(A), f64(W))
+    assert rel_max(f64(h), want) <= 1e-4
+    assert rel_max(f64(delta), want - h0) <= 1e-2
+
+
+@pytest.mark.parametrize("M,N,K", [(300, 256, 128), (300, 384, 9728)])
+def test_gemm_stream_k_forced_rejects(model, M, N, K):
+    """Too few K blocks per SM pair, or N not a multiple of 256: an error, no launch."""
+    A, W = randn((M, K), 41), randn((N, K), 42)
+    out = torch.zeros((M, N), dtype=torch.bfloat16, device="cuda")
+    with pytest.raises(fb.FlashBonError) as e:
+        fb.fb_op_gemm(model.handle, M, N, K, A, W, None, 0, out, None, None, None, None, 4)
+    assert e.value.status == fb.FB_ECUDA
+    _gemm_case(model, M, N, K, 0, impl=0)   # the model is still usable
+
+
 @pytest.mark.parametrize("M,N,K", [(300, 256, 128), (77, 24, 40)])
 @pytest.mark.parametrize("epi", [0, 1, 2, 3])
 def test_gemm_simt(model, M, N, K, epi):
@@ -115,7 +169,7 @@ ATTN_CASES = [
     (2, 1560, 1560, 2, 128, False),   # Wan2.1 self-attention length, ragged last tile
     (3, 256, 128, 1, 128, False),     # exact tile multiples
     (2, 129, 257, 2, 128, True),      # one row / one key past a tile
-    # grids of >= 2 CTAs per SM take the 256-query kernel (P kept in TMEM)
+    # grids of more than one wave of 128-query CTAs take the 256-query kernel (P in TMEM)
     (4, 1560, 1560, 12, 128, False),
     (9, 600, 512, 12, 128, True),     # last CTA: tile A partly valid, tile B past Lq
 ]
@@ -139,10 +193,17 @@ def test_attention_large_logits(model):
         assert rel_max(on[sl], want) <= 2e-2
 
 
-@pytest.mark.parametrize("impl", [0, 1], ids=["auto", "mma_sync"])
+@pytest.mark.parametrize("impl", [0, 1, 2, 3], ids=["auto", "mma_sync", "tc_q128", "tc_q256"])
 @pytest.mark.parametrize("batch,Lq,Lkv,heads,dh,shared", ATTN_CASES)
 def test_attention(model, batch, Lq, Lkv, heads, dh, shared, impl):
     D = heads * dh
+    if impl >= 2 and dh != 128:
+        z = torch.zeros((batch * max(Lq, Lkv), D), dtype=torch.bfloat16, device="cuda")
+        with pytest.raises(fb.FlashBonError) as e:
+            fb.fb_op_attention(model.handle, z, D, z, D, z, D, z, D, batch, Lq, Lkv, 0, heads,
+                               dh, impl)
+        assert e.value.status == fb.FB_EINVAL
+        return
     q = randn((batch * Lq, D), 21)
     kvb = 1 if shared else batch
     k = randn((kvb * Lkv, D), 22)
