@@ -245,6 +245,32 @@ fb_status fb_op_attention(fb_model* m, const void* Q, int ldq, const void* K, in
                           const void* V, int ldv, void* O, int ldo, int batch, int Lq,
                           int Lkv, int kv_batch_rows, int heads, int head_dim, int impl);
 
+/* ---- allocation-free stream-K GEMM (an engineering entry point: the paper has no
+ * counterpart; it computes what fb_op_gemm with impl 4 computes) ---------------------
+ * fb_gemm_streamk_noalloc: the same D = epi(A W^T + bias) as fb_op_gemm (same epi codes,
+ * argument meaning and DEVICE-pointer layouts) with the stream-K split of the 2-SM
+ * kernel, but with no model and no allocation of any kind: the partial accumulators,
+ * the per-tile counters and the device error word live in static device arrays of the
+ * library, sized for at most FB_NOALLOC_MAX_PAIRS SM pairs (76, a full GB300: 39.8 MB of
+ * fp32 partials, 76 x 16 counters). Their addresses are looked up once per device on the
+ * first call (cudaGetSymbolAddress, checked). The work is enqueued on `stream` (a
+ * cudaStream_t; NULL = the legacy default stream) and the call waits for it, then reads
+ * the error word.
+ * State: the counters must be zero when a call starts; they are zero at load, every
+ * successful call leaves them zero, and a call that reports a device error clears
+ * them before returning. The error word is cleared at the start of every call. Calls
+ * that overlap in time (other host threads, other streams) share these arrays and race:
+ * serialise them.
+ * Errors: FB_EINVAL for a NULL pointer, a bad epi, N % 256 != 0, shapes the tcgen05
+ * kernel does not take (K % 64, alignment), fewer than 4 K blocks per SM pair
+ * (ceil(M / 256) * N / 256 * K / 64 < 4 * pairs) or a device with more than
+ * FB_NOALLOC_MAX_PAIRS pairs; FB_ECUDA for a CUDA error or a device wait timeout. */
+#define FB_NOALLOC_MAX_PAIRS 76
+fb_status fb_gemm_streamk_noalloc(void* stream, int M, int N, int K, const void* A,
+                                  const void* W, const float* bias, int epi, void* out,
+                                  const float* resid, const float* gate, const float* base,
+                                  void* delta);
+
 #ifdef __cplusplus
 }
 #endif

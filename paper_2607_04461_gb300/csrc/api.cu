@@ -16,6 +16,7 @@
 #include <cstdlib>
 #include <cstring>
 #include <map>
+#include <mutex>
 #include <string>
 #include <vector>
 
@@ -1044,6 +1045,94 @@ fb_status fb_op_attention(fb_model* m, const void* Q, int ldq, const void* K, in
   CKS(begin_call(m));
   for (int r = 0; r < m->op_repeat; ++r) CKS(run_attn(m, a, FB_K_ATTN_SELF, impl));
   return end_call(m);
+}
+
+}  // extern "C"
+
+// ---- allocation-free stream-K GEMM --------------------------------------------------
+namespace {
+// Static device state of fb_gemm_streamk_noalloc: partials for FB_NOALLOC_MAX_PAIRS SM
+// pairs, their per-tile counters (zero at load, left zero by every launch) and an error
+// word. Shared by all calls on a device, so overlapping calls race.
+static __device__ __align__(256) float g_na_ws[FB_NOALLOC_MAX_PAIRS * SK_WS_FLOATS_PER_CLUSTER];
+static __device__ __align__(256) int g_na_ctr[FB_NOALLOC_MAX_PAIRS * SK_CTR_PER_CLUSTER];
+static __device__ __align__(256) int g_na_err[1];
+
+struct NoAllocDev {
+  bool ready = false;
+  float* ws = nullptr;
+  int* ctr = nullptr;
+  int* err = nullptr;
+  int num_sms = 0;
+};
+constexpr int kNoAllocDevices = 64;
+NoAllocDev g_na_dev[kNoAllocDevices];
+std::mutex g_na_mu;
+
+// Symbol addresses and SM count of the current device, looked up once per device.
+fb_status noalloc_setup(NoAllocDev** out) {
+  int dev = 0;
+  CK(cudaGetDevice(&dev));
+  if (dev < 0 || dev >= kNoAllocDevices) return fail(FB_EINVAL, "device %d out of range", dev);
+  std::lock_guard<std::mutex> lock(g_na_mu);
+  NoAllocDev& d = g_na_dev[dev];
+  if (!d.ready) {
+    CK(cudaGetSymbolAddress(reinterpret_cast<void**>(&d.ws), g_na_ws));
+    CK(cudaGetSymbolAddress(reinterpret_cast<void**>(&d.ctr), g_na_ctr));
+    CK(cudaGetSymbolAddress(reinterpret_cast<void**>(&d.err), g_na_err));
+    CK(cudaDeviceGetAttribute(&d.num_sms, cudaDevAttrMultiProcessorCount, dev));
+    d.ready = true;
+  }
+  *out = &d;
+  return FB_OK;
+}
+}  // namespace
+
+extern "C" {
+
+fb_status fb_gemm_streamk_noalloc(void* stream, int M, int N, int K, const void* A,
+                                  const void* W, const float* bias, int epi, void* out,
+                                  const float* resid, const float* gate, const float* base,
+                                  void* delta) {
+  if (!A || !W || !out) return fail(FB_EINVAL, "null argument");
+  if (M < 1 || N < 1 || K < 1 || epi < 0 || epi > 3) return fail(FB_EINVAL, "bad sizes / epi");
+  if (epi >= EPI_RESID && !resid) return fail(FB_EINVAL, "resid required");
+  if (epi == EPI_RESID_DELTA && (!base || !delta)) return fail(FB_EINVAL, "base/delta required");
+  if (N % 256) return fail(FB_EINVAL, "N must be a multiple of 256");
+  GemmArgs g = gemm_args(M, N, K, (const bf16*)A, (const bf16*)W, bias, epi, out);
+  g.epi.resid = resid;
+  g.epi.gate = gate;
+  g.epi.base = base;
+  g.epi.delta = (bf16*)delta;
+  if (!gemm_tc_supported(g)) return fail(FB_EINVAL, "shape or alignment not supported");
+  NoAllocDev* d = nullptr;
+  CKS(noalloc_setup(&d));
+  const int pairs = d->num_sms / 2;
+  if (pairs > FB_NOALLOC_MAX_PAIRS)
+    return fail(FB_EINVAL, "%d SM pairs: the static workspace holds %d", pairs,
+                FB_NOALLOC_MAX_PAIRS);
+  const long long units = (long long)((M + 255) / 256) * (N / 256) * (K / 64);
+  if (units < 4LL * pairs)
+    return fail(FB_EINVAL, "%lld (tile, K block) units: stream-K needs >= %d", units, 4 * pairs);
+  g.sk_ws = d->ws;
+  g.sk_ctr = d->ctr;
+  g.sk_clusters = FB_NOALLOC_MAX_PAIRS;
+  g.sk_mode = 2;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  fb_stream_op_not_kernel();
+  CK(cudaMemsetAsync(d->err, 0, sizeof(int), st));
+  CK(gemm_tc(g, d->err, d->num_sms, st, false));
+  int herr = 0;
+  fb_stream_op_not_kernel();
+  CK(cudaMemcpyAsync(&herr, d->err, sizeof(int), cudaMemcpyDeviceToHost, st));
+  CK(cudaStreamSynchronize(st));
+  if (herr != 0) {
+    CK(cudaMemsetAsync(d->ctr, 0, sizeof(int) * FB_NOALLOC_MAX_PAIRS * SK_CTR_PER_CLUSTER, st));
+    CK(cudaStreamSynchronize(st));
+    return fail(FB_ECUDA, herr == FB_DEVERR_WAIT_TIMEOUT ? "device wait timed out"
+                                                         : "device error %d", herr);
+  }
+  return FB_OK;
 }
 
 fb_status fb_set_op_repeat(fb_model* m, int n) {

@@ -50,7 +50,7 @@ EXPORTS = ["fb_weights_count", "fb_weights_entry", "fb_init_model", "fb_free", "
            "fb_encode_text", "fb_draft", "fb_refine", "fb_plan_from_phi", "fb_block_forward",
            "fb_last_error", "fb_set_timing", "fb_get_stats", "fb_reset_stats", "fb_kernel_name",
            "fb_op_gemm", "fb_op_attention", "fb_draft_ex", "fb_refine_ex", "fb_select_elo",
-           "fb_set_op_repeat"]
+           "fb_set_op_repeat", "fb_gemm_streamk_noalloc"]
 
 PAIR_VERIFIER = ctypes.CFUNCTYPE(ctypes.c_int, ctypes.c_void_p, ctypes.c_int, ctypes.c_int,
                                  ctypes.POINTER(ctypes.c_int))
@@ -91,6 +91,7 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
         "fb_kernel_name": (ctypes.c_char_p, [I]),
         "fb_op_gemm": (I, [P, I, I, I, P, P, P, I, P, P, P, P, P, I]),
         "fb_op_attention": (I, [P, P, I, P, I, P, I, P, I, I, I, I, I, I, I, I]),
+        "fb_gemm_streamk_noalloc": (I, [P, I, I, I, P, P, P, I, P, P, P, P, P]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(L, name)
@@ -277,6 +278,15 @@ def fb_op_gemm(model, M, N, K, A, W, bias, epi, out, resid=None, gate=None, base
     _check(load_library().fb_op_gemm(model, M, N, K, _ptr(A), _ptr(W), _ptr(bias), epi,
                                      _ptr(out), _ptr(resid), _ptr(gate), _ptr(base),
                                      _ptr(delta), impl))
+
+
+def fb_gemm_streamk_noalloc(stream, M, N, K, A, W, bias, epi, out, resid=None, gate=None,
+                            base=None, delta=None) -> None:
+    """The allocation-free stream-K GEMM (no model); `stream` is a cudaStream_t handle
+    (int) or None for the legacy default stream. Waits for the result."""
+    _check(load_library().fb_gemm_streamk_noalloc(stream, M, N, K, _ptr(A), _ptr(W),
+                                                  _ptr(bias), epi, _ptr(out), _ptr(resid),
+                                                  _ptr(gate), _ptr(base), _ptr(delta)))
 
 
 def fb_op_attention(model, Q, ldq, Kt, ldk, V, ldv, O, ldo, batch, Lq, Lkv, kv_batch_rows,
