@@ -175,7 +175,8 @@ ATTN_CASES = [
 ]
 
 
-def test_attention_large_logits(model):
+@pytest.mark.parametrize("impl", [0, 3], ids=["auto", "tc_q256"])
+def test_attention_large_logits(model, impl):
     """Scores spanning many powers of two exercise the rescaling of O."""
     batch, L, heads, dh = 2, 400, 2, 128
     D = heads * dh
@@ -183,7 +184,7 @@ def test_attention_large_logits(model):
     k = randn((batch * L, D), 42, scale=4.0)
     v = randn((batch * L, D), 43)
     o = torch.empty((batch * L, D), dtype=torch.bfloat16, device="cuda")
-    fb.fb_op_attention(model.handle, q, D, k, D, v, D, o, D, batch, L, L, L, heads, dh)
+    fb.fb_op_attention(model.handle, q, D, k, D, v, D, o, D, batch, L, L, L, heads, dh, impl)
     torch.cuda.synchronize()
     qn, kn, vn, on = f64(q), f64(k), f64(v), f64(o)
     for b in range(batch):
