@@ -46,6 +46,10 @@ Readings where the paper is silent or ambiguous (all arithmetic in fp64):
   R8 Elo selection (§4.2 Stage 2): base K and the expected-score formula are not given;
      K = 32 and the logistic 400-point expected score are used; the adjacent comparisons
      are passes over the rating-sorted survivors; ties go to the lower index.
+  R9 cached state (§4.2 Stage 3): the optional layer activations kept for warm-starting
+     activation proxies are, under R1, each layer's contribution Delta_l from its last
+     computed draft step, with that step's t. A refine step may proxy layer l from it
+     (order 0: h <- h + Delta_l); with no such steps the refine is phi_full exactly.
 """
 from __future__ import annotations
 
@@ -53,6 +57,7 @@ import numpy as np
 
 F64 = np.float64
 COMPUTE = -1
+STATE_SRC = 0xFFFF  # proxy source: the cached state of an earlier call (R9), order 0
 
 
 # ----------------------------------------------------------------------------------
@@ -209,10 +214,12 @@ def plan_from_phi(S, S_prime, n_skip, l_start, l_end, f_full, order, depth):
     return skip, proxy
 
 
-def resolve_plan(skip, proxy):
+def resolve_plan(skip, proxy, state_layers=()):
     """Validate a plan and list, per proxied (step, layer), its anchor steps (most recent
-    first). Raises ValueError on: skip and proxy both set; source step not earlier than
-    the step; layer not computed at the source step; order outside 0..2."""
+    first); a proxy from the cached state (source STATE_SRC, R9) has the anchor "state".
+    Raises ValueError on: skip and proxy both set; source step not earlier than the step;
+    layer not computed at the source step; order outside 0..2; a state proxy of order > 0
+    or of a layer the state does not hold."""
     skip = np.asarray(skip)
     proxy = np.asarray(proxy)
     S, L = skip.shape
@@ -230,6 +237,11 @@ def resolve_plan(skip, proxy):
             if code < 0:
                 raise ValueError(f"step {k} layer {l}: bad proxy code {code}")
             src, order = code & 0xFFFF, code >> 16
+            if src == STATE_SRC:
+                if order != 0 or l not in state_layers:
+                    raise ValueError(f"step {k} layer {l}: bad proxy from the cached state")
+                anchors[(k, l)] = ["state"]
+                continue
             if order > 2:
                 raise ValueError(f"step {k} layer {l}: order {order} > 2")
             if src >= k:
@@ -326,9 +338,11 @@ class OracleModel:
         return linear(a, w["head.w"], w["head.b"])
 
     # -- sampler ----------------------------------------------------------------------
-    def _blocks(self, i, h, t, mod, ctx_kv, skip, proxy, anchors, needed, cache, trace):
+    def _blocks(self, i, h, t, mod, ctx_kv, skip, proxy, anchors, needed, cache, trace,
+                last=None):
         """Blocks of step i on h: skip (Eq. 6), compute (Eq. 7, caching Delta_l when a
-        later proxy needs it) or proxy (Eqs. 3-5)."""
+        later proxy needs it; with `last`, also recording each layer's latest (t, Delta_l),
+        R9) or proxy (Eqs. 3-5)."""
         for l in range(self.cfg.depth):
             if skip[i][l]:
                 continue
@@ -336,37 +350,52 @@ class OracleModel:
                 h_new = self.block(l, h, mod, ctx_kv[l])
                 if (i, l) in needed:
                     cache[(i, l)] = (t, h_new - h)
+                if last is not None:
+                    last[l] = (t, h_new - h)
                 h = h_new
             else:
-                h = h + taylor_forecast([cache[(s, l)] for s in anchors[(i, l)]], t)
+                h = h + taylor_forecast([cache[(s, l)] if s != "state" else cache[("state", l)]
+                                         for s in anchors[(i, l)]], t)
             if trace is not None:
                 trace.append((i, l, h.copy()))
         return h
 
     def sample_one(self, z, ctx_kv, schedule, skip, proxy, trace=None, ctx_kv_uncond=None,
-                   guidance=1.0, sde_a=0.0, noise=None):
+                   guidance=1.0, sde_a=0.0, noise=None, keep_state=False, state=None):
         """One candidate through len(schedule)-1 steps under (skip, proxy).
 
         Step i goes from t = schedule[i] to t' = schedule[i+1]: h_0 = PatchEmbed(z);
         the blocks; v = Head(h); z <- z + (t' - t) v (the Euler step of dx = v dt).
         With ctx_kv_uncond the step runs a second, unconditional pass with its own proxy
         cache and uses the guided velocity (R6). With sde_a > 0 the step is App. A.1's
-        Euler-Maruyama update with the standard normal draws noise[i] (R7)."""
+        Euler-Maruyama update with the standard normal draws noise[i] (R7).
+
+        keep_state: also return the cached state, {layer: (t, Delta_l)} of each layer's
+        last computed step (R9; the conditional pass). state: such a dict, the source of
+        proxies coded STATE_SRC (single pass only)."""
         cfg = self.cfg
         sched = np.asarray(schedule, F64)
         n_steps = len(sched) - 1
-        anchors = resolve_plan(skip, proxy)
-        needed = {(s, l) for (k, l), steps in anchors.items() for s in steps}
+        if state is not None and ctx_kv_uncond is not None:
+            raise ValueError("a cached state warm-starts a single (unguided) pass")
+        anchors = resolve_plan(skip, proxy, () if state is None else tuple(state))
+        needed = {(s, l) for (k, l), steps in anchors.items() for s in steps if s != "state"}
         passes = [ctx_kv] if ctx_kv_uncond is None else [ctx_kv, ctx_kv_uncond]
         caches = [{} for _ in passes]
+        if state is not None:
+            for l, tl_d in state.items():
+                caches[0][("state", l)] = tl_d
+        last = {} if keep_state else None
         z = np.asarray(z, F64).copy()
         for i in range(n_steps):
             t, t_next = sched[i], sched[i + 1]
             temb, mod = self.time_embed(t)
             vs = []
             for kv, cache in zip(passes, caches):
+                cond = kv is ctx_kv
                 h = self._blocks(i, self.patch_embed(z), t, mod, kv, skip, proxy, anchors,
-                                 needed, cache, trace if kv is ctx_kv else None)
+                                 needed, cache, trace if cond else None,
+                                 last if cond else None)
                 vs.append(unpatchify(self.head(h, temb), cfg.latent_c, cfg.latent_h,
                                      cfg.latent_w, cfg.patch))
             v = vs[0] if len(vs) == 1 else guided_velocity(vs[0], vs[1], guidance)
@@ -374,33 +403,46 @@ class OracleModel:
                 z = euler_maruyama_step(z, v, t, t_next, sde_a, np.asarray(noise[i], F64))
             else:
                 z = z + (t_next - t) * v
-        return z
+        return (z, last) if keep_state else z
 
     def draft(self, z_T, ctx, schedule, skip, proxy, candidates=None, ctx_uncond=None,
-              guidance=1.0, sde_a=0.0, noise=None):
+              guidance=1.0, sde_a=0.0, noise=None, keep_state=False):
         """Stage 1 (Eq. 8): each candidate's z_T through the truncated, accelerated
         schedule. Candidates are independent; `candidates` picks a subset. noise, when
-        sde_a > 0, is [n_steps][N][C][H][W] (indexed by the candidate's position in z_T)."""
+        sde_a > 0, is [n_steps][N][C][H][W] (indexed by the candidate's position in z_T).
+        keep_state: also return each candidate's cached state (R9), a list of dicts."""
         z_T = np.asarray(z_T)
         idx = range(z_T.shape[0]) if candidates is None else candidates
         kv = self.encode_text(ctx)
         kvu = None if ctx_uncond is None else self.encode_text(ctx_uncond)
-        out = []
+        out, states = [], []
         for j in idx:
             nz = None if noise is None else np.asarray(noise)[:, j]
-            out.append(self.sample_one(z_T[j], kv, schedule, skip, proxy, ctx_kv_uncond=kvu,
-                                       guidance=guidance, sde_a=sde_a, noise=nz))
-        return np.stack(out)
+            r = self.sample_one(z_T[j], kv, schedule, skip, proxy, ctx_kv_uncond=kvu,
+                                guidance=guidance, sde_a=sde_a, noise=nz, keep_state=keep_state)
+            if keep_state:
+                out.append(r[0])
+                states.append(r[1])
+            else:
+                out.append(r)
+        return (np.stack(out), states) if keep_state else np.stack(out)
 
-    def refine(self, z, ctx, schedule, ctx_uncond=None, guidance=1.0, sde_a=0.0, noise=None):
+    def refine(self, z, ctx, schedule, ctx_uncond=None, guidance=1.0, sde_a=0.0, noise=None,
+               state=None, warm_steps=0):
         """Stage 3: resume from a cached latent with phi_full (no skip, no proxy).
-        noise, when sde_a > 0, is [n_steps][C][H][W]."""
+        noise, when sde_a > 0, is [n_steps][C][H][W]. With a cached state (R9) the first
+        warm_steps steps proxy every layer the state holds from it (order 0)."""
         n = len(schedule) - 1
         skip = np.zeros((n, self.cfg.depth), np.uint8)
         proxy = np.full((n, self.cfg.depth), COMPUTE, np.int32)
+        if state is not None:
+            for i in range(min(warm_steps, n)):
+                for l in state:
+                    proxy[i, l] = STATE_SRC
         kvu = None if ctx_uncond is None else self.encode_text(ctx_uncond)
         return self.sample_one(z, self.encode_text(ctx), schedule, skip, proxy,
-                               ctx_kv_uncond=kvu, guidance=guidance, sde_a=sde_a, noise=noise)
+                               ctx_kv_uncond=kvu, guidance=guidance, sde_a=sde_a, noise=noise,
+                               state=state)
 
 
 # ----------------------------------------------------------------------------------

@@ -361,6 +361,71 @@ def test_candidates_are_independent():
     np.testing.assert_array_equal(m.draft(z, ctx, sched, sk, px, candidates=[2])[0], all3[2])
 
 
+# -- NEXT row: the cached state and a warm-started refine (§4.2 Stage 3, R9) -----------------
+
+def test_state_holds_each_layers_last_computed_contribution():
+    """keep_state returns, per layer, Delta_l = h_after - h_before at the layer's last
+    computed step and that step's t; checked against the trace of h after each layer."""
+    cfg, w = _tiny()
+    m = O.OracleModel(cfg, w)
+    z = synth.make_latents(cfg, 1)[0]
+    ctx = synth.make_text(cfg)
+    kv = m.encode_text(ctx)
+    sched = synth.make_schedule(4)
+    skip, proxy = synth.tiny_plan()          # layer 1 skipped at step 2, layer 0 proxied at 3
+    trace = []
+    zo, state = m.sample_one(z, kv, sched, skip, proxy, trace=trace, keep_state=True)
+    np.testing.assert_array_equal(zo, m.sample_one(z, kv, sched, skip, proxy))
+    h = {(i, l): x for i, l, x in trace}
+    z2 = m.sample_one(z, kv, sched[:3], skip[:2], proxy[:2])
+    assert sorted(state) == [0, 1]
+    assert state[0][0] == sched[2] and state[1][0] == sched[3]
+    np.testing.assert_allclose(state[0][1], h[(2, 0)] - m.patch_embed(z2), rtol=0, atol=1e-12)
+    np.testing.assert_allclose(state[1][1], h[(3, 1)] - h[(3, 0)], rtol=0, atol=1e-12)
+
+
+def test_refine_without_warm_steps_is_phi_full():
+    cfg, w = _tiny()
+    m = O.OracleModel(cfg, w)
+    z = synth.make_latents(cfg, 1)
+    ctx = synth.make_text(cfg)
+    sched = synth.make_schedule(5)
+    zd, states = m.draft(z, ctx, sched[:3], *synth.empty_plan(2, 2), keep_state=True)
+    np.testing.assert_array_equal(m.refine(zd[0], ctx, sched[2:], state=states[0], warm_steps=0),
+                                  m.refine(zd[0], ctx, sched[2:]))
+
+
+def test_warm_step_adds_the_cached_state():
+    """A warm step proxies every layer from the state: h_L = PatchEmbed(z) + sum_l Delta_l,
+    then the Euler step; the steps after it are phi_full."""
+    cfg, w = _tiny()
+    m = O.OracleModel(cfg, w)
+    z = synth.make_latents(cfg, 1)
+    ctx = synth.make_text(cfg)
+    sched = synth.make_schedule(6)
+    zd, states = m.draft(z, ctx, sched[:3], *synth.empty_plan(2, 2), keep_state=True)
+    st = states[0]
+    t0, t1 = sched[2], sched[3]
+    temb, _ = m.time_embed(t0)
+    hL = m.patch_embed(zd[0]) + st[0][1] + st[1][1]
+    v = O.unpatchify(m.head(hL, temb), cfg.latent_c, cfg.latent_h, cfg.latent_w, cfg.patch)
+    z1 = zd[0].astype(np.float64) + (float(t1) - float(t0)) * v
+    np.testing.assert_allclose(m.refine(zd[0], ctx, sched[2:], state=st, warm_steps=1),
+                               m.refine(z1, ctx, sched[3:]), rtol=0, atol=1e-12)
+
+
+def test_state_proxy_rules():
+    skip = np.zeros((2, 2), np.uint8)
+    proxy = np.full((2, 2), O.COMPUTE, np.int32)
+    proxy[0, 1] = O.STATE_SRC
+    assert O.resolve_plan(skip, proxy, state_layers=(0, 1))[(0, 1)] == ["state"]
+    with pytest.raises(ValueError):
+        O.resolve_plan(skip, proxy, state_layers=(0,))         # layer 1 not in the state
+    proxy[0, 1] = O.STATE_SRC | (1 << 16)
+    with pytest.raises(ValueError):
+        O.resolve_plan(skip, proxy, state_layers=(0, 1))       # order 1 from a single anchor
+
+
 # -- NEXT rows: classifier-free guidance and the SDE step (App. A.1) ------------------------
 
 def test_sde_step_hand_value():
