@@ -138,6 +138,18 @@ typedef struct fb_sampler_opts {
   const float* text_uncond;
   float sde_a;
   const float* noise;
+  /* §8 NEXT row 4, the cached state of Stage 3 (§4.2: "the layer activations ... for
+   * warm-starting activation proxies"), read as each layer's contribution
+   * Delta_l = B_l(h) - h from its last computed draft step (with that step's t):
+   * keep_state (fb_draft_ex): != 0 keeps every candidate's state in the model after the
+   *   call, for fb_state_offload (conditional rows under guidance);
+   * state / warm_steps (fb_refine_ex): a state buffer of one candidate (fb_state_offload
+   *   layout, host or device); the first warm_steps steps proxy every layer the state
+   *   holds from it (order 0: h <- h + Delta_l), the other layers and steps compute.
+   *   warm_steps = 0 or state = NULL is the plain refine. Not with guidance (FB_EINVAL). */
+  int keep_state;
+  const void* state;
+  int warm_steps;
 } fb_sampler_opts;
 
 /* fb_draft_ex / fb_refine_ex: fb_draft / fb_refine with sampler options (opts may be
@@ -147,6 +159,23 @@ fb_status fb_draft_ex(fb_model* m, float* latents, int n, const float* text_ctx,
                       const int32_t* proxy_plan, const fb_sampler_opts* opts);
 fb_status fb_refine_ex(fb_model* m, float* latent, const float* text_ctx,
                        const float* full_schedule, int n_steps, const fb_sampler_opts* opts);
+
+/* ---- cached-state offload (§4.2 Stage 3; §8 NEXT row 4) -----------------------------
+ * The paper moves the cached tensors to host memory during drafting and brings only the
+ * selected candidate back for refinement; the copies are part of the wall-clock.
+ * State layout of one candidate (fb_state_bytes bytes): depth fp32 values t_l (NaN: the
+ * layer was never computed, no Delta), zero padding to byte 256, then depth blocks of
+ * bf16 Delta_l [tokens][dim] (zeros where t_l is NaN).
+ * fb_state_offload copies candidate `cand`'s state of the last fb_draft_ex call with
+ * keep_state to dst (host or device) on a model-owned copy stream and returns at once;
+ * with pinned host memory the copy overlaps whatever the model runs next. A later call
+ * that writes the cached contributions waits, per cache slot, only for the copies still
+ * reading that slot. fb_state_wait blocks until every issued copy has finished and
+ * reports their errors. Errors: FB_ESTATE when the last draft did not keep its state
+ * (or a later call reused the cache), FB_EINVAL for a bad cand or NULL dst. */
+fb_status fb_state_bytes(const fb_model* m, size_t* bytes);
+fb_status fb_state_offload(fb_model* m, int cand, void* dst);
+fb_status fb_state_wait(fb_model* m);
 
 /* fb_plan_from_phi: expands phi = (S', n_skip, l_start, l_end, f_full) (§4.1,
  * "Configuration Space") into skip_mask [S'][depth] and proxy_plan [S'][depth]

@@ -170,6 +170,18 @@ struct fb_model {
   size_t anchor_elems = 0;
   int* derr = nullptr;
   int* herr = nullptr;  // pinned
+  // cached draft state (fb_draft_ex with keep_state): per layer the anchor slot of its
+  // last computed contribution (-1: none) and that step's t; rows of nr candidates per slot
+  bool state_valid = false;
+  int state_n = 0, state_nr = 0;
+  std::vector<int> state_slot;
+  std::vector<float> state_tau;
+  // offloads in flight: a copy stream, and per anchor slot the event of the last copy
+  // reading it (pending until a later write has waited for it)
+  cudaStream_t copy_st = nullptr;
+  std::vector<cudaEvent_t> slot_ev;
+  std::vector<char> slot_pending;
+  size_t pending_elems = 0;  // slot size (elements) the pending copies were issued with
   // stream-K workspace of the 2-SM GEMM: partial accumulators and per-tile counters
   // (zero between launches; reset after a device error)
   float* sk_ws = nullptr;
@@ -465,10 +477,15 @@ struct Action {
 struct Plan {
   std::vector<std::vector<Action>> steps;
   int n_slots = 0;
+  // keep: per layer the slot holding its last computed contribution (-1: none) and t
+  std::vector<int> keep_slot;
+  std::vector<float> keep_tau;
+  // warm start: per layer the slot its cached-state contribution is uploaded to (-1: none)
+  std::vector<int> warm_src;
 };
 
 fb_status analyse_plan(const fb_cfg& c, const float* sched, int S, const uint8_t* skip,
-                       const int32_t* proxy, Plan* out) {
+                       const int32_t* proxy, Plan* out, bool keep = false) {
   const int L = c.depth;
   auto is_skip = [&](int k, int l) { return skip && skip[(size_t)k * L + l] != 0; };
   auto code = [&](int k, int l) { return proxy ? proxy[(size_t)k * L + l] : -1; };
@@ -497,6 +514,10 @@ fb_status analyse_plan(const fb_cfg& c, const float* sched, int S, const uint8_t
       for (int s : an) last_use[{s, l}] = k;
       anchors[{k, l}] = an;
     }
+  // the cached state: each layer's last computed contribution stays until the end
+  if (keep)
+    for (int l = 0; l < L; ++l)
+      if (!computed[l].empty()) last_use[{computed[l].back(), l}] = S;
   // slot assignment: per layer a pool; a slot is free once its last user has run
   std::vector<std::vector<int>> free_at(L);  // per layer: for each slot, step after which it is free
   std::vector<int> slot_base(L, 0);
@@ -516,6 +537,15 @@ fb_status analyse_plan(const fb_cfg& c, const float* sched, int S, const uint8_t
   int total = 0;
   for (int l = 0; l < L; ++l) { slot_base[l] = total; total += (int)free_at[l].size(); }
   out->n_slots = total;
+  out->keep_slot.assign(keep ? L : 0, -1);
+  out->keep_tau.assign(keep ? L : 0, std::nanf(""));
+  if (keep)
+    for (int l = 0; l < L; ++l)
+      if (!computed[l].empty()) {
+        const int k = computed[l].back();
+        out->keep_slot[l] = slot_base[l] + slot_of[{k, l}];
+        out->keep_tau[l] = sched[k];
+      }
   out->steps.assign(S, {});
   for (int k = 0; k < S; ++k) {
     auto& acts = out->steps[k];
@@ -550,6 +580,27 @@ fb_status analyse_plan(const fb_cfg& c, const float* sched, int S, const uint8_t
   return FB_OK;
 }
 
+// Refine plan warm-started from a cached state: at steps < warm every layer the state
+// holds (held[l]) is an order-0 proxy of its own slot (slot_of[l], coefficient 1);
+// everything else computes. Runs of consecutive proxied layers form one proxy action.
+void warm_plan(int L, int S, int warm, const std::vector<int>& slot_of, Plan* out) {
+  out->steps.assign(S, {});
+  out->n_slots = 0;
+  out->warm_src = slot_of;
+  for (int l = 0; l < L; ++l)
+    if (slot_of[l] >= 0) out->n_slots = std::max(out->n_slots, slot_of[l] + 1);
+  for (int k = 0; k < S; ++k)
+    for (int l = 0; l < L; ++l) {
+      auto& acts = out->steps[k];
+      if (k < warm && slot_of[l] >= 0) {
+        if (acts.empty() || acts.back().type != 1) acts.push_back(Action{1, -1, -1, {}});
+        acts.back().terms.push_back({slot_of[l], 1.0});
+      } else {
+        acts.push_back(Action{0, l, -1, {}});
+      }
+    }
+}
+
 fb_status check_schedule(const float* s, int n_steps) {
   if (!s) return fail(FB_EINVAL, "schedule is NULL");
   for (int i = 0; i <= n_steps; ++i)
@@ -577,24 +628,49 @@ struct SampOpts {
 
 // The sampler loop shared by fb_draft and fb_refine (latents z on the device). With
 // guidance the batch holds 2n candidates' rows: n conditional, then n unconditional.
+// Before a write into anchor slot `slot` of slot_elems elements: the compute stream waits
+// for the offload copies still reading it. Pending copies are tracked per slot of the
+// geometry they were issued with; under another geometry every pending copy is waited for.
+fb_status wait_slot(fb_model* m, int slot, size_t slot_elems) {
+  if (slot < 0) return FB_OK;
+  for (int s = 0; s < (int)m->slot_pending.size(); ++s) {
+    if (!m->slot_pending[s] || (slot_elems == m->pending_elems && s != slot)) continue;
+    fb_stream_op_not_kernel();
+    CK(cudaStreamWaitEvent(m->st, m->slot_ev[s], 0));
+    m->slot_pending[s] = 0;
+  }
+  return FB_OK;
+}
+
+// The contribution cache holds at least `need` elements; growing it first lets every
+// copy still reading it finish.
+fb_status ensure_anchors(fb_model* m, size_t need) {
+  if (need <= m->anchor_elems) return FB_OK;
+  fb_stream_op_not_kernel();
+  CK(cudaStreamSynchronize(m->st));
+  if (m->copy_st) {
+    CK(cudaStreamSynchronize(m->copy_st));
+    std::fill(m->slot_pending.begin(), m->slot_pending.end(), 0);
+  }
+  m->state_valid = false;
+  if (m->anchors) {
+    cudaFree(m->anchors);
+    m->allocs.erase(std::find(m->allocs.begin(), m->allocs.end(), (void*)m->anchors));
+    m->anchors = nullptr;
+    m->anchor_elems = 0;
+  }
+  CKS(dalloc_t(m, &m->anchors, need));
+  m->anchor_elems = need;
+  return FB_OK;
+}
+
 fb_status sample(fb_model* m, float* z, int n, const float* sched, int S, const Plan& plan,
                  const SampOpts& so) {
   const fb_cfg& c = m->c;
   const int nr = so.guided ? 2 * n : n;  // candidates' rows in the batch
   const size_t slot_elems = (size_t)nr * m->P * c.dim;
   const size_t need = slot_elems * plan.n_slots;
-  if (need > m->anchor_elems) {
-    fb_stream_op_not_kernel();
-    CK(cudaStreamSynchronize(m->st));
-    if (m->anchors) {
-      cudaFree(m->anchors);
-      m->allocs.erase(std::find(m->allocs.begin(), m->allocs.end(), (void*)m->anchors));
-      m->anchors = nullptr;
-      m->anchor_elems = 0;
-    }
-    CKS(dalloc_t(m, &m->anchors, need));
-    m->anchor_elems = need;
-  }
+  CKS(ensure_anchors(m, need));
   const int M = nr * m->P;
   const size_t zn = (size_t)n * c.latent_c * c.latent_h * c.latent_w;
   for (int k = 0; k < S; ++k) {
@@ -609,6 +685,7 @@ fb_status sample(fb_model* m, float* z, int n, const float* sched, int S, const 
     for (const Action& a : plan.steps[k]) {
       if (a.type == 0) {
         bf16* d = a.slot >= 0 ? m->anchors + (size_t)a.slot * slot_elems : nullptr;
+        CKS(wait_slot(m, a.slot, slot_elems));
         CKS(block_forward(m, a.layer, m->hA, nr, d, so.guided ? n : 0));
       } else {
         for (size_t i0 = 0; i0 < a.terms.size(); i0 += FB_PROXY_MAX_TERMS) {
@@ -647,6 +724,9 @@ fb_status sample(fb_model* m, float* z, int n, const float* sched, int S, const 
   }
   return FB_OK;
 }
+
+// Byte offset of the contributions in a cached-state buffer (after depth fp32 t values).
+size_t state_header_bytes(const fb_cfg& c) { return ((size_t)c.depth * 4 + 255) / 256 * 256; }
 
 fb_status run_sampler(fb_model* m, float* latents, int n, const float* text_ctx,
                       const float* sched, int S, const Plan& plan,
@@ -689,6 +769,23 @@ fb_status run_sampler(fb_model* m, float* latents, int n, const float* text_ctx,
     }
   }
   CKS(begin_call(m));
+  // from here on the contribution cache is rewritten: a kept state stays valid only if
+  // this call keeps a new one
+  m->state_valid = false;
+  if (!plan.warm_src.empty()) {
+    // warm start: each held layer's contribution into its slot (Plan::warm_src)
+    CKS(ensure_anchors(m, (size_t)m->P * c.dim * plan.n_slots));
+    const size_t hb = state_header_bytes(c), pd = (size_t)m->P * c.dim;
+    for (int l = 0; l < c.depth; ++l) {
+      const int sl = plan.warm_src[l];
+      if (sl < 0) continue;
+      CKS(wait_slot(m, sl, pd));
+      fb_stream_op_not_kernel();
+      CK(cudaMemcpyAsync(m->anchors + (size_t)sl * pd,
+                         static_cast<const uint8_t*>(opts->state) + hb + (size_t)l * pd * 2,
+                         pd * 2, cudaMemcpyDefault, m->st));
+    }
+  }
   CKS(encode_text(m, text_ctx, m->kvctx));
   if (so.guided) CKS(encode_text(m, opts->text_uncond, m->kvctx_u));
   const bool dev = is_device_ptr(latents);
@@ -702,7 +799,15 @@ fb_status run_sampler(fb_model* m, float* latents, int n, const float* text_ctx,
     fb_stream_op_not_kernel();
     CK(cudaMemcpyAsync(latents, z, zn * sizeof(float), cudaMemcpyDeviceToHost, m->st));
   }
-  return end_call(m);
+  const fb_status st = end_call(m);
+  if (st == FB_OK && !plan.keep_slot.empty()) {
+    m->state_valid = true;
+    m->state_n = n;
+    m->state_nr = so.guided ? 2 * n : n;
+    m->state_slot = plan.keep_slot;
+    m->state_tau = plan.keep_tau;
+  }
+  return st;
 }
 
 }  // namespace
@@ -744,6 +849,10 @@ void fb_free(fb_model* m) {
   if (m->st) cudaStreamSynchronize(m->st);
   for (auto& p : m->pending) { cudaEventDestroy(p.a); cudaEventDestroy(p.b); }
   for (auto e : m->ev_pool) cudaEventDestroy(e);
+  if (m->copy_st) cudaStreamSynchronize(m->copy_st);
+  for (auto e : m->slot_ev)
+    if (e) cudaEventDestroy(e);
+  if (m->copy_st) cudaStreamDestroy(m->copy_st);
   for (void* p : m->allocs) cudaFree(p);
   if (m->herr) cudaFreeHost(m->herr);
   if (m->own) cudaStreamDestroy(m->own);
@@ -930,7 +1039,8 @@ fb_status fb_draft_ex(fb_model* m, float* latents, int n, const float* text_ctx,
   if (!latents || !text_ctx) return fail(FB_EINVAL, "null latents or text_ctx");
   CKS(check_schedule(schedule, n_steps));
   Plan plan;
-  CKS(analyse_plan(m->c, schedule, n_steps, skip_mask, proxy_plan, &plan));
+  CKS(analyse_plan(m->c, schedule, n_steps, skip_mask, proxy_plan, &plan,
+                   opts && opts->keep_state));
   return run_sampler(m, latents, n, text_ctx, schedule, n_steps, plan, opts);
 }
 
@@ -947,8 +1057,92 @@ fb_status fb_refine_ex(fb_model* m, float* latent, const float* text_ctx,
   if (!latent || !text_ctx) return fail(FB_EINVAL, "null latent or text_ctx");
   CKS(check_schedule(full_schedule, n_steps));
   Plan plan;
-  CKS(analyse_plan(m->c, full_schedule, n_steps, nullptr, nullptr, &plan));
+  if (opts && opts->state && opts->warm_steps > 0) {
+    // §4.2 Stage 3 warm start from a cached state: read its per-layer t (NaN: no Delta)
+    if (opts->text_uncond) return fail(FB_EINVAL, "a cached state warm-starts an unguided refine");
+    const int L = m->c.depth;
+    std::vector<float> tau(L);
+    if (is_device_ptr(opts->state)) {
+      CK(cudaMemcpy(tau.data(), opts->state, L * sizeof(float), cudaMemcpyDeviceToHost));
+    } else {
+      std::memcpy(tau.data(), opts->state, L * sizeof(float));
+    }
+    std::vector<int> slot_of(L, -1);
+    int held = 0;
+    for (int l = 0; l < L; ++l)
+      if (!std::isnan(tau[l])) slot_of[l] = held++;
+    warm_plan(L, n_steps, opts->warm_steps, slot_of, &plan);
+  } else {
+    if (opts && opts->warm_steps < 0) return fail(FB_EINVAL, "warm_steps < 0");
+    CKS(analyse_plan(m->c, full_schedule, n_steps, nullptr, nullptr, &plan));
+  }
   return run_sampler(m, latent, 1, text_ctx, full_schedule, n_steps, plan, opts);
+}
+
+fb_status fb_state_bytes(const fb_model* m, size_t* bytes) {
+  if (!m || !bytes) return fail(FB_EINVAL, "null argument");
+  *bytes = state_header_bytes(m->c) + (size_t)m->c.depth * m->P * m->c.dim * 2;
+  return FB_OK;
+}
+
+fb_status fb_state_offload(fb_model* m, int cand, void* dst) {
+  if (!m || !dst) return fail(FB_EINVAL, "null argument");
+  if (!m->state_valid) return fail(FB_ESTATE, "no cached state: draft with keep_state first");
+  if (cand < 0 || cand >= m->state_n)
+    return fail(FB_EINVAL, "candidate %d outside [0, %d)", cand, m->state_n);
+  const fb_cfg& c = m->c;
+  const int L = c.depth;
+  if (!m->copy_st) CK(cudaStreamCreateWithFlags(&m->copy_st, cudaStreamNonBlocking));
+  const int n_slots = (int)(m->anchor_elems / ((size_t)m->state_nr * m->P * c.dim));
+  if ((int)m->slot_ev.size() < n_slots) {
+    const size_t old = m->slot_ev.size();
+    m->slot_ev.resize(n_slots, nullptr);
+    m->slot_pending.resize(n_slots, 0);
+    for (size_t i = old; i < m->slot_ev.size(); ++i)
+      CK(cudaEventCreateWithFlags(&m->slot_ev[i], cudaEventDisableTiming));
+  }
+  // the copies start once the work queued so far on the model's stream is done
+  cudaEvent_t ready = nullptr;
+  CK(cudaEventCreateWithFlags(&ready, cudaEventDisableTiming));
+  fb_stream_op_not_kernel();
+  CK(cudaEventRecord(ready, m->st));
+  CK(cudaStreamWaitEvent(m->copy_st, ready, 0));
+  CK(cudaEventDestroy(ready));
+  const bool dev = is_device_ptr(dst);
+  uint8_t* d = static_cast<uint8_t*>(dst);
+  const size_t hb = state_header_bytes(c), pd = (size_t)m->P * c.dim;
+  const size_t slot_elems = (size_t)m->state_nr * pd;
+  std::vector<uint8_t> hdr(hb, 0);
+  std::memcpy(hdr.data(), m->state_tau.data(), L * sizeof(float));
+  if (dev) CK(cudaMemcpyAsync(d, hdr.data(), hb, cudaMemcpyHostToDevice, m->copy_st));
+  else std::memcpy(d, hdr.data(), hb);
+  for (int l = 0; l < L; ++l) {
+    uint8_t* out = d + hb + (size_t)l * pd * 2;
+    const int sl = m->state_slot[l];
+    if (sl < 0) {
+      if (dev) CK(cudaMemsetAsync(out, 0, pd * 2, m->copy_st));
+      else std::memset(out, 0, pd * 2);
+      continue;
+    }
+    if (m->pending_elems != slot_elems) {
+      // copies issued under another slot geometry: wait for them before mixing
+      CK(cudaStreamSynchronize(m->copy_st));
+      std::fill(m->slot_pending.begin(), m->slot_pending.end(), 0);
+      m->pending_elems = slot_elems;
+    }
+    CK(cudaMemcpyAsync(out, m->anchors + (size_t)sl * slot_elems + (size_t)cand * pd, pd * 2,
+                       cudaMemcpyDefault, m->copy_st));
+    CK(cudaEventRecord(m->slot_ev[sl], m->copy_st));
+    m->slot_pending[sl] = 1;
+  }
+  return FB_OK;
+}
+
+fb_status fb_state_wait(fb_model* m) {
+  if (!m) return fail(FB_EINVAL, "model is NULL");
+  if (m->copy_st) CK(cudaStreamSynchronize(m->copy_st));
+  std::fill(m->slot_pending.begin(), m->slot_pending.end(), 0);
+  return FB_OK;
 }
 
 fb_status fb_plan_from_phi(int S, int S_prime, int n_skip, int l_start, int l_end, int f_full,

@@ -38,7 +38,9 @@ class fb_cfg(ctypes.Structure):
 
 class fb_sampler_opts(ctypes.Structure):
     _fields_ = [("guidance", ctypes.c_float), ("text_uncond", ctypes.c_void_p),
-                ("sde_a", ctypes.c_float), ("noise", ctypes.c_void_p)]
+                ("sde_a", ctypes.c_float), ("noise", ctypes.c_void_p),
+                ("keep_state", ctypes.c_int), ("state", ctypes.c_void_p),
+                ("warm_steps", ctypes.c_int)]
 
 
 class fb_kstat(ctypes.Structure):
@@ -50,7 +52,8 @@ EXPORTS = ["fb_weights_count", "fb_weights_entry", "fb_init_model", "fb_free", "
            "fb_encode_text", "fb_draft", "fb_refine", "fb_plan_from_phi", "fb_block_forward",
            "fb_last_error", "fb_set_timing", "fb_get_stats", "fb_reset_stats", "fb_kernel_name",
            "fb_op_gemm", "fb_op_attention", "fb_draft_ex", "fb_refine_ex", "fb_select_elo",
-           "fb_set_op_repeat", "fb_gemm_streamk_noalloc"]
+           "fb_set_op_repeat", "fb_gemm_streamk_noalloc", "fb_state_bytes", "fb_state_offload",
+           "fb_state_wait"]
 
 PAIR_VERIFIER = ctypes.CFUNCTYPE(ctypes.c_int, ctypes.c_void_p, ctypes.c_int, ctypes.c_int,
                                  ctypes.POINTER(ctypes.c_int))
@@ -92,6 +95,9 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
         "fb_op_gemm": (I, [P, I, I, I, P, P, P, I, P, P, P, P, P, I]),
         "fb_op_attention": (I, [P, P, I, P, I, P, I, P, I, I, I, I, I, I, I, I]),
         "fb_gemm_streamk_noalloc": (I, [P, I, I, I, P, P, P, I, P, P, P, P, P]),
+        "fb_state_bytes": (I, [P, ctypes.POINTER(S)]),
+        "fb_state_offload": (I, [P, I, P]),
+        "fb_state_wait": (I, [P]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(L, name)
@@ -195,12 +201,31 @@ def fb_refine(model: int, latent, text_ctx, full_schedule) -> None:
                                     _ptr(sched), len(sched) - 1))
 
 
-def make_opts(guidance=1.0, text_uncond=None, sde_a=0.0, noise=None):
-    """fb_sampler_opts; keeps references to the buffers it points to."""
+def make_opts(guidance=1.0, text_uncond=None, sde_a=0.0, noise=None, keep_state=False,
+              state=None, warm_steps=0):
+    """fb_sampler_opts; keeps references to the buffers it points to. state is a cached
+    state buffer (fb_state_offload layout: numpy uint8 array or torch tensor)."""
     o = fb_sampler_opts(float(guidance), _ptr(text_uncond, np.float32), float(sde_a),
-                        _ptr(noise, np.float32))
-    o._keep = (text_uncond, noise)
+                        _ptr(noise, np.float32), int(bool(keep_state)), _ptr(state),
+                        int(warm_steps))
+    o._keep = (text_uncond, noise, state)
     return o
+
+
+def fb_state_bytes(model) -> int:
+    n = ctypes.c_size_t()
+    _check(load_library().fb_state_bytes(model, ctypes.byref(n)))
+    return n.value
+
+
+def fb_state_offload(model, cand: int, dst) -> None:
+    """Starts the copy of candidate cand's cached state into dst (fb_state_bytes bytes;
+    pinned host memory lets it overlap later work); fb_state_wait waits for it."""
+    _check(load_library().fb_state_offload(model, cand, _ptr(dst)))
+
+
+def fb_state_wait(model) -> None:
+    _check(load_library().fb_state_wait(model))
 
 
 def fb_draft_ex(model: int, latents, n: int, text_ctx, schedule, skip_mask=None,
@@ -339,6 +364,15 @@ class Model:
             fb_refine(self.handle, latent, text_ctx, schedule)
         else:
             fb_refine_ex(self.handle, latent, text_ctx, schedule, opts)
+
+    def state_bytes(self) -> int:
+        return fb_state_bytes(self.handle)
+
+    def state_offload(self, cand, dst):
+        fb_state_offload(self.handle, cand, dst)
+
+    def state_wait(self):
+        fb_state_wait(self.handle)
 
     def block_forward(self, layer, h, n, t):
         fb_block_forward(self.handle, layer, h, n, t)

@@ -381,3 +381,125 @@ def test_pipeline_draft_select_refine(small4):
     m.refine(r, ctx, sched[Sp:])
     want = ref.refine(drafts[win], ctx, sched[Sp:])
     check_latents(r.cpu().numpy(), want, drafts[win], label="refine of the selected draft")
+
+
+# ---- NEXT row 4: cached-state offload and a warm-started refine (§4.2 Stage 3) --------
+
+def _parse_state(cfg, buf):
+    """(t per layer, Delta per layer as fp32 [tokens][dim]) from a state buffer."""
+    raw = (buf.cpu() if torch.is_tensor(buf) else torch.from_numpy(buf)).numpy().view(np.uint8)
+    L, pd = cfg.depth, cfg.tokens * cfg.dim
+    hb = (4 * L + 255) // 256 * 256
+    assert raw.size == hb + L * pd * 2
+    tau = raw[:4 * L].view(np.float32).copy()
+    u16 = raw[hb:].view(np.uint16).astype(np.uint32) << 16
+    return tau, u16.view(np.float32).reshape(L, cfg.tokens, cfg.dim)
+
+
+def _state_dict(tau, delta):
+    return {l: (float(tau[l]), delta[l].astype(np.float64))
+            for l in range(len(tau)) if not np.isnan(tau[l])}
+
+
+def _check_state(cfg, buf, want, label):
+    tau, delta = _parse_state(cfg, buf)
+    for l in range(cfg.depth):
+        if l in want:
+            assert tau[l] == np.float32(want[l][0]), (label, l)
+            err = rel_max(delta[l], want[l][1])
+            assert err <= 5e-2, f"{label} layer {l}: {err:.3e}"
+        else:
+            assert np.isnan(tau[l]) and not delta[l].any(), (label, l)
+
+
+def test_state_offload_matches_oracle(small4):
+    cfg, w, m, ref = small4
+    S, n = 4, 3
+    z = synth.make_latents(cfg, n)
+    ctx = synth.make_text(cfg)
+    sched = synth.make_schedule(S)
+    skip, proxy = synth.random_plan(S, cfg.depth, 1 / 3, 0.5, seed=5, order=1)
+    zd = cuda(z)
+    m.draft(zd, ctx, sched, skip, proxy, opts=fb.make_opts(keep_state=True))
+    bufs = [torch.empty(m.state_bytes(), dtype=torch.uint8).pin_memory() for _ in range(n)]
+    for j in range(n):
+        m.state_offload(j, bufs[j])
+    m.state_wait()
+    want_z, states = ref.draft(z, ctx, sched, skip, proxy, keep_state=True)
+    for j in range(n):
+        check_latents(zd.cpu().numpy()[j], want_z[j], z[j], label=f"keep_state cand {j}")
+        _check_state(cfg, bufs[j], states[j], f"state cand {j}")
+
+
+def test_state_offload_overlapped_with_the_next_draft(small4):
+    """The copies of draft A's state run while draft B rewrites the cache; B waits for
+    them per slot, so A's offloaded state and B's latents are both intact."""
+    cfg, w, m, ref = small4
+    S = 4
+    ctx = synth.make_text(cfg)
+    sched = synth.make_schedule(S)
+    skip, proxy = synth.random_plan(S, cfg.depth, 1 / 3, 0.5, seed=9, order=0)
+    za = synth.make_latents(cfg, 2)
+    zb = synth.make_latents(cfg, 2, seed_base=555)
+    da, db = cuda(za), cuda(zb)
+    m.draft(da, ctx, sched, skip, proxy, opts=fb.make_opts(keep_state=True))
+    bufs = [torch.empty(m.state_bytes(), dtype=torch.uint8).pin_memory() for _ in range(2)]
+    for j in range(2):
+        m.state_offload(j, bufs[j])
+    m.draft(db, ctx, sched, skip, proxy, opts=fb.make_opts(keep_state=True))
+    m.state_wait()
+    _, states_a = ref.draft(za, ctx, sched, skip, proxy, keep_state=True)
+    want_b = ref.draft(zb, ctx, sched, skip, proxy)
+    for j in range(2):
+        _check_state(cfg, bufs[j], states_a[j], f"draft A state cand {j}")
+        check_latents(db.cpu().numpy()[j], want_b[j], zb[j], label=f"draft B cand {j}")
+
+
+def test_warm_started_refine_matches_oracle(small4):
+    cfg, w, m, ref = small4
+    z = synth.make_latents(cfg, 2)
+    ctx = synth.make_text(cfg)
+    sched = synth.make_schedule(5)
+    zd = cuda(z)
+    m.draft(zd, ctx, sched[:3], *synth.empty_plan(2, cfg.depth),
+            opts=fb.make_opts(keep_state=True))
+    buf = torch.empty(m.state_bytes(), dtype=torch.uint8).pin_memory()
+    m.state_offload(1, buf)
+    m.state_wait()
+    start = zd[1].cpu().numpy()
+    state = _state_dict(*_parse_state(cfg, buf))
+    assert sorted(state) == list(range(cfg.depth))
+    for warm in (1, 2):
+        r = zd[1].clone()
+        m.refine(r, ctx, sched[2:], opts=fb.make_opts(state=buf, warm_steps=warm))
+        want = ref.refine(start, ctx, sched[2:], state=state, warm_steps=warm)
+        check_latents(r.cpu().numpy(), want, start, label=f"warm refine, {warm} warm steps")
+        rd = zd[1].clone()                                   # the state from device memory
+        m.refine(rd, ctx, sched[2:], opts=fb.make_opts(state=buf.cuda(), warm_steps=warm))
+        assert torch.equal(r, rd)
+    r0, r1 = zd[1].clone(), zd[1].clone()
+    m.refine(r0, ctx, sched[2:])
+    m.refine(r1, ctx, sched[2:], opts=fb.make_opts(state=buf, warm_steps=0))
+    assert torch.equal(r0, r1)
+
+
+def test_state_errors(small4):
+    cfg, w, m, _ = small4
+    ctx = synth.make_text(cfg)
+    sched = synth.make_schedule(2)
+    z = cuda(synth.make_latents(cfg, 2))
+    buf = torch.empty(m.state_bytes(), dtype=torch.uint8)
+    m.draft(z, ctx, sched)                                   # no keep_state
+    with pytest.raises(fb.FlashBonError) as e:
+        m.state_offload(0, buf)
+    assert e.value.status == fb.FB_ESTATE
+    m.draft(z, ctx, sched, opts=fb.make_opts(keep_state=True))
+    with pytest.raises(fb.FlashBonError) as e:
+        m.state_offload(2, buf)
+    assert e.value.status == fb.FB_EINVAL
+    m.state_offload(1, buf)
+    m.state_wait()
+    with pytest.raises(fb.FlashBonError) as e:               # no warm start under guidance
+        m.refine(z[0].clone(), ctx, sched,
+                 opts=fb.make_opts(2.0, ctx, state=buf, warm_steps=1))
+    assert e.value.status == fb.FB_EINVAL
