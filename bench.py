@@ -51,6 +51,9 @@ VARIANTS = {
     "base": "",
     "cfg": "; classifier-free guidance w=5 (16 candidates, 32 rows with the unconditional pass)",
     "sde": "; Euler-Maruyama SDE steps, a=0.7, caller-supplied N(0,1) draws",
+    "offload": "; every candidate's cached state (each layer's last contribution, bf16, "
+               "144 MB per candidate) copied to pinned host memory behind the refine and "
+               "the next draft",
 }
 
 
@@ -274,18 +277,30 @@ def run_gb300(args):
         nd = torch.from_numpy(synth.make_noise(cfg, S_DRAFT, NC, seed=2000 + rank)).cuda()
         nr = torch.from_numpy(synth.make_noise(cfg, S_TOTAL - S_DRAFT, 1, seed=3000 + rank)).cuda()
         opts_d, opts_r = fb.make_opts(sde_a=0.7, noise=nd), fb.make_opts(sde_a=0.7, noise=nr)
+    states = []
+    if args.variant == "offload":
+        states = [torch.empty(model.state_bytes(), dtype=torch.uint8).pin_memory()
+                  for _ in range(NC)]
+        opts_d = fb.make_opts(keep_state=True)
     setup_s = time.time() - t_setup
 
     def dev_step():
         with torch.cuda.stream(stream):
             z.copy_(z0)
         model.draft(z, ctx, draft_sched, skip, proxy, opts=opts_d)
+        if states:   # every candidate's state to pinned host memory, behind the refine
+            model.state_offload(0, states)
         with torch.cuda.stream(stream):
             zr.copy_(z[0])
         model.refine(zr, ctx, tail, opts=opts_r)
 
+    def finish():  # the last step's offload copies belong to the timed region
+        if states:
+            model.state_wait()
+
     for _ in range(args.warmup):
         dev_step()
+    finish()
     torch.cuda.synchronize()
     model.reset_stats()
     if pg:
@@ -297,6 +312,7 @@ def run_gb300(args):
         ev0.record(stream)
         for _ in range(args.steps):
             dev_step()
+        finish()
         ev1.record(stream)
         torch.cuda.synchronize()
     ms = ev0.elapsed_time(ev1)
@@ -307,9 +323,11 @@ def run_gb300(args):
     model.reset_stats()
     model.set_timing(1 << fb.K["gemm_tc"])
     e2, e3 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    finish()
     e2.record(stream)
     for _ in range(args.steps):
         dev_step()
+    finish()
     e3.record(stream)
     torch.cuda.synchronize()
     stats = model.stats()
@@ -333,16 +351,20 @@ def run_gb300(args):
     def host_step():
         zh.copy_(z0h)
         model.draft(zh, ctxh, draft_sched, skip, proxy, opts=opts_d)
+        if states:
+            model.state_offload(0, states)
         zrh.copy_(zh[0])
         model.refine(zrh, ctxh, tail, opts=opts_r)
 
     host_step()
+    finish()
     torch.cuda.synchronize()
     if pg:
         pg.barrier()
     t0 = time.perf_counter()
     for _ in range(args.steps):
         host_step()
+    finish()
     e2e_s = (time.perf_counter() - t0) / args.steps
     if pg:
         t = torch.tensor([e2e_s], device="cuda")
@@ -350,7 +372,7 @@ def run_gb300(args):
         e2e_s = float(t.item())
     zbytes = z0.numel() * 4
     h2d = zbytes + 2 * ctx_h.nbytes + zbytes // NC
-    d2h = zbytes + zbytes // NC
+    d2h = zbytes + zbytes // NC + sum(b.numel() for b in states)
 
     peaks, peak_kind = read_peaks()
     g = stats["gemm_tc"]

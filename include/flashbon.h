@@ -166,15 +166,17 @@ fb_status fb_refine_ex(fb_model* m, float* latent, const float* text_ctx,
  * State layout of one candidate (fb_state_bytes bytes): depth fp32 values t_l (NaN: the
  * layer was never computed, no Delta), zero padding to byte 256, then depth blocks of
  * bf16 Delta_l [tokens][dim] (zeros where t_l is NaN).
- * fb_state_offload copies candidate `cand`'s state of the last fb_draft_ex call with
- * keep_state to dst (host or device) on a model-owned copy stream and returns at once;
- * with pinned host memory the copy overlaps whatever the model runs next. A later call
- * that writes the cached contributions waits, per cache slot, only for the copies still
- * reading that slot. fb_state_wait blocks until every issued copy has finished and
- * reports their errors. Errors: FB_ESTATE when the last draft did not keep its state
- * (or a later call reused the cache), FB_EINVAL for a bad cand or NULL dst. */
+ * fb_state_offload copies the states of candidates first .. first + count - 1 of the last
+ * fb_draft_ex call with keep_state to dst[0] .. dst[count - 1] (host or device, each
+ * fb_state_bytes bytes) on a model-owned copy stream and returns at once; with pinned
+ * host memory the copies overlap whatever the model runs next. They are issued layer by
+ * layer (every candidate's layer 0, then layer 1, ...): a later call that rewrites the
+ * cached contributions waits, per cache slot, only for the copies still reading it.
+ * A buffer is complete only after fb_state_wait, which blocks until every issued copy
+ * has finished. Errors: FB_ESTATE when the last draft did not keep its state (or a later
+ * call reused the cache), FB_EINVAL for a bad range or a NULL pointer. */
 fb_status fb_state_bytes(const fb_model* m, size_t* bytes);
-fb_status fb_state_offload(fb_model* m, int cand, void* dst);
+fb_status fb_state_offload(fb_model* m, int first, int count, void* const* dst);
 fb_status fb_state_wait(fb_model* m);
 
 /* fb_plan_from_phi: expands phi = (S', n_skip, l_start, l_end, f_full) (§4.1,

@@ -46,7 +46,7 @@ Readings where the paper is silent or ambiguous (all arithmetic in fp64):
   R8 Elo selection (§4.2 Stage 2): base K and the expected-score formula are not given;
      K = 32 and the logistic 400-point expected score are used; the adjacent comparisons
      are passes over the rating-sorted survivors; ties go to the lower index.
-  R9 cached state (§4.2 Stage 3): the optional layer activations kept for warm-starting
+  R12 cached state (§4.2 Stage 3): the optional layer activations kept for warm-starting
      activation proxies are, under R1, each layer's contribution Delta_l from its last
      computed draft step, with that step's t. A refine step may proxy layer l from it
      (order 0: h <- h + Delta_l); with no such steps the refine is phi_full exactly.
@@ -57,7 +57,7 @@ import numpy as np
 
 F64 = np.float64
 COMPUTE = -1
-STATE_SRC = 0xFFFF  # proxy source: the cached state of an earlier call (R9), order 0
+STATE_SRC = 0xFFFF  # proxy source: the cached state of an earlier call (R12), order 0
 
 
 # ----------------------------------------------------------------------------------
@@ -216,7 +216,7 @@ def plan_from_phi(S, S_prime, n_skip, l_start, l_end, f_full, order, depth):
 
 def resolve_plan(skip, proxy, state_layers=()):
     """Validate a plan and list, per proxied (step, layer), its anchor steps (most recent
-    first); a proxy from the cached state (source STATE_SRC, R9) has the anchor "state".
+    first); a proxy from the cached state (source STATE_SRC, R12) has the anchor "state".
     Raises ValueError on: skip and proxy both set; source step not earlier than the step;
     layer not computed at the source step; order outside 0..2; a state proxy of order > 0
     or of a layer the state does not hold."""
@@ -371,7 +371,7 @@ class OracleModel:
         Euler-Maruyama update with the standard normal draws noise[i] (R7).
 
         keep_state: also return the cached state, {layer: (t, Delta_l)} of each layer's
-        last computed step (R9; the conditional pass). state: such a dict, the source of
+        last computed step (R12; the conditional pass). state: such a dict, the source of
         proxies coded STATE_SRC (single pass only)."""
         cfg = self.cfg
         sched = np.asarray(schedule, F64)
@@ -410,7 +410,7 @@ class OracleModel:
         """Stage 1 (Eq. 8): each candidate's z_T through the truncated, accelerated
         schedule. Candidates are independent; `candidates` picks a subset. noise, when
         sde_a > 0, is [n_steps][N][C][H][W] (indexed by the candidate's position in z_T).
-        keep_state: also return each candidate's cached state (R9), a list of dicts."""
+        keep_state: also return each candidate's cached state (R12), a list of dicts."""
         z_T = np.asarray(z_T)
         idx = range(z_T.shape[0]) if candidates is None else candidates
         kv = self.encode_text(ctx)
@@ -430,7 +430,7 @@ class OracleModel:
     def refine(self, z, ctx, schedule, ctx_uncond=None, guidance=1.0, sde_a=0.0, noise=None,
                state=None, warm_steps=0):
         """Stage 3: resume from a cached latent with phi_full (no skip, no proxy).
-        noise, when sde_a > 0, is [n_steps][C][H][W]. With a cached state (R9) the first
+        noise, when sde_a > 0, is [n_steps][C][H][W]. With a cached state (R12) the first
         warm_steps steps proxy every layer the state holds from it (order 0)."""
         n = len(schedule) - 1
         skip = np.zeros((n, self.cfg.depth), np.uint8)

@@ -629,12 +629,14 @@ struct SampOpts {
 // The sampler loop shared by fb_draft and fb_refine (latents z on the device). With
 // guidance the batch holds 2n candidates' rows: n conditional, then n unconditional.
 // Before a write into anchor slot `slot` of slot_elems elements: the compute stream waits
-// for the offload copies still reading it. Pending copies are tracked per slot of the
-// geometry they were issued with; under another geometry every pending copy is waited for.
+// for the offload copies still reading any part of it. Pending copies are tracked per
+// slot of the geometry (pending_elems) they were issued with.
 fb_status wait_slot(fb_model* m, int slot, size_t slot_elems) {
   if (slot < 0) return FB_OK;
+  const size_t b = (size_t)slot * slot_elems, e = b + slot_elems;
   for (int s = 0; s < (int)m->slot_pending.size(); ++s) {
-    if (!m->slot_pending[s] || (slot_elems == m->pending_elems && s != slot)) continue;
+    const size_t sb = (size_t)s * m->pending_elems, se = sb + m->pending_elems;
+    if (!m->slot_pending[s] || se <= b || e <= sb) continue;
     fb_stream_op_not_kernel();
     CK(cudaStreamWaitEvent(m->st, m->slot_ev[s], 0));
     m->slot_pending[s] = 0;
@@ -1085,21 +1087,32 @@ fb_status fb_state_bytes(const fb_model* m, size_t* bytes) {
   return FB_OK;
 }
 
-fb_status fb_state_offload(fb_model* m, int cand, void* dst) {
+fb_status fb_state_offload(fb_model* m, int first, int count, void* const* dst) {
   if (!m || !dst) return fail(FB_EINVAL, "null argument");
   if (!m->state_valid) return fail(FB_ESTATE, "no cached state: draft with keep_state first");
-  if (cand < 0 || cand >= m->state_n)
-    return fail(FB_EINVAL, "candidate %d outside [0, %d)", cand, m->state_n);
+  if (first < 0 || count < 1 || first + count > m->state_n)
+    return fail(FB_EINVAL, "candidates [%d, %d) outside [0, %d)", first, first + count,
+                m->state_n);
+  for (int j = 0; j < count; ++j)
+    if (!dst[j]) return fail(FB_EINVAL, "dst[%d] is NULL", j);
   const fb_cfg& c = m->c;
   const int L = c.depth;
   if (!m->copy_st) CK(cudaStreamCreateWithFlags(&m->copy_st, cudaStreamNonBlocking));
-  const int n_slots = (int)(m->anchor_elems / ((size_t)m->state_nr * m->P * c.dim));
+  const size_t hb = state_header_bytes(c), pd = (size_t)m->P * c.dim;
+  const size_t slot_elems = (size_t)m->state_nr * pd;
+  const int n_slots = (int)(m->anchor_elems / slot_elems);
   if ((int)m->slot_ev.size() < n_slots) {
     const size_t old = m->slot_ev.size();
     m->slot_ev.resize(n_slots, nullptr);
     m->slot_pending.resize(n_slots, 0);
     for (size_t i = old; i < m->slot_ev.size(); ++i)
       CK(cudaEventCreateWithFlags(&m->slot_ev[i], cudaEventDisableTiming));
+  }
+  if (m->pending_elems != slot_elems) {
+    // copies issued under another slot geometry: let them finish before mixing
+    CK(cudaStreamSynchronize(m->copy_st));
+    std::fill(m->slot_pending.begin(), m->slot_pending.end(), 0);
+    m->pending_elems = slot_elems;
   }
   // the copies start once the work queued so far on the model's stream is done
   cudaEvent_t ready = nullptr;
@@ -1108,32 +1121,30 @@ fb_status fb_state_offload(fb_model* m, int cand, void* dst) {
   CK(cudaEventRecord(ready, m->st));
   CK(cudaStreamWaitEvent(m->copy_st, ready, 0));
   CK(cudaEventDestroy(ready));
-  const bool dev = is_device_ptr(dst);
-  uint8_t* d = static_cast<uint8_t*>(dst);
-  const size_t hb = state_header_bytes(c), pd = (size_t)m->P * c.dim;
-  const size_t slot_elems = (size_t)m->state_nr * pd;
   std::vector<uint8_t> hdr(hb, 0);
   std::memcpy(hdr.data(), m->state_tau.data(), L * sizeof(float));
-  if (dev) CK(cudaMemcpyAsync(d, hdr.data(), hb, cudaMemcpyHostToDevice, m->copy_st));
-  else std::memcpy(d, hdr.data(), hb);
+  std::vector<char> dev(count);
+  for (int j = 0; j < count; ++j) {
+    dev[j] = is_device_ptr(dst[j]);
+    if (dev[j]) CK(cudaMemcpyAsync(dst[j], hdr.data(), hb, cudaMemcpyHostToDevice, m->copy_st));
+    else std::memcpy(dst[j], hdr.data(), hb);
+  }
   for (int l = 0; l < L; ++l) {
-    uint8_t* out = d + hb + (size_t)l * pd * 2;
     const int sl = m->state_slot[l];
-    if (sl < 0) {
-      if (dev) CK(cudaMemsetAsync(out, 0, pd * 2, m->copy_st));
-      else std::memset(out, 0, pd * 2);
-      continue;
+    for (int j = 0; j < count; ++j) {
+      uint8_t* out = static_cast<uint8_t*>(dst[j]) + hb + (size_t)l * pd * 2;
+      if (sl < 0) {
+        if (dev[j]) CK(cudaMemsetAsync(out, 0, pd * 2, m->copy_st));
+        else std::memset(out, 0, pd * 2);
+        continue;
+      }
+      CK(cudaMemcpyAsync(out, m->anchors + (size_t)sl * slot_elems + (size_t)(first + j) * pd,
+                         pd * 2, cudaMemcpyDefault, m->copy_st));
     }
-    if (m->pending_elems != slot_elems) {
-      // copies issued under another slot geometry: wait for them before mixing
-      CK(cudaStreamSynchronize(m->copy_st));
-      std::fill(m->slot_pending.begin(), m->slot_pending.end(), 0);
-      m->pending_elems = slot_elems;
+    if (sl >= 0) {
+      CK(cudaEventRecord(m->slot_ev[sl], m->copy_st));
+      m->slot_pending[sl] = 1;
     }
-    CK(cudaMemcpyAsync(out, m->anchors + (size_t)sl * slot_elems + (size_t)cand * pd, pd * 2,
-                       cudaMemcpyDefault, m->copy_st));
-    CK(cudaEventRecord(m->slot_ev[sl], m->copy_st));
-    m->slot_pending[sl] = 1;
   }
   return FB_OK;
 }

@@ -96,7 +96,7 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
         "fb_op_attention": (I, [P, P, I, P, I, P, I, P, I, I, I, I, I, I, I, I]),
         "fb_gemm_streamk_noalloc": (I, [P, I, I, I, P, P, P, I, P, P, P, P, P]),
         "fb_state_bytes": (I, [P, ctypes.POINTER(S)]),
-        "fb_state_offload": (I, [P, I, P]),
+        "fb_state_offload": (I, [P, I, I, ctypes.POINTER(P)]),
         "fb_state_wait": (I, [P]),
     }
     for name, (res, args) in sig.items():
@@ -218,10 +218,12 @@ def fb_state_bytes(model) -> int:
     return n.value
 
 
-def fb_state_offload(model, cand: int, dst) -> None:
-    """Starts the copy of candidate cand's cached state into dst (fb_state_bytes bytes;
-    pinned host memory lets it overlap later work); fb_state_wait waits for it."""
-    _check(load_library().fb_state_offload(model, cand, _ptr(dst)))
+def fb_state_offload(model, first: int, dsts) -> None:
+    """Starts the copies of candidates first .. first + len(dsts) - 1's cached states into
+    dsts (fb_state_bytes bytes each; pinned host memory lets them overlap later work);
+    fb_state_wait waits for them."""
+    arr = (ctypes.c_void_p * len(dsts))(*[_ptr(d) for d in dsts])
+    _check(load_library().fb_state_offload(model, first, len(dsts), arr))
 
 
 def fb_state_wait(model) -> None:
@@ -368,8 +370,8 @@ class Model:
     def state_bytes(self) -> int:
         return fb_state_bytes(self.handle)
 
-    def state_offload(self, cand, dst):
-        fb_state_offload(self.handle, cand, dst)
+    def state_offload(self, first, dsts):
+        fb_state_offload(self.handle, first, dsts)
 
     def state_wait(self):
         fb_state_wait(self.handle)

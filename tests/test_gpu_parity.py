@@ -422,8 +422,8 @@ def test_state_offload_matches_oracle(small4):
     zd = cuda(z)
     m.draft(zd, ctx, sched, skip, proxy, opts=fb.make_opts(keep_state=True))
     bufs = [torch.empty(m.state_bytes(), dtype=torch.uint8).pin_memory() for _ in range(n)]
-    for j in range(n):
-        m.state_offload(j, bufs[j])
+    m.state_offload(0, bufs[:1])
+    m.state_offload(1, bufs[1:])
     m.state_wait()
     want_z, states = ref.draft(z, ctx, sched, skip, proxy, keep_state=True)
     for j in range(n):
@@ -444,8 +444,7 @@ def test_state_offload_overlapped_with_the_next_draft(small4):
     da, db = cuda(za), cuda(zb)
     m.draft(da, ctx, sched, skip, proxy, opts=fb.make_opts(keep_state=True))
     bufs = [torch.empty(m.state_bytes(), dtype=torch.uint8).pin_memory() for _ in range(2)]
-    for j in range(2):
-        m.state_offload(j, bufs[j])
+    m.state_offload(0, bufs)
     m.draft(db, ctx, sched, skip, proxy, opts=fb.make_opts(keep_state=True))
     m.state_wait()
     _, states_a = ref.draft(za, ctx, sched, skip, proxy, keep_state=True)
@@ -464,7 +463,7 @@ def test_warm_started_refine_matches_oracle(small4):
     m.draft(zd, ctx, sched[:3], *synth.empty_plan(2, cfg.depth),
             opts=fb.make_opts(keep_state=True))
     buf = torch.empty(m.state_bytes(), dtype=torch.uint8).pin_memory()
-    m.state_offload(1, buf)
+    m.state_offload(1, [buf])
     m.state_wait()
     start = zd[1].cpu().numpy()
     state = _state_dict(*_parse_state(cfg, buf))
@@ -491,13 +490,13 @@ def test_state_errors(small4):
     buf = torch.empty(m.state_bytes(), dtype=torch.uint8)
     m.draft(z, ctx, sched)                                   # no keep_state
     with pytest.raises(fb.FlashBonError) as e:
-        m.state_offload(0, buf)
+        m.state_offload(0, [buf])
     assert e.value.status == fb.FB_ESTATE
     m.draft(z, ctx, sched, opts=fb.make_opts(keep_state=True))
     with pytest.raises(fb.FlashBonError) as e:
-        m.state_offload(2, buf)
+        m.state_offload(1, [buf, buf])                      # candidates 1..2 of 2
     assert e.value.status == fb.FB_EINVAL
-    m.state_offload(1, buf)
+    m.state_offload(1, [buf])
     m.state_wait()
     with pytest.raises(fb.FlashBonError) as e:               # no warm start under guidance
         m.refine(z[0].clone(), ctx, sched,

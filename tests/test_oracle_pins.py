@@ -361,7 +361,7 @@ def test_candidates_are_independent():
     np.testing.assert_array_equal(m.draft(z, ctx, sched, sk, px, candidates=[2])[0], all3[2])
 
 
-# -- NEXT row: the cached state and a warm-started refine (§4.2 Stage 3, R9) -----------------
+# -- NEXT row: the cached state and a warm-started refine (§4.2 Stage 3, R12) -----------------
 
 def test_state_holds_each_layers_last_computed_contribution():
     """keep_state returns, per layer, Delta_l = h_after - h_before at the layer's last
