@@ -342,7 +342,7 @@ class OracleModel:
                 last=None):
         """Blocks of step i on h: skip (Eq. 6), compute (Eq. 7, caching Delta_l when a
         later proxy needs it; with `last`, also recording each layer's latest (t, Delta_l),
-        R9) or proxy (Eqs. 3-5)."""
+        R12) or proxy (Eqs. 3-5)."""
         for l in range(self.cfg.depth):
             if skip[i][l]:
                 continue
