@@ -62,6 +62,28 @@ __device__ __forceinline__ uint64_t desc_mn_sw128(uint32_t saddr, uint32_t lbo) 
   return d;
 }
 
+// three-input maximum (one instruction on sm_100 and later)
+__device__ __forceinline__ float fmax3(float a, float b, float c) {
+  float r;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(r) : "f"(a), "f"(b), "f"(c));
+  return r;
+}
+// maximum of a 128-score row: eight independent chains of three-input maxima, so the
+// reduction is a few dependent steps instead of 128
+__device__ __forceinline__ float rowmax128(const float* s) {
+  float m[8];
+#pragma unroll
+  for (int k = 0; k < 8; ++k) m[k] = fmax3(s[k], s[k + 8], s[k + 16]);
+#pragma unroll
+  for (int i = 24; i + 16 <= 120; i += 16) {
+#pragma unroll
+    for (int k = 0; k < 8; ++k) m[k] = fmax3(m[k], s[i + k], s[i + 8 + k]);
+  }
+#pragma unroll
+  for (int k = 0; k < 8; ++k) m[k] = fmaxf(m[k], s[120 + k]);
+  return fmaxf(fmax3(m[0], m[1], m[2]), fmax3(fmax3(m[3], m[4], m[5]), m[6], m[7]));
+}
+
 __device__ __forceinline__ float ex2(float x) {
   float y;
   asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
@@ -243,10 +265,7 @@ __global__ void __launch_bounds__(THREADS, 1)
         for (int i = 0; i < 128; ++i)
           if (i >= valid) s[i] = -INFINITY;
       }
-      float mx = -INFINITY;
-#pragma unroll
-      for (int i = 0; i < 128; ++i) mx = fmaxf(mx, s[i]);
-      mx *= p.scale_log2;
+      const float mx = rowmax128(s) * p.scale_log2;
       if (j > 0) {
         // PV_{j-1} must be done before P is overwritten and before O is touched
         const bool ok2 = mbar_wait(o_done, (j - 1) & 1, err);
@@ -272,14 +291,14 @@ __global__ void __launch_bounds__(THREADS, 1)
         }
         tmem_st_wait();
       }
-      float lsum = 0.f;
+      float ls[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};  // independent partial sums
 #pragma unroll
       for (int ch = 0; ch < 16; ++ch) {  // 16-byte chunks of 8 keys
         float e[8];
 #pragma unroll
         for (int q = 0; q < 8; ++q) {
           e[q] = ex2(fmaf(s[ch * 8 + q], p.scale_log2, -m_used));
-          lsum += e[q];
+          ls[q] += e[q];
         }
         uint4 v;
         v.x = pack_bf16x2(e[0], e[1]);
@@ -289,7 +308,7 @@ __global__ void __launch_bounds__(THREADS, 1)
         const int sub = ch >> 3, c16 = (ch & 7) ^ (r & 7);
         *reinterpret_cast<uint4*>(prow + sub * SUB + c16 * 16) = v;
       }
-      l += lsum;
+      l += ((ls[0] + ls[1]) + (ls[2] + ls[3])) + ((ls[4] + ls[5]) + (ls[6] + ls[7]));
       fence_async_smem();  // P visible to the tensor core (async proxy)
       tc_fence_before();
       __syncwarp();
@@ -524,10 +543,7 @@ __global__ void __launch_bounds__(THREADS2, 1)
         for (int i = 0; i < 128; ++i)
           if (i >= valid) s[i] = -INFINITY;
       }
-      float mx = -INFINITY;
-#pragma unroll
-      for (int i = 0; i < 128; ++i) mx = fmaxf(mx, s[i]);
-      mx *= p.scale_log2;
+      const float mx = rowmax128(s) * p.scale_log2;
       if (j == 0) {
         m_used = mx;
       } else if (__any_sync(0xffffffffu, mx > m_used + 8.f)) {
@@ -546,7 +562,7 @@ __global__ void __launch_bounds__(THREADS2, 1)
           tmem_st32(lane_base + o_col + c * 32, u);
         }
       }
-      float lsum = 0.f;
+      float ls[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};  // independent partial sums
 #pragma unroll
       for (int c = 0; c < 2; ++c) {
         uint32_t u[32];
@@ -554,12 +570,13 @@ __global__ void __launch_bounds__(THREADS2, 1)
         for (int i = 0; i < 32; ++i) {
           const float e0 = ex2(fmaf(s[c * 64 + 2 * i], p.scale_log2, -m_used));
           const float e1 = ex2(fmaf(s[c * 64 + 2 * i + 1], p.scale_log2, -m_used));
-          lsum += e0 + e1;
+          ls[(2 * i) & 7] += e0;
+          ls[(2 * i + 1) & 7] += e1;
           u[i] = pack_bf16x2(e0, e1);
         }
         tmem_st32(lane_base + s_col + c * 32, u);
       }
-      l += lsum;
+      l += ((ls[0] + ls[1]) + (ls[2] + ls[3])) + ((ls[4] + ls[5]) + (ls[6] + ls[7]));
       tmem_st_wait();
       tc_fence_before();
       __syncwarp();
