@@ -383,7 +383,7 @@ cudaError_t qk_norm_rope(bf16* x, int rows, int ld, int D, int nseg, int col0, c
     case 256: return QKN(64, 1);
     case 512: return QKN(128, 1);
     case 1024: return QKN(128, 2);
-    case 1536: return QKN(128, 3);
+    case 1536: return QKN(32, 12);  // one warp per row: 96 bytes in flight per thread
     case 2048: return QKN(128, 4);
     case 3072: return QKN(256, 3);
     case 4096: return QKN(256, 4);
