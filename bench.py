@@ -284,15 +284,19 @@ def run_gb300(args):
         opts_d = fb.make_opts(keep_state=True)
     setup_s = time.time() - t_setup
 
-    def dev_step():
+    def dev_step(after=None):
         with torch.cuda.stream(stream):
             z.copy_(z0)
         model.draft(z, ctx, draft_sched, skip, proxy, opts=opts_d)
+        if after:
+            after("draft")
         if states:   # every candidate's state to pinned host memory, behind the refine
             model.state_offload(0, states)
         with torch.cuda.stream(stream):
             zr.copy_(z[0])
         model.refine(zr, ctx, tail, opts=opts_r)
+        if after:
+            after("refine")
 
     def finish():  # the last step's offload copies belong to the timed region
         if states:
@@ -324,9 +328,19 @@ def run_gb300(args):
     model.set_timing(1 << fb.K["gemm_tc"])
     e2, e3 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     finish()
+    # the GEMM statistics of the draft and of the refine separately (each call collects
+    # its launches' event times before it returns)
+    by_phase = {ph: {"launches": 0, "ms": 0.0, "flops": 0.0} for ph in ("draft", "refine")}
+    last = [model.stats()["gemm_tc"]]
+
+    def after(ph):
+        cur = model.stats()["gemm_tc"]
+        for k in by_phase[ph]:
+            by_phase[ph][k] += cur[k] - last[0][k]
+        last[0] = cur
     e2.record(stream)
     for _ in range(args.steps):
-        dev_step()
+        dev_step(after)
     finish()
     e3.record(stream)
     torch.cuda.synchronize()
@@ -399,7 +413,13 @@ def run_gb300(args):
                         "launches": g["launches"], "ms": g["ms"] / args.steps,
                         "measured_in": "timed pass 2 (same steps, per-launch CUDA events on "
                                        "the library stream)",
-                        "pass2_ms_per_step": ms_instrumented / args.steps},
+                        "pass2_ms_per_step": ms_instrumented / args.steps,
+                        "by_phase": {ph: {"launches": v["launches"],
+                                          "achieved": (v["flops"] / (v["ms"] / 1e3) / 1e12
+                                                       if v["ms"] > 0 else None),
+                                          "frac": (v["flops"] / (v["ms"] / 1e3) / 1e12 / peak
+                                                   if v["ms"] > 0 else None)}
+                                     for ph, v in by_phase.items()}},
            "step_tflops": algo_flops / (ms_step / 1e3) / 1e12,
            "step_frac_of_peak": algo_flops / (ms_step / 1e3) / 1e12 / peak,
            "e2e": {"value": ws * NC / e2e_s, "unit": "candidates/s",
