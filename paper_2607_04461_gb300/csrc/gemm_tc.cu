@@ -501,6 +501,18 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
         tma_load_2d(wtiles + b * CC::TILE_BYTES, &tmR, &rload[2 * we + b],
                     n0 + (half * 4 + cc) * 32, row0);
       };
+      // bias and gate of this warp's four chunks, one column per lane, requested before
+      // the accumulator is ready (the chunks broadcast them with shuffles)
+      const int ecol = n0 + half * 128 + lane;
+      const float eb0 = epi.bias ? __ldg(epi.bias + ecol) : 0.f;
+      const float eb1 = epi.bias ? __ldg(epi.bias + ecol + 32) : 0.f;
+      const float eb2 = epi.bias ? __ldg(epi.bias + ecol + 64) : 0.f;
+      const float eb3 = epi.bias ? __ldg(epi.bias + ecol + 96) : 0.f;
+      const bool has_gate = KIND == EPI_RESID && epi.gate;
+      const float eg0 = has_gate ? __ldg(epi.gate + ecol) : 1.f;
+      const float eg1 = has_gate ? __ldg(epi.gate + ecol + 32) : 1.f;
+      const float eg2 = has_gate ? __ldg(epi.gate + ecol + 64) : 1.f;
+      const float eg3 = has_gate ? __ldg(epi.gate + ecol + 96) : 1.f;
       // whole tiles: the first two residual chunks load while the mainloop runs
       const bool early = KIND == EPI_RESID && whole && row0 < M;
       if (early) {
@@ -606,25 +618,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
           }
           const int b = cc & 1;
           uint8_t* tile_b = wtiles + b * CC::TILE_BYTES;
-          float bv[32];
-#pragma unroll
-          for (int j = 0; j < 32; j += 8) {
-            if (epi.bias) load_f32x8(epi.bias + col0 + j, bv + j);
-            else {
-#pragma unroll
-              for (int q = 0; q < 8; ++q) bv[j + q] = 0.f;
-            }
-          }
+          // this chunk's bias / gate (lane j holds column j; see eb / eg)
+          const float bl = cc == 0 ? eb0 : cc == 1 ? eb1 : cc == 2 ? eb2 : eb3;
+          const float gl = cc == 0 ? eg0 : cc == 1 ? eg1 : cc == 2 ? eg2 : eg3;
           if (KIND == EPI_RESID) {
-            float gv[32];
-#pragma unroll
-            for (int j = 0; j < 32; j += 8) {
-              if (epi.gate) load_f32x8(epi.gate + col0 + j, gv + j);
-              else {
-#pragma unroll
-                for (int q = 0; q < 8; ++q) gv[j + q] = 1.f;
-              }
-            }
             const bool lok = mbar_wait(&rload[2 * we + b], (rl_phase >> b) & 1u, err);
             rl_phase ^= 1u << b;
             if (!__all_sync(0xffffffffu, lok)) { failed = true; break; }
@@ -632,10 +629,16 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
             for (int j4 = 0; j4 < 8; ++j4) {
               float4* p4 = reinterpret_cast<float4*>(tile_b + swz128(lane, j4));
               float4 o = *p4;
-              o.x += gv[4 * j4] * (v[4 * j4] + bv[4 * j4]);
-              o.y += gv[4 * j4 + 1] * (v[4 * j4 + 1] + bv[4 * j4 + 1]);
-              o.z += gv[4 * j4 + 2] * (v[4 * j4 + 2] + bv[4 * j4 + 2]);
-              o.w += gv[4 * j4 + 3] * (v[4 * j4 + 3] + bv[4 * j4 + 3]);
+              float bb[4], gg[4];
+#pragma unroll
+              for (int q = 0; q < 4; ++q) {
+                bb[q] = __shfl_sync(0xffffffffu, bl, 4 * j4 + q);
+                gg[q] = __shfl_sync(0xffffffffu, gl, 4 * j4 + q);
+              }
+              o.x += gg[0] * (v[4 * j4] + bb[0]);
+              o.y += gg[1] * (v[4 * j4 + 1] + bb[1]);
+              o.z += gg[2] * (v[4 * j4 + 2] + bb[2]);
+              o.w += gg[3] * (v[4 * j4 + 3] + bb[3]);
               *p4 = o;
             }
           } else {
@@ -648,7 +651,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
               float y[8];
 #pragma unroll
               for (int i = 0; i < 8; ++i) {
-                y[i] = v[8 * q + i] + bv[8 * q + i];
+                y[i] = v[8 * q + i] + __shfl_sync(0xffffffffu, bl, 8 * q + i);
                 if (KIND == EPI_GELU_BF16) y[i] = gelu_tanh_f(y[i]);
               }
               *reinterpret_cast<uint4*>(tile_b + swz64(lane, q)) =
