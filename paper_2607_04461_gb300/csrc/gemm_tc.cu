@@ -625,22 +625,28 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
             const bool lok = mbar_wait(&rload[2 * we + b], (rl_phase >> b) & 1u, err);
             rl_phase ^= 1u << b;
             if (!__all_sync(0xffffffffu, lok)) { failed = true; break; }
+            // all eight residual loads first: a load after a store to the same tile
+            // would otherwise wait for it
+            float4 rr[8];
+#pragma unroll
+            for (int j4 = 0; j4 < 8; ++j4)
+              rr[j4] = *reinterpret_cast<const float4*>(tile_b + swz128(lane, j4));
 #pragma unroll
             for (int j4 = 0; j4 < 8; ++j4) {
-              float4* p4 = reinterpret_cast<float4*>(tile_b + swz128(lane, j4));
-              float4 o = *p4;
               float bb[4], gg[4];
 #pragma unroll
               for (int q = 0; q < 4; ++q) {
                 bb[q] = __shfl_sync(0xffffffffu, bl, 4 * j4 + q);
                 gg[q] = __shfl_sync(0xffffffffu, gl, 4 * j4 + q);
               }
-              o.x += gg[0] * (v[4 * j4] + bb[0]);
-              o.y += gg[1] * (v[4 * j4 + 1] + bb[1]);
-              o.z += gg[2] * (v[4 * j4 + 2] + bb[2]);
-              o.w += gg[3] * (v[4 * j4 + 3] + bb[3]);
-              *p4 = o;
+              rr[j4].x += gg[0] * (v[4 * j4] + bb[0]);
+              rr[j4].y += gg[1] * (v[4 * j4 + 1] + bb[1]);
+              rr[j4].z += gg[2] * (v[4 * j4 + 2] + bb[2]);
+              rr[j4].w += gg[3] * (v[4 * j4 + 3] + bb[3]);
             }
+#pragma unroll
+            for (int j4 = 0; j4 < 8; ++j4)
+              *reinterpret_cast<float4*>(tile_b + swz128(lane, j4)) = rr[j4];
           } else {
             // the store issued from this tile two chunks ago has left shared memory (the
             // one outstanding group allowed is the other tile's, one chunk ago)
