@@ -258,7 +258,9 @@ const char* fb_kernel_name(int kind);
  * between pairs are summed from fp32 partials in the model's workspace, in K order (so
  * the result does not depend on timing). impl 4 needs N % 256 == 0 and at least 4 K
  * blocks per SM pair (ceil(M / 256) * N / 256 * K / 64 >= 4 * pairs), else FB_ECUDA;
- * impl 0 uses whole tiles. */
+ * impl 0 takes the stream-K split only when K >= 96 * 64 and the whole 256 x 256 tiles
+ * number fewer than the SM pairs that can be resident (e.g. 1560 x 1536 x 8960), whole
+ * tiles otherwise. */
 /* fb_set_op_repeat: fb_op_gemm / fb_op_attention launch their kernel n >= 1 times back
  * to back (default 1), for timing a kernel without a stream synchronisation per launch. */
 fb_status fb_set_op_repeat(fb_model* m, int n);

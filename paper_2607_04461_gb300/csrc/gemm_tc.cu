@@ -421,7 +421,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
                     (first.kb0 + i) * BK, (first.tile % n_nt) * C2_BN + 128 * (int)rank);
   }
   griddep_wait();
-  griddep_launch();
+  // With the stream-K split a finisher waits for other clusters: no dependent grid may
+  // take SMs before this grid is done, so the dependents are released only at the end.
+  if (!use_sk) griddep_launch();
 
   if (warp == 0) {
     if (lane == 0) {
@@ -513,8 +515,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
       const float eg1 = has_gate ? __ldg(epi.gate + ecol + 32) : 1.f;
       const float eg2 = has_gate ? __ldg(epi.gate + ecol + 64) : 1.f;
       const float eg3 = has_gate ? __ldg(epi.gate + ecol + 96) : 1.f;
-      // whole tiles: the first two residual chunks load while the mainloop runs
-      const bool early = KIND == EPI_RESID && whole && row0 < M;
+      // the cluster holding K blocks 0.. of a cut tile finishes it (see the work split)
+      const bool head = !whole && sg.kb0 == 0;
+      // tiles this cluster finishes: the first two residual chunks load during the mainloop
+      const bool early = KIND == EPI_RESID && (whole || head) && row0 < M;
       if (early) {
         if (lane == 0) {
           bulk_wait_read<0>();
@@ -534,33 +538,53 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
       bool finish = whole;
       int c_lo = 0, n_c = 1;
       if (!whole) {
-        // a cut tile: publish this warp's partial, then count in on the tile's counter
         c_lo = sk_owner((long long)tile * nk, U, n_clusters);
         n_c = sk_owner((long long)(tile + 1) * nk - 1, U, n_clusters) - c_lo + 1;
-        float* part = sk_part(sk.ws, cluster, tile, U, n_clusters, nk, (int)rank, we);
-#pragma unroll 1
-        for (int cc = 0; cc < 4; ++cc) {
-          uint32_t r[32];
-          tmem_ld32(taddr + (half * 4 + cc) * 32, r);
-          tmem_ld_wait();
-          reg_fence32(r);
-          float4* dst = reinterpret_cast<float4*>(part + cc * 1024) + lane;
-#pragma unroll
-          for (int j4 = 0; j4 < 8; ++j4)
-            dst[j4 * 32] = make_float4(__uint_as_float(r[4 * j4]), __uint_as_float(r[4 * j4 + 1]),
-                                       __uint_as_float(r[4 * j4 + 2]),
-                                       __uint_as_float(r[4 * j4 + 3]));
-        }
-        __threadfence();
-        __syncwarp();
         int* ctr = sk.ctr + ((size_t)c_lo * 2 + rank) * 8 + we;
-        int old = 0;
-        if (lane == 0) old = atomicAdd(ctr, 1);
-        old = __shfl_sync(0xffffffffu, old, 0);
-        finish = old == n_c - 1;
-        if (finish) {
+        if (!head) {
+          // a later part of a cut tile: publish this warp's partial and count in
+          float* part = sk_part(sk.ws, cluster, tile, U, n_clusters, nk, (int)rank, we);
+#pragma unroll 1
+          for (int cc = 0; cc < 4; ++cc) {
+            uint32_t r[32];
+            tmem_ld32(taddr + (half * 4 + cc) * 32, r);
+            tmem_ld_wait();
+            reg_fence32(r);
+            float4* dst = reinterpret_cast<float4*>(part + cc * 1024) + lane;
+#pragma unroll
+            for (int j4 = 0; j4 < 8; ++j4)
+              dst[j4 * 32] = make_float4(__uint_as_float(r[4 * j4]),
+                                         __uint_as_float(r[4 * j4 + 1]),
+                                         __uint_as_float(r[4 * j4 + 2]),
+                                         __uint_as_float(r[4 * j4 + 3]));
+          }
           __threadfence();
-          if (lane == 0) *ctr = 0;  // every contributor has counted in: ready for reuse
+          __syncwarp();
+          if (lane == 0) atomicAdd(ctr, 1);
+        } else {
+          // the finisher: wait (bounded) until the other contributors' warps have counted
+          // in. They computed their parts at the start of their ranges, or over ranges no
+          // longer than this one, so the wait is short; all clusters are resident (the
+          // grid is at most the resident-cluster count, and in this mode no dependent
+          // grid starts before this one ends).
+          bool ok2 = true;
+          if (lane == 0) {
+            const uint64_t t0 = fb_globaltimer();
+            while (*(volatile int*)ctr < n_c - 1) {
+              if (*(volatile int*)err != 0) { ok2 = false; break; }
+              if (fb_globaltimer() - t0 > FB_WAIT_LIMIT_NS) {
+                atomicExch(err, FB_DEVERR_WAIT_TIMEOUT);
+                ok2 = false;
+                break;
+              }
+              __nanosleep(64);
+            }
+            if (ok2) *(volatile int*)ctr = 0;  // every contributor is in: ready for reuse
+          }
+          ok2 = __shfl_sync(0xffffffffu, ok2, 0);
+          if (!ok2) { failed = true; break; }
+          __threadfence();
+          finish = true;
         }
       }
       if (finish && row0 < M) {
@@ -698,6 +722,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
     tc_fence_after();
     tmem_dealloc_cg2(tmem_base, C2_TMEM_COLS);
   }
+  if (use_sk) griddep_launch();
 }
 
 PFN_cuTensorMapEncodeTiled_v12000 get_encode() {
@@ -806,16 +831,19 @@ cudaError_t launch2(const GemmArgs& g, int* err, int num_sms, cudaStream_t st) {
   const int tiles = ((g.M + 2 * BM - 1) / (2 * BM)) * (g.N / C2_BN);
   const int nk = g.K / BK;
   SkArgs sk{0, g.sk_ws, g.sk_ctr};
-  // Stream-K only on request (sk_mode 2): with every SM busy the mainloop's K blocks
-  // take longer and the partial write-back and sum of a cut tile cost more than the
-  // idle pairs of a short last wave save (measured at 1560 x 1536 x {1536, 8960}).
+  // Stream-K automatically only for a long K (>= 96 blocks) whose whole tiles leave pairs
+  // idle: there the spare pairs' share of the K loop outweighs writing and summing the
+  // partials of cut tiles (1560 x 1536 x 8960: 43.2 vs 47.9 us). With a short K, or with
+  // more tiles than pairs, the write-back and the waits cost more than the idle pairs of
+  // a short last wave save (1560 x 1536 x 1536: 22.9 vs 15.8 us).
   const long long U = (long long)tiles * nk;
   const bool sk_ok = g.sk_ws && g.sk_ctr && mc <= g.sk_clusters && U >= 4LL * mc;
   if (g.sk_mode == 2) {
     if (!sk_ok) return cudaErrorInvalidValue;
     sk.on = 1;
+  } else if (g.sk_mode == 0 && sk_ok && nk >= 96 && tiles < mc) {
+    sk.on = 1;
   }
-  (void)nk;
   const int clusters = sk.on ? mc : (tiles < mc ? tiles : mc);
   return launch_k(gemm_tc2_kernel<KIND>, dim3(2 * clusters), dim3(NUM_THREADS), C2_SMEM_BYTES, st,
                   ma, mw, mo, mr, g.M, g.N, g.K, g.epi, sk, err);

@@ -88,6 +88,27 @@ def test_gemm_stream_k_is_deterministic_and_matches_whole_tiles(model, M, N, K):
     assert rel_max(f64(outs[0]), f64(outs[2])) <= 1e-5
 
 
+@pytest.mark.parametrize("M,N,K,twin", [
+    (1560, 1536, 8960, 4),   # 42 tiles, 140 K blocks: stream-K
+    (640, 1536, 8960, 4),    # 18 tiles, 140 K blocks: stream-K
+    (1560, 1536, 1536, 3),   # 24 K blocks: whole tiles
+    (49920, 1536, 8960, 3),  # more tiles than SM pairs: whole tiles
+])
+def test_gemm_automatic_stream_k_choice(model, M, N, K, twin):
+    """impl 0 takes the stream-K split only for a long K under one wave of pair tiles: its
+    result is bit-identical to the forced variant it chose."""
+    A = randn((M, K), 51)
+    W = randn((N, K), 52, scale=K ** -0.5)
+    resid = randn((M, N), 53, dtype=torch.float32)
+    outs = []
+    for impl in (0, twin):
+        out = torch.empty((M, N), dtype=torch.float32, device="cuda")
+        fb.fb_op_gemm(model.handle, M, N, K, A, W, None, 2, out, resid, None, None, None, impl)
+        outs.append(out)
+    torch.cuda.synchronize()
+    assert torch.equal(outs[0], outs[1])
+
+
 def test_gemm_stream_k_in_place_residual(model):
     M, N, K = 1560, 1536, 8960
     A, W = randn((M, K), 31), randn((N, K), 32, scale=K ** -0.5)
