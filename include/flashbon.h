@@ -247,7 +247,7 @@ const char* fb_kernel_name(int kind);
  *   0: out bf16 = acc + bias
  *   1: out bf16 = gelu_tanh(acc + bias)
  *   2: out fp32 = resid[M][N] + gate[N] * (acc + bias)  (gate may be NULL = 1; resid may
- *      equal out)
+ *      equal out, or be NULL = 0: out fp32 = gate * (acc + bias))
  *   3: as 2, and also delta bf16 = out - base[M][N] (fp32), base may equal out
  * A, W bf16 row-major, leading dimensions K; out / resid / base / delta leading
  * dimension N. impl: 0 = automatic (tcgen05 when N % 128 == 0 and K % 64 == 0: the

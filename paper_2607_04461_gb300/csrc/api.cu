@@ -153,6 +153,14 @@ struct fb_model {
   float *patch_b, *time_b1, *time_b2, *mod_b, *text_b1, *text_b2, *head_table, *head_b;
   float* tables;  // [depth][6][D]
   std::vector<Layer> L;
+  // tensor-core patch embedding and head (C p p % 64 == 0, D % 128 == 0): bf16 patch rows
+  // [Mmax][PD]; head weights and bias zero-padded to npad = PD rounded up to 128 rows, and
+  // the head output [Mmax][npad] fp32. Null: the CUDA-core kernels.
+  bf16* patch_a = nullptr;
+  bf16* head_wp = nullptr;
+  float* head_bp = nullptr;
+  float* vbuf = nullptr;
+  int npad = 0;
   // activations
   float *hA = nullptr, *hB = nullptr;
   bf16 *act = nullptr, *qkv = nullptr, *ao = nullptr, *cqb = nullptr, *ffh = nullptr;
@@ -679,10 +687,19 @@ fb_status sample(fb_model* m, float* z, int n, const float* sched, int S, const 
     const float t = sched[k], t1 = sched[k + 1];
     CKS(time_embed(m, t));
     for (int u = 0; u < (so.guided ? 2 : 1); ++u) {
+      float* hu = m->hA + (size_t)u * n * m->P * c.dim;
       KTimer kt(m, FB_K_EMBED, 2.0 * n * m->P * (double)c.dim * m->PD,
-                4.0 * n * m->P * (double)(c.dim + m->PD));
-      CK(patch_embed(z, n, c.latent_c, c.latent_h, c.latent_w, c.patch, m->patch_w, m->patch_b,
-                     c.dim, m->hA + (size_t)u * n * m->P * c.dim, m->st));
+                4.0 * n * m->P * (double)(c.dim + m->PD), m->patch_a ? 2 : 1);
+      if (m->patch_a) {
+        // tensor cores: bf16 patch rows, then h = patches W_p^T + b_p (fp32, no residual)
+        CK(patchify(z, n, c.latent_c, c.latent_h, c.latent_w, c.patch, m->patch_a, m->st));
+        const GemmArgs g = gemm_args(n * m->P, c.dim, m->PD, m->patch_a, m->patch_w, m->patch_b,
+                                     EPI_RESID, hu);
+        CK(gemm_tc(g, m->derr, m->num_sms, m->st));
+      } else {
+        CK(patch_embed(z, n, c.latent_c, c.latent_h, c.latent_w, c.patch, m->patch_w, m->patch_b,
+                       c.dim, hu, m->st));
+      }
     }
     for (const Action& a : plan.steps[k]) {
       if (a.type == 0) {
@@ -719,9 +736,18 @@ fb_status sample(fb_model* m, float* z, int n, const float* sched, int S, const 
         hs.noise = so.noise + (size_t)k * zn;
       }
       KTimer kt(m, FB_K_HEAD, 2.0 * M * (double)c.dim * m->PD,
-                2.0 * M * (double)c.dim + 8.0 * M * m->PD);
-      CK(head_euler(m->act, n, c.latent_c, c.latent_h, c.latent_w, c.patch, m->head_w, m->head_b,
-                    c.dim, hs, z, m->st));
+                2.0 * M * (double)c.dim + 8.0 * M * m->PD, m->vbuf ? 2 : 1);
+      if (m->vbuf) {
+        // tensor cores: v = a W_h^T + b_h over npad zero-padded outputs, then the step
+        const GemmArgs g = gemm_args(M, m->npad, c.dim, m->act, m->head_wp, m->head_bp, EPI_RESID,
+                                     m->vbuf);
+        CK(gemm_tc(g, m->derr, m->num_sms, m->st));
+        CK(euler_step(m->vbuf, m->npad, n, c.latent_c, c.latent_h, c.latent_w, c.patch, hs, z,
+                      m->st));
+      } else {
+        CK(head_euler(m->act, n, c.latent_c, c.latent_h, c.latent_w, c.patch, m->head_w,
+                      m->head_b, c.dim, hs, z, m->st));
+      }
     }
   }
   return FB_OK;
@@ -986,6 +1012,22 @@ fb_status fb_init_model(const fb_cfg* cfg, const float* weights_host, fb_model**
   if (cudaMemset(m->sk_ctr, 0, (size_t)m->sk_clusters * SK_CTR_PER_CLUSTER * sizeof(int)) !=
       cudaSuccess)
     return bail(fail(FB_ECUDA, "cudaMemset failed"));
+  if (m->PD % 64 == 0 && D % 128 == 0) {
+    const size_t PDs = m->PD;
+    m->npad = (m->PD + 127) / 128 * 128;
+    if ((s = dalloc_t(m, &m->patch_a, M * PDs)) ||
+        (s = dalloc_t(m, &m->head_wp, (size_t)m->npad * D)) ||
+        (s = dalloc_t(m, &m->head_bp, (size_t)m->npad)) ||
+        (s = dalloc_t(m, &m->vbuf, M * m->npad)))
+      return bail(s);
+    if (cudaMemset(m->head_wp, 0, (size_t)m->npad * D * sizeof(bf16)) != cudaSuccess ||
+        cudaMemset(m->head_bp, 0, (size_t)m->npad * sizeof(float)) != cudaSuccess ||
+        cudaMemcpy(m->head_wp, m->head_w, PDs * D * sizeof(bf16), cudaMemcpyDeviceToDevice) !=
+            cudaSuccess ||
+        cudaMemcpy(m->head_bp, m->head_b, PDs * sizeof(float), cudaMemcpyDeviceToDevice) !=
+            cudaSuccess)
+      return bail(fail(FB_ECUDA, "head weight padding failed"));
+  }
   // RoPE table: pair j of a head rotates by the token's row (j < head_dim/4) or column,
   // with frequency theta^(-2 j' / (head_dim/2)), j' = j mod head_dim/4.
   {
@@ -1221,7 +1263,7 @@ fb_status fb_op_gemm(fb_model* m, int M, int N, int K, const void* A, const void
                      const float* gate, const float* base, void* delta, int impl) {
   if (!m || !A || !W || !out) return fail(FB_EINVAL, "null argument");
   if (M < 1 || N < 1 || K < 1 || epi < 0 || epi > 3) return fail(FB_EINVAL, "bad sizes / epi");
-  if (epi >= EPI_RESID && !resid) return fail(FB_EINVAL, "resid required");
+  if (epi == EPI_RESID_DELTA && !resid) return fail(FB_EINVAL, "resid required");
   if (epi == EPI_RESID_DELTA && (!base || !delta)) return fail(FB_EINVAL, "base/delta required");
   if (N % 8) return fail(FB_EINVAL, "N must be a multiple of 8");
   GemmArgs g = gemm_args(M, N, K, (const bf16*)A, (const bf16*)W, bias, epi, out);
@@ -1301,7 +1343,7 @@ fb_status fb_gemm_streamk_noalloc(void* stream, int M, int N, int K, const void*
                                   void* delta) {
   if (!A || !W || !out) return fail(FB_EINVAL, "null argument");
   if (M < 1 || N < 1 || K < 1 || epi < 0 || epi > 3) return fail(FB_EINVAL, "bad sizes / epi");
-  if (epi >= EPI_RESID && !resid) return fail(FB_EINVAL, "resid required");
+  if (epi == EPI_RESID_DELTA && !resid) return fail(FB_EINVAL, "resid required");
   if (epi == EPI_RESID_DELTA && (!base || !delta)) return fail(FB_EINVAL, "base/delta required");
   if (N % 256) return fail(FB_EINVAL, "N must be a multiple of 256");
   GemmArgs g = gemm_args(M, N, K, (const bf16*)A, (const bf16*)W, bias, epi, out);

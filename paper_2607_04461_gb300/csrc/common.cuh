@@ -336,7 +336,7 @@ struct SkArgs {
 struct GemmEpi {
   const float* bias;   // [N] or null
   void* out;           // bf16 (EPI_BF16, EPI_GELU_BF16) or fp32 (EPI_RESID*)
-  const float* resid;  // fp32 [M][ldo]
+  const float* resid;  // fp32 [M][ldo]; EPI_RESID: null = no residual (out = gate * (acc + bias))
   const float* gate;   // fp32 [N] or null (= 1)
   const float* base;   // fp32 [M][ldo] (EPI_RESID_DELTA)
   bf16* delta;         // bf16 [M][ldo] (EPI_RESID_DELTA)
@@ -347,7 +347,7 @@ struct GemmEpi {
 // the next tile's rows into L2 while the mainloop runs, so those reads hit L2.
 template <int KIND>
 __device__ __forceinline__ void epi_prefetch(const GemmEpi& e, int row, int col, int ncols) {
-  if (KIND >= EPI_RESID) {
+  if (KIND >= EPI_RESID && e.resid) {
     const size_t off = (size_t)row * e.ldo + col;
     prefetch_l2_bulk(e.resid + off, ncols * 4);
     if (KIND == EPI_RESID_DELTA && e.base != e.resid) prefetch_l2_bulk(e.base + off, ncols * 4);
@@ -367,7 +367,12 @@ __device__ __forceinline__ void epi_apply32(const GemmEpi& e, int row, int col, 
     float r[32], bs[32];
 #pragma unroll
     for (int j = 0; j < 32; j += 8) {
-      load_f32x8(e.resid + off + j, r + j);
+      if (KIND == EPI_RESID_DELTA || e.resid) {
+        load_f32x8(e.resid + off + j, r + j);
+      } else {
+#pragma unroll
+        for (int q = 0; q < 8; ++q) r[j + q] = 0.f;
+      }
       if (KIND == EPI_RESID_DELTA) load_f32x8(e.base + off + j, bs + j);
     }
 #pragma unroll
@@ -427,7 +432,12 @@ __device__ __forceinline__ void epi_apply8(const GemmEpi& e, int row, int col, f
     store_bf16x8(reinterpret_cast<bf16*>(e.out) + off, v);
   } else {
     float r[8], g[8];
-    load_f32x8(e.resid + off, r);
+    if (KIND == EPI_RESID_DELTA || e.resid) {
+      load_f32x8(e.resid + off, r);
+    } else {
+#pragma unroll
+      for (int j = 0; j < 8; ++j) r[j] = 0.f;
+    }
     if (e.gate) {
       load_f32x8(e.gate + col, g);
     } else {

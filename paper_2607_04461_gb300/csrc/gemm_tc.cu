@@ -304,12 +304,14 @@ __device__ __forceinline__ void epi_resid_staged(const GemmEpi& e, float* stg, i
 // Data-parallel: cluster c computes whole tiles c, c + G, c + 2G, ... (G clusters).
 // Stream-K: the U = tiles x nk (tile, K-block) units, tile-major, are cut into G
 // contiguous ranges of floor(c U / G) .. floor((c + 1) U / G); a cluster walks its range
-// as segments (one tile, K-blocks kb0..kb1). A tile cut between clusters c_lo..c_hi gets
-// one fp32 partial accumulator per contributor; each epilogue warp writes its part of the
-// partial to the workspace and counts itself on the tile's counter, and the last of the
-// contributors' warps to arrive adds the partials in contributor (= K) order, so the sum
-// does not depend on arrival order, runs the epilogue and resets the counter to zero.
-// With U >= G every range is non-empty, so c_hi - c_lo + 1 clusters contribute.
+// as segments (one tile, K-blocks kb0..kb1). A tile cut between clusters c_lo..c_hi is
+// finished by c_lo, which holds its first K blocks as the last segment of its range; the
+// others reach it as the first segment of theirs. Each of their epilogue warps writes its
+// part of an fp32 partial to the workspace and counts itself on the tile's counter; c_lo's
+// matching warp waits (bounded) for the count, adds the partials in contributor (= K)
+// order, so the sum does not depend on arrival order, runs the epilogue and resets the
+// counter to zero. With U >= G every range is non-empty, so c_hi - c_lo + 1 clusters
+// contribute.
 struct Seg {
   int tile, kb0, kb1;
 };
@@ -421,9 +423,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
                     (first.kb0 + i) * BK, (first.tile % n_nt) * C2_BN + 128 * (int)rank);
   }
   griddep_wait();
-  // With the stream-K split a finisher waits for other clusters: no dependent grid may
-  // take SMs before this grid is done, so the dependents are released only at the end.
-  if (!use_sk) griddep_launch();
+  // Dependents may start once every CTA of this grid has passed here: with the stream-K
+  // split all contributors are then resident, so a finisher's wait cannot be starved.
+  griddep_launch();
 
   if (warp == 0) {
     if (lane == 0) {
@@ -518,7 +520,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
       // the cluster holding K blocks 0.. of a cut tile finishes it (see the work split)
       const bool head = !whole && sg.kb0 == 0;
       // tiles this cluster finishes: the first two residual chunks load during the mainloop
-      const bool early = KIND == EPI_RESID && (whole || head) && row0 < M;
+      const bool has_r = KIND == EPI_RESID && epi.resid != nullptr;
+      const bool early = has_r && (whole || head) && row0 < M;
       if (early) {
         if (lane == 0) {
           bulk_wait_read<0>();
@@ -564,9 +567,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
         } else {
           // the finisher: wait (bounded) until the other contributors' warps have counted
           // in. They computed their parts at the start of their ranges, or over ranges no
-          // longer than this one, so the wait is short; all clusters are resident (the
-          // grid is at most the resident-cluster count, and in this mode no dependent
-          // grid starts before this one ends).
+          // longer than this one, so the wait is short. Every contributor gets an SM: the
+          // grid is at most the resident-cluster count, and a dependent grid starts only
+          // after all of this grid's CTAs have started.
           bool ok2 = true;
           if (lane == 0) {
             const uint64_t t0 = fb_globaltimer();
@@ -588,7 +591,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
         }
       }
       if (finish && row0 < M) {
-        if (KIND == EPI_RESID && !early) {
+        if (has_r && !early) {
           if (lane == 0) {
             bulk_wait_read<0>();
             for (int cc = 0; cc < 2; ++cc) rload_issue(cc);
@@ -646,15 +649,24 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
           const float bl = cc == 0 ? eb0 : cc == 1 ? eb1 : cc == 2 ? eb2 : eb3;
           const float gl = cc == 0 ? eg0 : cc == 1 ? eg1 : cc == 2 ? eg2 : eg3;
           if (KIND == EPI_RESID) {
-            const bool lok = mbar_wait(&rload[2 * we + b], (rl_phase >> b) & 1u, err);
-            rl_phase ^= 1u << b;
-            if (!__all_sync(0xffffffffu, lok)) { failed = true; break; }
-            // all eight residual loads first: a load after a store to the same tile
-            // would otherwise wait for it
             float4 rr[8];
+            if (has_r) {
+              const bool lok = mbar_wait(&rload[2 * we + b], (rl_phase >> b) & 1u, err);
+              rl_phase ^= 1u << b;
+              if (!__all_sync(0xffffffffu, lok)) { failed = true; break; }
+              // all eight residual loads first: a load after a store to the same tile
+              // would otherwise wait for it
 #pragma unroll
-            for (int j4 = 0; j4 < 8; ++j4)
-              rr[j4] = *reinterpret_cast<const float4*>(tile_b + swz128(lane, j4));
+              for (int j4 = 0; j4 < 8; ++j4)
+                rr[j4] = *reinterpret_cast<const float4*>(tile_b + swz128(lane, j4));
+            } else {
+              // no residual: only the store issued from this tile two chunks ago must
+              // have left shared memory
+              if (lane == 0) bulk_wait_read<1>();
+              __syncwarp();
+#pragma unroll
+              for (int j4 = 0; j4 < 8; ++j4) rr[j4] = make_float4(0.f, 0.f, 0.f, 0.f);
+            }
 #pragma unroll
             for (int j4 = 0; j4 < 8; ++j4) {
               float bb[4], gg[4];
@@ -694,7 +706,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
           if (lane == 0) {
             tma_store_2d(&tmO, smem_u32(tile_b), col0, row0);
             bulk_commit();
-            if (KIND == EPI_RESID && cc + 2 < 4) {
+            if (has_r && cc + 2 < 4) {
               bulk_wait_read<0>();  // the tile is free again: next residual chunk into it
               rload_issue(cc + 2);
             }
@@ -722,7 +734,6 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
     tc_fence_after();
     tmem_dealloc_cg2(tmem_base, C2_TMEM_COLS);
   }
-  if (use_sk) griddep_launch();
 }
 
 PFN_cuTensorMapEncodeTiled_v12000 get_encode() {
@@ -807,7 +818,9 @@ cudaError_t launch2(const GemmArgs& g, int* err, int num_sms, cudaStream_t st) {
   if (C2Cfg<KIND>::TMA_EPI &&
       !make_epi_map(&mo, g.epi.out, KIND == EPI_RESID, g.M, g.N, g.epi.ldo))
     return cudaErrorInvalidValue;
-  if (KIND == EPI_RESID && !make_epi_map(&mr, g.epi.resid, true, g.M, g.N, g.epi.ldo))
+  mr = CUtensorMap{};  // unused without a residual
+  if (KIND == EPI_RESID && g.epi.resid &&
+      !make_epi_map(&mr, g.epi.resid, true, g.M, g.N, g.epi.ldo))
     return cudaErrorInvalidValue;
   constexpr int C2_SMEM_BYTES = C2Cfg<KIND>::SMEM_BYTES;
   cudaError_t e = cudaFuncSetAttribute(gemm_tc2_kernel<KIND>,
@@ -865,7 +878,7 @@ bool gemm_tc_supported(const GemmArgs& g) {
   auto al16 = [](const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15) == 0; };
   return g.M >= 1 && g.N % 128 == 0 && g.K % BK == 0 && g.K >= BK && g.lda % 8 == 0 &&
          g.ldw % 8 == 0 && g.epi.ldo % 8 == 0 && al16(g.A) && al16(g.W) && al16(g.epi.out) &&
-         (g.kind < EPI_RESID || al16(g.epi.resid)) &&
+         (g.kind < EPI_RESID || al16(g.epi.resid)) && (g.kind != EPI_RESID_DELTA || g.epi.resid) &&
          (g.kind != EPI_RESID_DELTA || (al16(g.epi.base) && al16(g.epi.delta)));
 }
 

@@ -83,6 +83,14 @@ struct HeadStep {
 };
 cudaError_t head_euler(const bf16* a, int n, int C, int H, int W, int p, const bf16* Wh,
                        const float* bh, int D, const HeadStep& hs, float* z, cudaStream_t st);
+// out[b P + tok][(ch, dy, dx)] = bf16(z[b][ch][r p + dy][c p + dx]) for token tok = r (W/p) + c:
+// the patch rows of z, the A operand of the tensor-core patch embedding (C p p % 8 == 0).
+cudaError_t patchify(const float* z, int n, int C, int H, int W, int p, bf16* out,
+                     cudaStream_t st);
+// The guidance combination and step of head_euler, with v[row][o] (fp32, leading dimension
+// ldv >= C p p) the head output a Wh^T + bh computed by the tensor-core GEMM.
+cudaError_t euler_step(const float* v, int ldv, int n, int C, int H, int W, int p,
+                       const HeadStep& hs, float* z, cudaStream_t st);
 // y[o] = act_out(b[o] + sum_k W[o][k] act_in(x[k])), act: 0 none, 1 SiLU.
 cudaError_t gemv(const bf16* W, const float* b, const float* x, float* y, int O, int K,
                  int act_in, int act_out, cudaStream_t st);

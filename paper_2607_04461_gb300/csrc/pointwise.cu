@@ -6,7 +6,9 @@
 //               contributions): h += sum_t c_t Delta_t, one read and write of h per run.
 //  patch_embed  2x2 patchify + linear (D x C p p), writes the fp32 residual stream.
 //  head_euler   output projection D -> C p p, unpatchify and the Euler step
-//               z += (t' - t) v of dx = v dt, fused.
+//               z += (t' - t) v of dx = v dt, fused (CUDA cores, any C p p).
+//  patchify     z -> bf16 patch rows, the A operand of the tensor-core patch embedding.
+//  euler_step   the step of head_euler from the tensor-core head GEMM's output.
 //  gemv, timestep_sincos, mod_prepare, f32_to_bf16: per-step conditioning, conversions.
 #include "kernels.h"
 
@@ -80,7 +82,8 @@ cudaError_t ln_mod_launch(const float* x, bf16* out, int rows, int D, float eps,
 }
 
 // ---------------------------------------------------------------------------------
-// qk_norm_rope: THREADS threads per (row, segment), VPT chunks of 4 bf16 per thread.
+// qk_norm_rope: THREADS threads per (row, segment), VPT chunks of 4 bf16 per thread, ROWS
+// rows per block (ROWS > 1 only with one warp per row).
 __device__ __forceinline__ void load_bf16x4(const bf16* p, float* v) {
   uint2 u = *reinterpret_cast<const uint2*>(p);
   float2 a = unpack_bf16x2(u.x), b = unpack_bf16x2(u.y);
@@ -93,15 +96,18 @@ __device__ __forceinline__ void store_bf16x4(bf16* p, const float* v) {
   *reinterpret_cast<uint2*>(p) = u;
 }
 
-template <int THREADS, int VPT>
-__global__ void __launch_bounds__(THREADS) qk_norm_rope_kernel(
-    bf16* __restrict__ x, int ld, int D, int col0, const float* __restrict__ w0, int col1,
-    const float* __restrict__ w1, float eps, const float2* __restrict__ rope, int tokens,
-    int head_dim) {
+template <int THREADS, int VPT, int ROWS>
+__global__ void __launch_bounds__(THREADS * ROWS) qk_norm_rope_kernel(
+    bf16* __restrict__ x, int rows, int ld, int D, int col0, const float* __restrict__ w0,
+    int col1, const float* __restrict__ w1, float eps, const float2* __restrict__ rope,
+    int tokens, int head_dim) {
+  static_assert(ROWS == 1 || THREADS == 32, "several rows per block need one warp per row");
   griddep_wait();
   griddep_launch();
   __shared__ float red[THREADS / 32 > 0 ? THREADS / 32 : 1];
-  const size_t row = blockIdx.x;
+  const size_t row = (size_t)blockIdx.x * ROWS + threadIdx.x / THREADS;
+  if (row >= (size_t)rows) return;
+  const int tid = threadIdx.x % THREADS;
   const int seg = blockIdx.y;
   const int col0s = seg ? col1 : col0;
   const float* w = seg ? w1 : w0;
@@ -110,7 +116,7 @@ __global__ void __launch_bounds__(THREADS) qk_norm_rope_kernel(
   float ss = 0.f;
 #pragma unroll
   for (int i = 0; i < VPT; ++i) {
-    load_bf16x4(xr + (i * THREADS + threadIdx.x) * 4, v[i]);
+    load_bf16x4(xr + (i * THREADS + tid) * 4, v[i]);
 #pragma unroll
     for (int j = 0; j < 4; ++j) ss += v[i][j] * v[i][j];
   }
@@ -118,7 +124,7 @@ __global__ void __launch_bounds__(THREADS) qk_norm_rope_kernel(
   const float2* rp = rope ? rope + (size_t)(row % tokens) * (head_dim / 2) : nullptr;
 #pragma unroll
   for (int i = 0; i < VPT; ++i) {
-    const int col = (i * THREADS + threadIdx.x) * 4;
+    const int col = (i * THREADS + tid) * 4;
     const float4 wv = *reinterpret_cast<const float4*>(w + col);
     v[i][0] *= r * wv.x; v[i][1] *= r * wv.y; v[i][2] *= r * wv.z; v[i][3] *= r * wv.w;
     if (rp) {
@@ -135,13 +141,13 @@ __global__ void __launch_bounds__(THREADS) qk_norm_rope_kernel(
   }
 }
 
-template <int THREADS, int VPT>
+template <int THREADS, int VPT, int ROWS = 1>
 cudaError_t qkn_launch(bf16* x, int rows, int ld, int D, int nseg, int col0, const float* w0,
                        int col1, const float* w1, float eps, const float2* rope, int tokens,
                        int head_dim, cudaStream_t st) {
-  dim3 grid(rows, nseg);
-  return launch_k(qk_norm_rope_kernel<THREADS, VPT>, grid, dim3(THREADS), 0, st, x, ld, D, col0, w0,
-                  col1, w1, eps, rope, tokens, head_dim);
+  dim3 grid((rows + ROWS - 1) / ROWS, nseg);
+  return launch_k(qk_norm_rope_kernel<THREADS, VPT, ROWS>, grid, dim3(THREADS * ROWS), 0, st, x,
+                  rows, ld, D, col0, w0, col1, w1, eps, rope, tokens, head_dim);
 }
 
 // ---------------------------------------------------------------------------------
@@ -206,6 +212,64 @@ __global__ void __launch_bounds__(256) patch_embed_kernel(const float* __restric
 #pragma unroll
     for (int t = 0; t < PE_TOK; ++t)
       if (tok0 + t < M) h[(size_t)(tok0 + t) * D + col] = acc[t];
+  }
+}
+
+// ---------------------------------------------------------------------------------
+// patchify: the patch rows of z in bf16, the A operand of the tensor-core patch
+// embedding. Thread -> 8 consecutive columns (ch, dy, dx) of one row (b P + token).
+__global__ void __launch_bounds__(256) patchify_kernel(const float* __restrict__ z, int n, int C,
+                                                       int H, int W, int p,
+                                                       bf16* __restrict__ out) {
+  griddep_wait();
+  griddep_launch();
+  const int PD = C * p * p, gw = W / p, P = (H / p) * gw, pp = p * p;
+  const size_t total = (size_t)n * P * (PD / 8);
+  for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < total;
+       i += (size_t)gridDim.x * blockDim.x) {
+    const size_t row = i / (PD / 8);
+    const int k0 = (int)(i % (PD / 8)) * 8;
+    const int b = (int)(row / P), pt = (int)(row % P), r = pt / gw, cc = pt % gw;
+    float v[8];
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      const int k = k0 + j, ch = k / pp, dy = (k / p) % p, dx = k % p;
+      v[j] = z[(((size_t)b * C + ch) * H + r * p + dy) * W + cc * p + dx];
+    }
+    store_bf16x8(out + row * PD + k0, v);
+  }
+}
+
+// euler_step: the guidance combination and the ODE / SDE step of head_euler, from the
+// head output v[row][o] (bias included) of the tensor-core head GEMM. Thread -> one
+// element (b, ch, y, x) of z, which reads output o = (ch, y % p, x % p) of token
+// (y / p, x / p) of candidate b.
+__global__ void __launch_bounds__(256) euler_step_kernel(const float* __restrict__ v, int ldv,
+                                                         int n, int C, int H, int W, int p,
+                                                         HeadStep hs, float* __restrict__ z) {
+  griddep_wait();
+  griddep_launch();
+  const int gw = W / p, P = (H / p) * gw;
+  const size_t total = (size_t)n * C * H * W;
+  for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < total;
+       i += (size_t)gridDim.x * blockDim.x) {
+    const int x = (int)(i % W);
+    size_t t = i / W;
+    const int y = (int)(t % H);
+    t /= H;
+    const int ch = (int)(t % C), b = (int)(t / C);
+    const size_t tok = (size_t)b * P + (y / p) * gw + x / p;
+    const int o = (ch * p + y % p) * p + x % p;
+    float vv = v[tok * ldv + o];
+    if (hs.uncond_rows) {
+      const float vu = v[(tok + hs.uncond_rows) * ldv + o];
+      vv = vu + hs.w * (vv - vu);
+    }
+    const float zo = z[i];
+    if (hs.noise)
+      z[i] = zo + (vv + hs.sde_c * (zo + (1.f - hs.t) * vv)) * hs.dt + hs.nscale * hs.noise[i];
+    else
+      z[i] = zo + hs.dt * vv;
   }
 }
 
@@ -377,13 +441,16 @@ cudaError_t qk_norm_rope(bf16* x, int rows, int ld, int D, int nseg, int col0, c
                          int col1, const float* w1, float eps, const float2* rope, int tokens,
                          int head_dim, cudaStream_t st) {
   if (rows == 0) return cudaSuccess;
-#define QKN(T, V) qkn_launch<T, V>(x, rows, ld, D, nseg, col0, w0, col1, w1, eps, rope, tokens, head_dim, st)
+#define QKN(T, V, ...) \
+  qkn_launch<T, V, ##__VA_ARGS__>(x, rows, ld, D, nseg, col0, w0, col1, w1, eps, rope, tokens, head_dim, st)
   switch (D) {  // threads * 4 * VPT == D
     case 128: return QKN(32, 1);
     case 256: return QKN(64, 1);
     case 512: return QKN(128, 1);
     case 1024: return QKN(128, 2);
-    case 1536: return QKN(32, 12);  // one warp per row: 96 bytes in flight per thread
+    // one warp per row (96 bytes in flight per thread), two rows per block: at 49920 x
+    // 2 x 1536 this runs at 6.1 TB/s against 5.4 with one row per block
+    case 1536: return QKN(32, 12, 2);
     case 2048: return QKN(128, 4);
     case 3072: return QKN(256, 3);
     case 4096: return QKN(256, 4);
@@ -391,6 +458,25 @@ cudaError_t qk_norm_rope(bf16* x, int rows, int ld, int D, int nseg, int col0, c
   }
 #undef QKN
   return cudaErrorInvalidValue;
+}
+
+cudaError_t patchify(const float* z, int n, int C, int H, int W, int p, bf16* out,
+                     cudaStream_t st) {
+  const int PD = C * p * p;
+  if (PD % 8 || H % p || W % p) return cudaErrorInvalidValue;
+  const size_t work = (size_t)n * (H / p) * (W / p) * (PD / 8);
+  if (work == 0) return cudaSuccess;
+  return launch_k(patchify_kernel, dim3(grid_for(work, 256)), dim3(256), 0, st, z, n, C, H, W, p,
+                  out);
+}
+
+cudaError_t euler_step(const float* v, int ldv, int n, int C, int H, int W, int p,
+                       const HeadStep& hs, float* z, cudaStream_t st) {
+  if (H % p || W % p || ldv < C * p * p) return cudaErrorInvalidValue;
+  const size_t work = (size_t)n * C * H * W;
+  if (work == 0) return cudaSuccess;
+  return launch_k(euler_step_kernel, dim3(grid_for(work, 256)), dim3(256), 0, st, v, ldv, n, C, H,
+                  W, p, hs, z);
 }
 
 cudaError_t proxy_add(float* h, size_t n_elems, const ProxyTerms& t, cudaStream_t st) {

@@ -165,6 +165,30 @@ def _gemm_case(model, M, N, K, epi, impl):
             assert rel_max(f64(delta), want - f64(base)) <= 1e-2
 
 
+@pytest.mark.parametrize("M,N,K,impl", [
+    (4999, 1536, 64, 0),     # the patch embedding: 2-SM kernel, one K block, ragged rows
+    (3000, 128, 1536, 0),    # the padded head: 1-SM kernel, N = 128
+    (300, 256, 128, 3),      # 2-SM whole tiles
+    (1560, 1536, 8960, 4),   # 2-SM stream-K (cut tiles summed before the epilogue)
+    (300, 256, 128, 2),      # 1-SM kernel forced
+    (77, 24, 40, 1),         # CUDA-core kernel
+])
+@pytest.mark.parametrize("gated", [False, True])
+def test_gemm_fp32_out_without_residual(model, M, N, K, impl, gated):
+    """epi 2 with resid NULL: out = gate * (A W^T + bias) in fp32, every element written."""
+    A = randn((M, K), 61)
+    W = randn((N, K), 62, scale=K ** -0.5)
+    bias = randn((N,), 63, dtype=torch.float32)
+    gate = randn((N,), 64, dtype=torch.float32) if gated else None
+    out = torch.full((M, N), float("nan"), dtype=torch.float32, device="cuda")
+    fb.fb_op_gemm(model.handle, M, N, K, A, W, bias, 2, out, None, gate, None, None, impl)
+    torch.cuda.synchronize()
+    y = O.linear(f64(A), f64(W), f64(bias))
+    want = f64(gate) * y if gated else y
+    assert not torch.isnan(out).any()
+    assert rel_max(f64(out), want) <= 1e-4
+
+
 def test_gemm_in_place_residual(model):
     """out == resid and base == out (the block's last GEMM runs this way)."""
     M, N, K = 257, 256, 128
