@@ -284,6 +284,55 @@ def test_wan13_draft_pool_full_size(wan13_pool):
     check_latents(two.cpu().numpy()[0], want[0], z[0], label="wan13 cand 0, 2 steps")
 
 
+# ---- the other shapes of the scope table: Wan2.1-14B width, 4096 tokens ---------------
+# One-block models: every kernel shape of the full models (D = 5120 with 40 heads and
+# FFN 13824; 4096 tokens per candidate, 32 key tiles), at an oracle cost of seconds.
+
+@pytest.fixture(scope="module", params=["wan14", "wan13_1k"])
+def wide(request):
+    cfg = {"wan14": synth.WAN14, "wan13_1k": synth.WAN13_1K}[request.param].with_(depth=1,
+                                                                                 max_n=2)
+    w = synth.make_weights(cfg)
+    m = fb.Model(cfg, w)
+    yield request.param, cfg, w, m
+    m.close()
+
+
+def test_wide_single_block_n2(wide):
+    """One block at N=2: both candidates against the oracle."""
+    name, cfg, w, m = wide
+    ctx = synth.make_text(cfg)
+    rng = np.random.default_rng(12)
+    n, t = 2, 0.7
+    h = rng.standard_normal((n * cfg.tokens, cfg.dim)).astype(np.float32)
+    m.encode_text(ctx)
+    hd = cuda(h)
+    m.block_forward(0, hd, n, t)
+    got = hd.cpu().numpy().astype(np.float64) - h
+    ref = O.OracleModel(cfg, w)
+    kv = ref.encode_text(ctx)
+    _, mod = ref.time_embed(np.float32(t))
+    for j in range(n):
+        sl = slice(j * cfg.tokens, (j + 1) * cfg.tokens)
+        want = ref.block(0, h[sl].astype(np.float64), mod, kv[0]) - h[sl]
+        e = rel_max(got[sl], want)
+        assert e <= BLOCK_TOL, f"{name} cand {j}: {e:.3e}"
+
+
+def test_wide_two_step_draft(wide):
+    """Two full steps of one candidate: patch embedding, time embedding, block and head
+    at these widths against the oracle."""
+    name, cfg, w, m = wide
+    ctx = synth.make_text(cfg)
+    sched = synth.make_schedule(50)[:3]
+    skip, proxy = synth.empty_plan(2, cfg.depth)
+    z = synth.make_latents(cfg, 1)
+    a = cuda(z)
+    m.draft(a, ctx, sched, skip, proxy)
+    want = O.OracleModel(cfg, w).draft(z, ctx, sched, skip, proxy)
+    check_latents(a.cpu().numpy()[0], want[0], z[0], label=f"{name} 2 steps")
+
+
 # ---- NEXT rows: classifier-free guidance and SDE steps -------------------------------
 
 @pytest.fixture(scope="module")
