@@ -47,6 +47,31 @@ def workload():
     return cfg, sched, skip, proxy
 
 
+# The paper's searched configuration phi* on the Wan2.1-1.3B shape (Sec. 4.1): S = 50,
+# S' = 49 draft steps, blocks 22-23 skipped from step 3 on, a full step every 5 steps, the
+# others forecast with second-order proxies; N = 8 candidates; the remaining step refines
+# candidate 0.
+PHI_STAR = dict(S=50, S_prime=49, n_skip=3, l_start=22, l_end=23, f_full=5, order=2)
+PHI_N = 8
+
+
+def plan_for(variant):
+    """(cfg, schedule, skip, proxy, draft steps) of a bench variant."""
+    if variant == "full50":  # the same N and schedule sampled without any acceleration
+        cfg = synth.WAN13.with_(max_n=PHI_N)
+        skip, proxy = synth.empty_plan(PHI_STAR["S"], cfg.depth)
+        return cfg, synth.make_schedule(PHI_STAR["S"]), skip, proxy, PHI_STAR["S"]
+    if variant != "phi_star":
+        cfg, sched, skip, proxy = workload()
+        return cfg, sched, skip, proxy, S_DRAFT
+    from paper_2607_04461_gb300 import flashbon as fb
+    cfg = synth.WAN13.with_(max_n=PHI_N)
+    ph = PHI_STAR
+    skip, proxy = fb.fb_plan_from_phi(ph["S"], ph["S_prime"], ph["n_skip"], ph["l_start"],
+                                      ph["l_end"], ph["f_full"], ph["order"], cfg.depth)
+    return cfg, synth.make_schedule(ph["S"]), skip, proxy, ph["S_prime"]
+
+
 VARIANTS = {
     "base": "",
     "cfg": "; classifier-free guidance w=5 (16 candidates, 32 rows with the unconditional pass)",
@@ -54,15 +79,33 @@ VARIANTS = {
     "offload": "; every candidate's cached state (each layer's last contribution, bf16, "
                "144 MB per candidate) copied to pinned host memory behind the refine and "
                "the next draft",
+    "phi_star": "",
+    "full50": "",
 }
 
 
 def n_candidates(variant):
-    return N_CAND // 2 if variant == "cfg" else N_CAND
+    return {"cfg": N_CAND // 2, "phi_star": PHI_N, "full50": PHI_N}.get(variant, N_CAND)
 
 
 def config_dict(cfg, variant="base"):
     n = n_candidates(variant)
+    if variant == "phi_star":
+        ph = PHI_STAR
+        return {"workload": f"wan2.1-1.3B, the paper's phi*: N={n}, 480x832 (1560 tokens), "
+                            f"{ph['S_prime']} of {ph['S']} steps, blocks {ph['l_start']}-"
+                            f"{ph['l_end']} skipped from step {ph['n_skip']}, a full step "
+                            f"every {ph['f_full']}, order-{ph['order']} proxies between, "
+                            "then the remaining step of candidate 0",
+                "n_candidates": n, "tokens": cfg.tokens, "dim": cfg.dim, "depth": cfg.depth,
+                "draft_steps": ph["S_prime"], "refine_steps": ph["S"] - ph["S_prime"],
+                "l2": "inputs larger than L2 (2.6 GB weights), no flush"}
+    if variant == "full50":
+        return {"workload": f"wan2.1-1.3B: N={n}, 480x832 (1560 tokens), all 50 steps, every "
+                            "block computed (sampling without the paper's acceleration)",
+                "n_candidates": n, "tokens": cfg.tokens, "dim": cfg.dim, "depth": cfg.depth,
+                "draft_steps": PHI_STAR["S"], "refine_steps": 0,
+                "l2": "inputs larger than L2 (2.6 GB weights), no flush"}
     return {"workload": f"wan2.1-1.3B draft pool: N={n}, 480x832 (1560 tokens), 10 of 50 "
                         "steps, 1/3 blocks skipped, half of the rest proxied on odd steps, "
                         "then a 40-step full refine of candidate 0" + VARIANTS[variant],
@@ -254,7 +297,7 @@ def run_gb300(args):
         import torch.distributed as dist
         dist.init_process_group("nccl", device_id=torch.device("cuda", local))
         pg = dist
-    cfg, sched, skip, proxy = workload()
+    cfg, sched, skip, proxy, s_draft = plan_for(args.variant)
     NC = n_candidates(args.variant)
     t_setup = time.time()
     w = synth.make_weights(cfg)
@@ -268,7 +311,7 @@ def run_gb300(args):
     ctx = torch.from_numpy(ctx_h).cuda()
     z = torch.empty_like(z0)
     zr = torch.empty_like(z0[0])
-    draft_sched, tail = sched[: S_DRAFT + 1], sched[S_DRAFT:]
+    draft_sched, tail = sched[: s_draft + 1], sched[s_draft:]
     opts_d = opts_r = None
     if args.variant == "cfg":
         ctx_u = torch.from_numpy(synth.make_text(cfg, seed=8)).cuda()
@@ -397,7 +440,7 @@ def run_gb300(args):
     launches = sum(s["launches"] for s in launch_stats.values())
     passes = 2 if args.variant == "cfg" else 1
     algo_flops = passes * (NC * computed_blocks(skip, proxy) * block_flops(cfg) +
-                           (S_TOTAL - S_DRAFT) * cfg.depth * block_flops(cfg))
+                           (S_TOTAL - s_draft) * cfg.depth * block_flops(cfg))
     out = {"metric": METRIC, "value": value, "unit": "candidates/s", "n_gpus": ws,
            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_step,
            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
