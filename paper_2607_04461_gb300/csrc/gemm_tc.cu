@@ -374,7 +374,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
   uint64_t* tmem_full = empty + C2_STAGES;
   uint64_t* tmem_empty = tmem_full + 2;
   uint64_t* rload = tmem_empty + 2;  // residual tile loads: 2 per epilogue warp
-  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(rload + 16);
+  uint64_t* pload = rload + 16;     // stream-K finisher: one partial prefetch per epilogue warp
+  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(pload + 8);
 
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
   const uint32_t rank = cluster_ctarank();
@@ -393,6 +394,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
       mbar_init(&tmem_empty[a], 16);  // 8 epilogue warps x 2 CTAs
     }
     for (int b = 0; b < 16; ++b) mbar_init(&rload[b], 1);
+    for (int b = 0; b < 8; ++b) mbar_init(&pload[b], 1);
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     tma_prefetch_desc(&tmA);
     tma_prefetch_desc(&tmW);
@@ -587,6 +589,19 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
           ok2 = __shfl_sync(0xffffffffu, ok2, 0);
           if (!ok2) { failed = true; break; }
           __threadfence();
+          // The next contributor's partial (16 KB for this warp) into this warp's part of
+          // the operand ring, idle now: a head segment is the last of the cluster's range,
+          // so every MMA that read the ring has completed and no load follows. One bulk
+          // copy instead of a round trip per chunk below. Only for rows the chunk loop
+          // handles: that loop waits for the copy before the CTA can leave.
+          if (lane == 0 && row0 < M) {
+            fence_proxy_async_global();
+            mbar_expect_tx(&pload[we], 16384);
+            bulk_load_1d(smem + we * 16384,
+                         sk_part(sk.ws, c_lo + 1, tile, U, n_clusters, nk, (int)rank, we), 16384,
+                         &pload[we]);
+          }
+          __syncwarp();
           finish = true;
         }
       }
@@ -610,7 +625,12 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
 #pragma unroll
             for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(r[j]);
           } else {
-            // the contributors' partials summed in K order, this cluster's from TMEM
+            // the contributors' partials summed in K order, this cluster's from TMEM, the
+            // next one's from the copy in shared memory (waited for once, at chunk 0)
+            if (cc == 0) {
+              const bool pok = mbar_wait(&pload[we], 0, err);
+              if (!__all_sync(0xffffffffu, pok)) { failed = true; break; }
+            }
 #pragma unroll
             for (int j = 0; j < 32; ++j) v[j] = 0.f;
 #pragma unroll 1
@@ -623,6 +643,18 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
                 reg_fence32(r);
 #pragma unroll
                 for (int j = 0; j < 32; ++j) v[j] += __uint_as_float(r[j]);
+              } else if (cq == c_lo + 1) {  // shared memory: generic loads
+                const float4* src = reinterpret_cast<const float4*>(
+                                        reinterpret_cast<const float*>(smem + we * 16384) +
+                                        cc * 1024) + lane;
+#pragma unroll
+                for (int j4 = 0; j4 < 8; ++j4) {
+                  const float4 f = src[j4 * 32];
+                  v[4 * j4] += f.x;
+                  v[4 * j4 + 1] += f.y;
+                  v[4 * j4 + 2] += f.z;
+                  v[4 * j4 + 3] += f.w;
+                }
               } else {
                 const float4* src = reinterpret_cast<const float4*>(
                                         sk_part(sk.ws, cq, tile, U, n_clusters, nk, (int)rank, we) +
