@@ -26,6 +26,7 @@ import json
 import os
 import subprocess
 import sys
+import threading
 import time
 
 import numpy as np
@@ -82,6 +83,11 @@ VARIANTS = {
     "phi_star": "",
     "full50": "",
 }
+
+
+# variants whose value pass may run with the split schedule (see run_gb300)
+SPLIT_VARIANTS = ("base", "sde", "cfg")
+REFINE_SMS = 40
 
 
 def n_candidates(variant):
@@ -302,6 +308,18 @@ def run_gb300(args):
     t_setup = time.time()
     w = synth.make_weights(cfg)
     model = fb.Model(cfg, w)
+    # the split schedule: step k's refine on a small SM partition beside step k + 1's
+    # draft on the rest (green contexts); a second model instance serves the refine
+    split, split_note, model_r = None, None, None
+    if args.schedule != "seq" and args.variant in SPLIT_VARIANTS:
+        try:
+            split = fb.SmSplit(args.refine_sms)
+        except fb.FlashBonError as e:
+            if args.schedule == "split":
+                raise
+            split_note = f"sequential: no SM partition ({e})"
+    if split:
+        model_r = fb.Model(cfg.with_(max_n=2), w)
     del w
     stream = torch.cuda.Stream()
     model.set_stream(stream)
@@ -326,6 +344,50 @@ def run_gb300(args):
                   for _ in range(NC)]
         opts_d = fb.make_opts(keep_state=True)
     setup_s = time.time() - t_setup
+    if split:
+        s_ref, s_dr = split.streams
+        t_dr = torch.cuda.ExternalStream(s_dr)
+        zr2 = [torch.empty_like(z0[0]) for _ in range(2)]
+        pipe = {"k": 0}
+
+        def use_split():
+            model.set_stream(s_dr)
+            model.set_sm_budget(split.sms[1])
+            model_r.set_stream(s_ref)
+            model_r.set_sm_budget(split.sms[0])
+
+        def pipe_step(z_in, z_buf, zr_bufs, ctx_in, to_dev):
+            """Draft of a new pool (large part) while candidate 0 of the previous pool is
+            refined (small part, another host thread); both finished on return."""
+            k = pipe["k"]
+            err = []
+
+            def ref():
+                try:
+                    model_r.refine(zr_bufs[(k - 1) % 2], ctx_in, tail, opts=opts_r)
+                except BaseException as e:  # re-raised on the main thread
+                    err.append(e)
+            th = threading.Thread(target=ref) if k > 0 else None
+            if th:
+                th.start()
+            if to_dev:
+                with torch.cuda.stream(t_dr):
+                    z_buf.copy_(z_in)
+            else:
+                z_buf.copy_(z_in)
+            model.draft(z_buf, ctx_in, draft_sched, skip, proxy, opts=opts_d)
+            if to_dev:
+                with torch.cuda.stream(t_dr):
+                    zr_bufs[k % 2].copy_(z_buf[0])
+                t_dr.synchronize()
+            else:
+                zr_bufs[k % 2].copy_(z_buf[0])
+            if th:
+                th.join()
+            if err:
+                raise err[0]
+            pipe["k"] = k + 1
+        use_split()
 
     def dev_step(after=None):
         with torch.cuda.stream(stream):
@@ -345,25 +407,43 @@ def run_gb300(args):
         if states:
             model.state_wait()
 
+    def value_step():
+        if split:
+            pipe_step(z0, z, zr2, ctx, True)
+        else:
+            dev_step()
+    tstream = t_dr if split else stream
     for _ in range(args.warmup):
-        dev_step()
+        value_step()
     finish()
     torch.cuda.synchronize()
     model.reset_stats()
+    if model_r:
+        model_r.reset_stats()
     if pg:
         pg.barrier()
     torch.cuda.synchronize()
-    # timed pass 1 (the reported value): no per-kernel instrumentation
+    # timed pass 1 (the reported value): no per-kernel instrumentation. With the split
+    # schedule each timed step drafts a new pool and refines candidate 0 of the previous
+    # one (the pipeline was filled in the warm-up); every call has returned, so all of
+    # that work lies between the two events.
     ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     with ClockSampler(local) as clk:
-        ev0.record(stream)
+        ev0.record(tstream)
         for _ in range(args.steps):
-            dev_step()
+            value_step()
         finish()
-        ev1.record(stream)
+        ev1.record(tstream)
         torch.cuda.synchronize()
     ms = ev0.elapsed_time(ev1)
     launch_stats = model.stats()
+    if model_r:
+        for k, v in model_r.stats().items():
+            for f in ("launches", "flops", "bytes", "ms"):
+                launch_stats[k][f] += v[f]
+        # the roofline pass runs the steps one after the other on the whole GPU
+        model.set_stream(stream)
+        model.set_sm_budget(0)
     # timed pass 2 (roofline of the dominant kernel): the same K steps with CUDA events
     # around every tcgen05 GEMM launch on the library's stream. The events themselves
     # cost a few per cent of the step, which is why pass 1 runs without them.
@@ -401,11 +481,19 @@ def run_gb300(args):
     # end to end through the C-ABI with host buffers (pinned), copies inside the region
     zh = torch.empty(z0.shape, dtype=torch.float32, pin_memory=True)
     zrh = torch.empty(z0.shape[1:], dtype=torch.float32, pin_memory=True)
+    zrh2 = [torch.empty(z0.shape[1:], dtype=torch.float32, pin_memory=True) for _ in range(2)]
     ctxh = torch.from_numpy(ctx_h).pin_memory()
     z0h = z0.cpu()
-    model.set_stream(None)
+    if split:
+        use_split()
+        pipe["k"] = 0
+    else:
+        model.set_stream(None)
 
     def host_step():
+        if split:
+            pipe_step(z0h, zh, zrh2, ctxh, False)
+            return
         zh.copy_(z0h)
         model.draft(zh, ctxh, draft_sched, skip, proxy, opts=opts_d)
         if states:
@@ -444,7 +532,13 @@ def run_gb300(args):
     out = {"metric": METRIC, "value": value, "unit": "candidates/s", "n_gpus": ws,
            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_step,
            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
-           "data": "synthetic", "config": config_dict(cfg, args.variant),
+           "data": "synthetic",
+           "config": {**config_dict(cfg, args.variant),
+                      "schedule": (f"split: step k's refine of candidate 0 on {split.sms[0]} "
+                                   f"SMs beside step k+1's draft on {split.sms[1]} (SM "
+                                   "partitions); each timed step drafts a pool and refines "
+                                   "the previous pool's candidate 0"
+                                   if split else split_note or "sequential")},
            "roofline": {"bound": "tensor", "kernel": "gemm_tc (tcgen05/TMEM GEMM, all "
                         "projections)", "achieved": achieved, "peak": peak,
                         "unit": "TFLOP/s", "frac": (achieved / peak) if achieved else None,
@@ -454,8 +548,9 @@ def run_gb300(args):
                                         "of the FFN probes x this run's algorithmic bytes "
                                         "per GEMM launch (profiles/gemm_tc_ffn_wan13.md)",
                         "launches": g["launches"], "ms": g["ms"] / args.steps,
-                        "measured_in": "timed pass 2 (same steps, per-launch CUDA events on "
-                                       "the library stream)",
+                        "measured_in": "timed pass 2 (same steps, one after the other on "
+                                       "the whole GPU, per-launch CUDA events on the "
+                                       "library stream)",
                         "pass2_ms_per_step": ms_instrumented / args.steps,
                         "by_phase": {ph: {"launches": v["launches"],
                                           "achieved": (v["flops"] / (v["ms"] / 1e3) / 1e12
@@ -484,7 +579,12 @@ def run_gb300(args):
                       f"{(S_TOTAL - S_DRAFT) * cfg.depth} refine block evaluations"}
     if rank == 0:
         print(json.dumps(out))
+    model.set_stream(None)
     model.close()
+    if model_r:
+        model_r.close()
+    if split:
+        split.close()
     if pg:
         pg.destroy_process_group()
     return 0
@@ -542,7 +642,7 @@ def run_probe(args):
         base, D = qkv.data_ptr(), H * dh
         call = lambda: fb.fb_op_attention(m.handle, base, 3 * D, base + 2 * D, 3 * D,  # noqa
                                           base + 4 * D, 3 * D, o, D, n, P, P, P, H, dh,
-                                          1 if args.probe == "attn_mma" else 0)
+                                          1 if args.probe == "attn_mma" else 3)
     if args.probe == "gemm_shapes":
         return probe_gemm_shapes(m, rnd, args)
     if args.probe == "attn_shapes":
@@ -697,6 +797,11 @@ def main():
     ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
     ap.add_argument("--cpu-budget", type=float, default=15.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--schedule", choices=["auto", "seq", "split"], default="auto",
+                    help="auto: the split schedule (refine on a small SM partition beside "
+                         "the next draft) where the variant allows it and the driver offers "
+                         "SM partitions, else sequential")
+    ap.add_argument("--refine-sms", type=int, default=REFINE_SMS)
     ap.add_argument("--variant", choices=list(VARIANTS), default="base",
                     help="base: the draft-pool workload; cfg / sde: the same with guidance "
                          "or SDE steps")

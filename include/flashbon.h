@@ -82,6 +82,31 @@ fb_status fb_init_model(const fb_cfg* cfg, const float* weights_host, fb_model**
 void fb_free(fb_model* m);
 /* stream: a cudaStream_t (NULL = the model's own stream). */
 fb_status fb_set_stream(fb_model* m, void* stream);
+/* fb_set_sm_budget: the number of SMs the model's launches may occupy (0 = all of the
+ * device's). Persistent GEMM grids, the stream-K co-residency rule and the attention
+ * kernel's CTA size are sized to it. Set it to the SM count of a partition whose stream
+ * the model runs on (fb_sm_split_*): a GEMM that assumed more resident SM pairs than the
+ * partition holds would leave its stream-K finishers waiting until their time limit.
+ * FB_EINVAL outside [2, device SMs]. Waits for the model's stream first. */
+fb_status fb_set_sm_budget(fb_model* m, int n_sms);
+
+/* ---- SM partitions (an engineering entry point: the paper has no counterpart) ------
+ * The paper runs generation and verification on separate GPUs (Sec. 5). On one GPU, the
+ * draft pool (compute-bound, many waves) and the refinement of one candidate (a chain of
+ * one-wave launches) can run side by side on disjoint SM sets. fb_sm_split_create splits
+ * the current device's SMs into a group of n_sms (the driver may round the count to its
+ * granularity) and the rest, each with a green context and a non-blocking stream in it;
+ * kernels enqueued on a part's stream run only on that part's SMs, on the same device
+ * memory. fb_sm_split_info(part 0 = the n_sms group, 1 = the rest) returns the part's
+ * stream (a cudaStream_t; the split owns it) and its SM count, to pass to fb_set_stream
+ * and fb_set_sm_budget. fb_sm_split_free waits for both streams and releases them; the
+ * models that used them must be given other streams first. Errors: FB_EINVAL for n_sms
+ * outside [2, device SMs - 2], FB_ECUDA when the driver offers no green contexts or a
+ * call fails (nothing is left allocated). */
+typedef struct fb_sm_split fb_sm_split;
+fb_status fb_sm_split_create(int n_sms, fb_sm_split** out);
+fb_status fb_sm_split_info(const fb_sm_split* split, int part, void** stream, int* sms);
+void fb_sm_split_free(fb_sm_split* split);
 
 /* fb_encode_text: text projection of the prompt embedding x (§3) and, per block, the
  * cross-attention keys and values; they do not change across steps or candidates and

@@ -7,6 +7,7 @@
 // launch, a skipped block launches nothing. Cached contributions Delta_l are written by
 // the epilogue of the block's last GEMM into a ring of anchor slots; slots are assigned
 // on the host from the plan, so only contributions some later proxy reads are stored.
+#include <cuda.h>
 #include <cuda_runtime.h>
 
 #include <algorithm>
@@ -144,7 +145,8 @@ struct fb_model {
   fb_cfg c;
   int P, PD, gh, gw;
   size_t Mmax;
-  int num_sms;
+  int num_sms;      // SMs the model's launches may use (fb_set_sm_budget), <= dev_sms
+  int dev_sms = 0;  // the device's SMs
   cudaStream_t own = nullptr, st = nullptr;
   // weights
   void* wmat = nullptr;  // bf16 matrices
@@ -344,6 +346,7 @@ GemmArgs gemm_args(int M, int N, int K, const bf16* A, const bf16* W, const floa
 fb_status run_attn(fb_model* m, const AttnArgs& a0, int kind, int impl = 0) {
   AttnArgs a = a0;
   a.tc_variant = impl >= 2 ? impl - 1 : 0;
+  a.sms = m->num_sms;
   const double flops = 4.0 * a.batch * a.heads * (double)a.Lq * a.Lkv * a.head_dim;
   const double kvb = (a.kv_batch_rows ? a.batch : 1) * 2.0 * a.Lkv * a.heads * a.head_dim * 2;
   const double bytes = 2.0 * a.batch * a.Lq * (double)a.heads * a.head_dim * 2 + kvb;
@@ -1005,6 +1008,7 @@ fb_status fb_init_model(const fb_cfg* cfg, const float* weights_host, fb_model**
       (s = dalloc_t(m, &m->rope, (size_t)m->P * c.head_dim / 2)) ||
       (s = dalloc_t(m, &m->zbuf, zn)) || (s = dalloc_t(m, &m->derr, 1)))
     return bail(s);
+  m->dev_sms = m->num_sms;
   m->sk_clusters = m->num_sms / 2;
   if ((s = dalloc_t(m, &m->sk_ws, (size_t)m->sk_clusters * SK_WS_FLOATS_PER_CLUSTER)) ||
       (s = dalloc_t(m, &m->sk_ctr, (size_t)m->sk_clusters * SK_CTR_PER_CLUSTER)))
@@ -1057,6 +1061,16 @@ fb_status fb_set_stream(fb_model* m, void* stream) {
   CK(cudaStreamSynchronize(m->st));
   m->st = stream ? reinterpret_cast<cudaStream_t>(stream) : m->own;
   fb_stream_op_not_kernel();
+  return FB_OK;
+}
+
+fb_status fb_set_sm_budget(fb_model* m, int n_sms) {
+  if (!m) return fail(FB_EINVAL, "model is NULL");
+  if (n_sms == 0) n_sms = m->dev_sms;
+  if (n_sms < 2 || n_sms > m->dev_sms)
+    return fail(FB_EINVAL, "n_sms=%d outside [2, %d]", n_sms, m->dev_sms);
+  CK(cudaStreamSynchronize(m->st));
+  m->num_sms = n_sms;
   return FB_OK;
 }
 
@@ -1385,6 +1399,114 @@ fb_status fb_gemm_streamk_noalloc(void* stream, int M, int N, int K, const void*
 fb_status fb_set_op_repeat(fb_model* m, int n) {
   if (!m || n < 1) return fail(FB_EINVAL, "model is NULL or n < 1");
   m->op_repeat = n;
+  return FB_OK;
+}
+
+}  // extern "C"
+
+// ---- SM partitions (green contexts) ------------------------------------------------
+// The driver's green-context calls are looked up at run time (as cuTensorMapEncodeTiled
+// is), so the library needs no link against the driver library.
+struct fb_sm_split {
+  CUgreenCtx g[2] = {nullptr, nullptr};
+  CUstream s[2] = {nullptr, nullptr};
+  int sms[2] = {0, 0};
+};
+
+namespace {
+template <typename F>
+bool drv_fn(const char* name, int version, F* out) {
+  void* p = nullptr;
+  cudaDriverEntryPointQueryResult q;
+  if (cudaGetDriverEntryPointByVersion(name, &p, version, cudaEnableDefault, &q) !=
+          cudaSuccess ||
+      q != cudaDriverEntryPointSuccess || !p) {
+    cudaGetLastError();
+    return false;
+  }
+  *out = reinterpret_cast<F>(p);
+  return true;
+}
+struct GreenFns {
+  decltype(&cuDeviceGetDevResource) get_res = nullptr;
+  decltype(&cuDevSmResourceSplitByCount) split = nullptr;
+  decltype(&cuDevResourceGenerateDesc) gen_desc = nullptr;
+  decltype(&cuGreenCtxCreate) create = nullptr;
+  decltype(&cuGreenCtxStreamCreate) stream_create = nullptr;
+  decltype(&cuGreenCtxDestroy) destroy = nullptr;
+  decltype(&cuStreamDestroy) stream_destroy = nullptr;
+  bool ok = false;
+};
+const GreenFns& green_fns() {
+  static const GreenFns f = [] {
+    GreenFns g;
+    g.ok = drv_fn("cuDeviceGetDevResource", 12040, &g.get_res) &&
+           drv_fn("cuDevSmResourceSplitByCount", 12040, &g.split) &&
+           drv_fn("cuDevResourceGenerateDesc", 12040, &g.gen_desc) &&
+           drv_fn("cuGreenCtxCreate", 12040, &g.create) &&
+           drv_fn("cuGreenCtxStreamCreate", 12050, &g.stream_create) &&
+           drv_fn("cuGreenCtxDestroy", 12040, &g.destroy) &&
+           drv_fn("cuStreamDestroy", 4000, &g.stream_destroy);
+    return g;
+  }();
+  return f;
+}
+}  // namespace
+
+extern "C" {
+
+void fb_sm_split_free(fb_sm_split* sp) {
+  if (!sp) return;
+  const GreenFns& f = green_fns();
+  for (int i = 0; i < 2; ++i) {
+    if (sp->s[i]) {
+      cudaStreamSynchronize(reinterpret_cast<cudaStream_t>(sp->s[i]));
+      if (f.ok) f.stream_destroy(sp->s[i]);
+    }
+    if (sp->g[i] && f.ok) f.destroy(sp->g[i]);
+  }
+  cudaGetLastError();
+  delete sp;
+}
+
+fb_status fb_sm_split_create(int n_sms, fb_sm_split** out) {
+  if (!out) return fail(FB_EINVAL, "out is NULL");
+  *out = nullptr;
+  const GreenFns& f = green_fns();
+  if (!f.ok) return fail(FB_ECUDA, "green contexts are not available from this driver");
+  int dev = 0;
+  CK(cudaGetDevice(&dev));
+  CK(cudaFree(nullptr));  // the device's primary context exists from here on
+  CUdevResource all;
+  if (f.get_res(static_cast<CUdevice>(dev), &all, CU_DEV_RESOURCE_TYPE_SM) != CUDA_SUCCESS)
+    return fail(FB_ECUDA, "cuDeviceGetDevResource failed");
+  if (n_sms < 2 || n_sms > (int)all.sm.smCount - 2)
+    return fail(FB_EINVAL, "n_sms=%d outside [2, %u]", n_sms, all.sm.smCount - 2);
+  CUdevResource parts[2];
+  unsigned n_groups = 1;
+  if (f.split(&parts[0], &n_groups, &all, &parts[1], 0, (unsigned)n_sms) != CUDA_SUCCESS ||
+      n_groups != 1)
+    return fail(FB_ECUDA, "cuDevSmResourceSplitByCount failed");
+  fb_sm_split* sp = new fb_sm_split;
+  for (int i = 0; i < 2; ++i) {
+    CUdevResourceDesc desc;
+    if (f.gen_desc(&desc, &parts[i], 1) != CUDA_SUCCESS ||
+        f.create(&sp->g[i], desc, static_cast<CUdevice>(dev), CU_GREEN_CTX_DEFAULT_STREAM) !=
+            CUDA_SUCCESS ||
+        f.stream_create(&sp->s[i], sp->g[i], CU_STREAM_NON_BLOCKING, 0) != CUDA_SUCCESS) {
+      fb_sm_split_free(sp);
+      return fail(FB_ECUDA, "green context %d creation failed", i);
+    }
+    sp->sms[i] = (int)parts[i].sm.smCount;
+  }
+  *out = sp;
+  return FB_OK;
+}
+
+fb_status fb_sm_split_info(const fb_sm_split* sp, int part, void** stream, int* sms) {
+  if (!sp || !stream || !sms || part < 0 || part > 1) return fail(FB_EINVAL, "bad argument");
+  *stream = reinterpret_cast<void*>(sp->s[part]);
+  *sms = sp->sms[part];
   return FB_OK;
 }
 

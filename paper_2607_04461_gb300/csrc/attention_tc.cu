@@ -665,9 +665,10 @@ cudaError_t attention_tc(const AttnArgs& a, int* err, cudaStream_t st) {
   if (!map_128x64(&mq, a.Q, a.batch * a.Lq, cols, a.ldq) ||
       !map_128x64(&mk, a.K, kv_rows, cols, a.ldk) || !map_128x64(&mv, a.V, kv_rows, cols, a.ldv))
     return cudaErrorInvalidValue;
-  int dev = 0, sms = 148;
-  if (cudaGetDevice(&dev) == cudaSuccess)
-    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  int dev = 0, sms = a.sms;
+  if (sms <= 0 && (cudaGetDevice(&dev) != cudaSuccess ||
+                   cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess))
+    sms = 148;
   Params p;
   p.Lq = a.Lq;
   p.Lkv = a.Lkv;
@@ -677,11 +678,14 @@ cudaError_t attention_tc(const AttnArgs& a, int* err, cudaStream_t st) {
   p.scale_log2 = 1.4426950408889634f / sqrtf(128.f);
   p.err = err;
   // 256-query CTAs share each K/V tile between two query tiles and overlap one tile's
-  // softmax with the other's MMAs; the 128-query kernel only where all of its CTAs fit
-  // in one wave (one CTA per SM), which then finishes sooner (e.g. 1 x 1560 queries x 12
-  // heads: 156 CTAs of 128 > 152 SMs, 256-query CTAs 18 % faster).
+  // softmax with the other's MMAs; one costs about 1.7 times a 128-query CTA in steady
+  // state (one CTA per SM either way). The choice compares waves: on 152 SMs, 1 x 1560
+  // queries x 12 heads is 2 waves of 128-query CTAs (156) or 1 of 256-query CTAs (84,
+  // 18 % faster); on a 40-SM partition it is 4 waves against 3 (1.7 x 3 > 4).
   const long ctas1 = (long)((a.Lq + TB - 1) / TB) * a.heads * a.batch;
-  const bool two = a.tc_variant == 2 || (a.tc_variant == 0 && ctas1 > sms);
+  const long ctas2 = (long)((a.Lq + 2 * TB - 1) / (2 * TB)) * a.heads * a.batch;
+  const long w1 = (ctas1 + sms - 1) / sms, w2 = (ctas2 + sms - 1) / sms;
+  const bool two = a.tc_variant == 2 || (a.tc_variant == 0 && 10 * w1 >= 17 * w2);
   if (two) {
     cudaError_t e = cudaFuncSetAttribute(attn_tc2_kernel,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM2_BYTES);

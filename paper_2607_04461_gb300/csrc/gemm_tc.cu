@@ -858,10 +858,11 @@ cudaError_t launch2(const GemmArgs& g, int* err, int num_sms, cudaStream_t st) {
   cudaError_t e = cudaFuncSetAttribute(gemm_tc2_kernel<KIND>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, C2_SMEM_BYTES);
   if (e != cudaSuccess) return e;
-  // as many clusters as can be resident at once (pairs must share a GPC)
-  static int max_clusters[4] = {0, 0, 0, 0};
-  int& mc = max_clusters[KIND];
-  if (mc == 0) {
+  // as many clusters as can be resident at once (pairs must share a GPC), and no more than
+  // the num_sms SMs this launch may use allow
+  static int occ_clusters[5] = {0, 0, 0, 0, 0};
+  int& occ = occ_clusters[KIND];
+  if (occ == 0) {
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(num_sms, 1, 1);
     cfg.blockDim = dim3(NUM_THREADS, 1, 1);
@@ -871,22 +872,28 @@ cudaError_t launch2(const GemmArgs& g, int* err, int num_sms, cudaStream_t st) {
       cudaGetLastError();
       n = num_sms / 2;
     }
-    mc = n < num_sms / 2 ? n : num_sms / 2;
+    occ = n;
   }
+  const int mc = occ < num_sms / 2 ? occ : num_sms / 2;
   const int tiles = ((g.M + 2 * BM - 1) / (2 * BM)) * (g.N / C2_BN);
   const int nk = g.K / BK;
   SkArgs sk{0, g.sk_ws, g.sk_ctr};
-  // Stream-K automatically only for a long K (>= 96 blocks) whose whole tiles leave pairs
-  // idle: there the spare pairs' share of the K loop outweighs writing and summing the
-  // partials of cut tiles (1560 x 1536 x 8960: 43.2 vs 47.9 us). With a short K, or with
-  // more tiles than pairs, the write-back and the waits cost more than the idle pairs of
-  // a short last wave save (1560 x 1536 x 1536: 22.9 vs 15.8 us).
+  // Stream-K automatically only for a few rounds of tiles (<= 4) whose last round leaves
+  // at least 24 K blocks' worth of work per pair idle ((rounds - tiles / pairs) * nk >=
+  // 24). There the idle pairs' share of the K loop outweighs writing and summing the
+  // partials of cut tiles. Measured on all 76 pairs: 1560 x 1536 x 8960 gains (43.2 vs
+  // 47.9 us); a short K (1560 x 1536 x 1536: 22.9 vs 15.8 us) and 1560 x 8960 x 1536
+  // (3.2 rounds: 41.4 vs 37.6 us) lose. With many rounds the contiguous unit ranges would
+  // also spread each round over far-apart tiles and lose L2 reuse. On a partition of 20
+  // pairs the 1560 x 1536 x 8960 shape's 42 tiles take 3 rounds, the last 90 % empty.
   const long long U = (long long)tiles * nk;
   const bool sk_ok = g.sk_ws && g.sk_ctr && mc <= g.sk_clusters && U >= 4LL * mc;
+  const int rounds = (tiles + mc - 1) / mc;
+  const bool sk_pays = rounds <= 4 && ((long long)rounds * mc - tiles) * nk >= 24LL * mc;
   if (g.sk_mode == 2) {
     if (!sk_ok) return cudaErrorInvalidValue;
     sk.on = 1;
-  } else if (g.sk_mode == 0 && sk_ok && nk >= 96 && tiles < mc) {
+  } else if (g.sk_mode == 0 && sk_ok && sk_pays) {
     sk.on = 1;
   }
   const int clusters = sk.on ? mc : (tiles < mc ? tiles : mc);

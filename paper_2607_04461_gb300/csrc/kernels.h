@@ -44,6 +44,7 @@ struct AttnArgs {
   int kv_batch_rows;       // row offset of batch b's K/V (0 = shared)
   int heads, head_dim;
   int tc_variant;          // tcgen05 kernel: 0 automatic, 1 128-query CTAs, 2 256-query CTAs
+  int sms;                 // SMs the launch may use (its choice of CTA size); 0: the device's
 };
 // mma.sync (warp-level) kernel: head_dim 64 or 128.
 cudaError_t attention(const AttnArgs& a, cudaStream_t st);

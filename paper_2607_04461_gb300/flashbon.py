@@ -53,7 +53,8 @@ EXPORTS = ["fb_weights_count", "fb_weights_entry", "fb_init_model", "fb_free", "
            "fb_last_error", "fb_set_timing", "fb_get_stats", "fb_reset_stats", "fb_kernel_name",
            "fb_op_gemm", "fb_op_attention", "fb_draft_ex", "fb_refine_ex", "fb_select_elo",
            "fb_set_op_repeat", "fb_gemm_streamk_noalloc", "fb_state_bytes", "fb_state_offload",
-           "fb_state_wait"]
+           "fb_state_wait", "fb_set_sm_budget", "fb_sm_split_create", "fb_sm_split_info",
+           "fb_sm_split_free"]
 
 PAIR_VERIFIER = ctypes.CFUNCTYPE(ctypes.c_int, ctypes.c_void_p, ctypes.c_int, ctypes.c_int,
                                  ctypes.POINTER(ctypes.c_int))
@@ -98,6 +99,10 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
         "fb_state_bytes": (I, [P, ctypes.POINTER(S)]),
         "fb_state_offload": (I, [P, I, I, ctypes.POINTER(P)]),
         "fb_state_wait": (I, [P]),
+        "fb_set_sm_budget": (I, [P, I]),
+        "fb_sm_split_create": (I, [I, ctypes.POINTER(P)]),
+        "fb_sm_split_info": (I, [P, I, ctypes.POINTER(P), ctypes.POINTER(I)]),
+        "fb_sm_split_free": (None, [P]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(L, name)
@@ -175,6 +180,39 @@ def fb_set_stream(model: int, stream) -> None:
     """stream: a torch.cuda.Stream, a raw cudaStream_t int, or None (model's own)."""
     s = getattr(stream, "cuda_stream", stream)
     _check(load_library().fb_set_stream(model, s))
+
+
+def fb_set_sm_budget(model: int, n_sms: int) -> None:
+    _check(load_library().fb_set_sm_budget(model, int(n_sms)))
+
+
+class SmSplit:
+    """Two disjoint SM partitions of the current device (green contexts), each with its
+    own stream: part 0 holds n_sms SMs, part 1 the rest. streams[i] is a raw
+    cudaStream_t handle (int) for Model.set_stream; sms[i] the part's SM count."""
+
+    def __init__(self, n_sms: int):
+        L = load_library()
+        h = ctypes.c_void_p()
+        _check(L.fb_sm_split_create(int(n_sms), ctypes.byref(h)))
+        self.handle = h.value
+        self.streams, self.sms = [], []
+        for part in (0, 1):
+            st, n = ctypes.c_void_p(), ctypes.c_int()
+            _check(L.fb_sm_split_info(self.handle, part, ctypes.byref(st), ctypes.byref(n)))
+            self.streams.append(st.value)
+            self.sms.append(n.value)
+
+    def close(self):
+        if self.handle:
+            load_library().fb_sm_split_free(self.handle)
+            self.handle = None
+
+    def __enter__(self):
+        return self
+
+    def __exit__(self, *exc):
+        self.close()
 
 
 def fb_encode_text(model: int, text_ctx) -> None:
@@ -349,6 +387,9 @@ class Model:
 
     def set_stream(self, stream):
         fb_set_stream(self.handle, stream)
+
+    def set_sm_budget(self, n_sms):
+        fb_set_sm_budget(self.handle, n_sms)
 
     def encode_text(self, ctx):
         fb_encode_text(self.handle, ctx)

@@ -551,3 +551,69 @@ def test_state_errors(small4):
         m.refine(z[0].clone(), ctx, sched,
                  opts=fb.make_opts(2.0, ctx, state=buf, warm_steps=1))
     assert e.value.status == fb.FB_EINVAL
+
+
+# ---- SM partitions: a model confined to part of the GPU ----------------------------
+
+def test_sm_split_and_budget_reproduce_the_whole_gpu_run():
+    """A draft on a 40-SM partition (green context) with the matching SM budget gives the
+    same latents, bit for bit, as on the whole GPU: the kernels' choices are the same at
+    this size and each output element's arithmetic does not depend on the grid."""
+    cfg = synth.SMALL
+    w = synth.make_weights(cfg, bf16=True, norm_std=0.2)
+    z = synth.make_latents(cfg, cfg.max_n)
+    ctx = synth.make_text(cfg)
+    sched = synth.make_schedule(4)
+    skip, proxy = synth.random_plan(4, cfg.depth, 1 / 3, 0.5, seed=3)
+    with fb.Model(cfg, w) as m:
+        whole = cuda(z)
+        m.draft(whole, ctx, sched, skip, proxy)
+        with fb.SmSplit(40) as sp:
+            assert sp.sms[0] >= 2 and sp.sms[1] >= 2
+            assert sp.sms[0] + sp.sms[1] == torch.cuda.get_device_properties(0).multi_processor_count
+            m.set_stream(sp.streams[0])
+            m.set_sm_budget(sp.sms[0])
+            part = cuda(z)
+            m.draft(part, ctx, sched, skip, proxy)
+            m.set_stream(None)
+            m.set_sm_budget(0)
+        assert torch.equal(part, whole)
+
+
+def test_stream_k_on_a_partition():
+    """On 20 SM pairs the 1560 x 1536 x 8960 GEMM's 42 tiles take 3 rounds, so the
+    automatic choice is the stream-K split; every contributor must be resident inside the
+    partition. Bit-identical to the forced split, within fp32 summation order of whole
+    tiles, and right against the oracle."""
+    M, N, K = 1560, 1536, 8960
+    g = torch.Generator().manual_seed(91)
+    A = (torch.randn(M, K, generator=g)).to(torch.bfloat16).cuda()
+    W = (torch.randn(N, K, generator=g) * K ** -0.5).to(torch.bfloat16).cuda()
+    resid = torch.randn(M, N, generator=g).cuda()
+    with fb.Model(synth.TINY, synth.make_weights(synth.TINY)) as m, fb.SmSplit(40) as sp:
+        m.set_stream(sp.streams[0])
+        m.set_sm_budget(sp.sms[0])
+        outs = []
+        for impl in (0, 4, 3):
+            out = torch.empty(M, N, device="cuda")
+            fb.fb_op_gemm(m.handle, M, N, K, A, W, None, 2, out, resid, None, None, None, impl)
+            outs.append(out)
+        torch.cuda.synchronize()
+        m.set_stream(None)
+    assert torch.equal(outs[0], outs[1])
+    assert rel_max(outs[0].cpu().double().numpy(), outs[2].cpu().double().numpy()) <= 1e-5
+    want = resid.cpu().double().numpy() + O.linear(A.float().cpu().double().numpy(),
+                                                   W.float().cpu().double().numpy())
+    assert rel_max(outs[0].cpu().double().numpy(), want) <= 1e-4
+
+
+def test_sm_budget_and_split_reject_bad_sizes():
+    with fb.Model(synth.TINY, synth.make_weights(synth.TINY)) as m:
+        for n in (1, 100000):
+            with pytest.raises(fb.FlashBonError) as e:
+                m.set_sm_budget(n)
+            assert e.value.status == fb.FB_EINVAL
+    for n in (1, 100000):
+        with pytest.raises(fb.FlashBonError) as e:
+            fb.SmSplit(n)
+        assert e.value.status == fb.FB_EINVAL
