@@ -880,16 +880,21 @@ cudaError_t launch2(const GemmArgs& g, int* err, int num_sms, cudaStream_t st) {
   SkArgs sk{0, g.sk_ws, g.sk_ctr};
   // Stream-K automatically only for a few rounds of tiles (<= 4) whose last round leaves
   // at least 24 K blocks' worth of work per pair idle ((rounds - tiles / pairs) * nk >=
-  // 24). There the idle pairs' share of the K loop outweighs writing and summing the
-  // partials of cut tiles. Measured on all 76 pairs: 1560 x 1536 x 8960 gains (43.2 vs
-  // 47.9 us); a short K (1560 x 1536 x 1536: 22.9 vs 15.8 us) and 1560 x 8960 x 1536
-  // (3.2 rounds: 41.4 vs 37.6 us) lose. With many rounds the contiguous unit ranges would
-  // also spread each round over far-apart tiles and lose L2 reuse. On a partition of 20
-  // pairs the 1560 x 1536 x 8960 shape's 42 tiles take 3 rounds, the last 90 % empty.
+  // 24), with A and W together within half of L2. There the idle pairs' share of the K
+  // loop outweighs writing and summing the partials of cut tiles. Measured on all 76
+  // pairs: 1560 x 1536 x 8960 gains (43.2 vs 47.9 us); a short K (1560 x 1536 x 1536:
+  // 22.9 vs 15.8 us) and 1560 x 8960 x 1536 (3.2 rounds: 41.4 vs 37.6 us) lose. The
+  // contiguous unit ranges spread each round over far-apart tiles, so operands larger
+  // than L2 are read several times: 8192 x 1536 x 8960 (2.5 rounds, A 147 MB) took 203
+  // us and 1.07 GB of DRAM reads against 156 us and 0.34 GB over whole tiles. On a
+  // partition of 20 pairs the 1560 x 1536 x 8960 shape's 42 tiles take 3 rounds, the
+  // last 90 % empty.
   const long long U = (long long)tiles * nk;
   const bool sk_ok = g.sk_ws && g.sk_ctr && mc <= g.sk_clusters && U >= 4LL * mc;
   const int rounds = (tiles + mc - 1) / mc;
-  const bool sk_pays = rounds <= 4 && ((long long)rounds * mc - tiles) * nk >= 24LL * mc;
+  const double operand_bytes = 2.0 * ((double)g.M + g.N) * g.K;
+  const bool sk_pays = rounds <= 4 && ((long long)rounds * mc - tiles) * nk >= 24LL * mc &&
+                       operand_bytes <= 64.0 * 1024 * 1024;
   if (g.sk_mode == 2) {
     if (!sk_ok) return cudaErrorInvalidValue;
     sk.on = 1;

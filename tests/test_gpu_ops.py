@@ -93,6 +93,7 @@ def test_gemm_stream_k_is_deterministic_and_matches_whole_tiles(model, M, N, K):
     (640, 1536, 8960, 4),    # 18 tiles, 140 K blocks: stream-K
     (1560, 1536, 1536, 3),   # 24 K blocks: whole tiles
     (49920, 1536, 8960, 3),  # more tiles than SM pairs: whole tiles
+    (8192, 1536, 8960, 3),   # 2.5 rounds but A and W (166 MB) larger than half of L2
 ])
 def test_gemm_automatic_stream_k_choice(model, M, N, K, twin):
     """impl 0 takes the stream-K split only for a long K under one wave of pair tiles: its
