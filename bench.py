@@ -413,7 +413,9 @@ def run_gb300(args):
         else:
             dev_step()
     tstream = t_dr if split else stream
-    for _ in range(args.warmup):
+    # at least one untimed step with the split schedule: it fills the pipeline, so that
+    # every timed step holds a draft and a refine
+    for _ in range(max(args.warmup, 1 if split else 0)):
         value_step()
     finish()
     torch.cuda.synchronize()

@@ -19,6 +19,8 @@
 // Every mbarrier wait is bounded (mbar_wait): on timeout the kernel records the error,
 // stops issuing work, waits (bounded) for its own TMA loads, frees TMEM and returns.
 #include <cudaTypedefs.h>
+
+#include <atomic>
 #include <string.h>
 
 #include "kernels.h"
@@ -769,15 +771,18 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
 }
 
 PFN_cuTensorMapEncodeTiled_v12000 get_encode() {
-  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
-  if (!fn) {
+  // looked up once; a function-local static is initialised thread-safely (the bench
+  // drives two models from two host threads)
+  static const PFN_cuTensorMapEncodeTiled_v12000 fn = [] {
     cudaDriverEntryPointQueryResult q;
     void* p = nullptr;
     if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
                                          &q) == cudaSuccess &&
         q == cudaDriverEntryPointSuccess)
-      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
-  }
+      return reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+    cudaGetLastError();
+    return static_cast<PFN_cuTensorMapEncodeTiled_v12000>(nullptr);
+  }();
   return fn;
 }
 
@@ -860,8 +865,8 @@ cudaError_t launch2(const GemmArgs& g, int* err, int num_sms, cudaStream_t st) {
   if (e != cudaSuccess) return e;
   // as many clusters as can be resident at once (pairs must share a GPC), and no more than
   // the num_sms SMs this launch may use allow
-  static int occ_clusters[5] = {0, 0, 0, 0, 0};
-  int& occ = occ_clusters[KIND];
+  static std::atomic<int> occ_clusters[4];  // zero until a launch has asked (any thread)
+  int occ = occ_clusters[KIND].load(std::memory_order_relaxed);
   if (occ == 0) {
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(num_sms, 1, 1);
@@ -873,6 +878,7 @@ cudaError_t launch2(const GemmArgs& g, int* err, int num_sms, cudaStream_t st) {
       n = num_sms / 2;
     }
     occ = n;
+    occ_clusters[KIND].store(n, std::memory_order_relaxed);
   }
   const int mc = occ < num_sms / 2 ? occ : num_sms / 2;
   const int tiles = ((g.M + 2 * BM - 1) / (2 * BM)) * (g.N / C2_BN);
