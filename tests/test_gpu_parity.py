@@ -333,6 +333,29 @@ def test_wide_two_step_draft(wide):
     check_latents(a.cpu().numpy()[0], want[0], z[0], label=f"{name} 2 steps")
 
 
+def test_wan13_refine_on_a_partition_matches_the_whole_gpu(wan13_pool):
+    """The refine as the bench runs it: one candidate on a 40-SM partition, where the FFN
+    down-projection takes the stream-K split and attention the 128-query kernel. Against
+    the same refine on the whole GPU (whose draft path the oracle checks above) only fp32
+    summation orders differ."""
+    cfg, w, m = wan13_pool
+    z = synth.make_latents(cfg, 1)[0]
+    ctx = synth.make_text(cfg)
+    sched = synth.make_schedule(50)[10:13]          # two steps from t_10
+    whole = cuda(z)
+    m.refine(whole, ctx, sched)
+    with fb.SmSplit(40) as sp:
+        m.set_stream(sp.streams[0])
+        m.set_sm_budget(sp.sms[0])
+        part = cuda(z)
+        m.refine(part, ctx, sched)
+        m.set_stream(None)
+        m.set_sm_budget(0)
+    assert torch.isfinite(part).all()
+    e = rel_max(part.cpu().double().numpy() - z, whole.cpu().double().numpy() - z)
+    assert e <= 1e-2, f"displacement {e:.3e}"
+
+
 # ---- NEXT rows: classifier-free guidance and SDE steps -------------------------------
 
 @pytest.fixture(scope="module")
