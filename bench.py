@@ -54,10 +54,17 @@ def workload():
 # candidate 0.
 PHI_STAR = dict(S=50, S_prime=49, n_skip=3, l_start=22, l_end=23, f_full=5, order=2)
 PHI_N = 8
+# The 14B draft pool: N = 8, the first 10 of 50 steps, a seeded quarter of the blocks
+# skipped per step, every remaining block proxied on odd steps; the drafts only.
+W14_N = 8
 
 
 def plan_for(variant):
     """(cfg, schedule, skip, proxy, draft steps) of a bench variant."""
+    if variant == "wan14":  # the 14B draft pool; the schedule ends with the draft
+        cfg = synth.WAN14.with_(max_n=W14_N)
+        skip, proxy = synth.random_plan(S_DRAFT, cfg.depth, 0.25, 1.0, seed=PLAN_SEED)
+        return cfg, synth.make_schedule(S_TOTAL)[: S_DRAFT + 1], skip, proxy, S_DRAFT
     if variant == "full50":  # the same N and schedule sampled without any acceleration
         cfg = synth.WAN13.with_(max_n=PHI_N)
         skip, proxy = synth.empty_plan(PHI_STAR["S"], cfg.depth)
@@ -82,6 +89,7 @@ VARIANTS = {
                "the next draft",
     "phi_star": "",
     "full50": "",
+    "wan14": "",
 }
 
 
@@ -93,7 +101,8 @@ REFINE_SMS = 40
 
 
 def n_candidates(variant):
-    return {"cfg": N_CAND // 2, "phi_star": PHI_N, "full50": PHI_N}.get(variant, N_CAND)
+    return {"cfg": N_CAND // 2, "phi_star": PHI_N, "full50": PHI_N,
+            "wan14": W14_N}.get(variant, N_CAND)
 
 
 def config_dict(cfg, variant="base"):
@@ -108,6 +117,14 @@ def config_dict(cfg, variant="base"):
                 "n_candidates": n, "tokens": cfg.tokens, "dim": cfg.dim, "depth": cfg.depth,
                 "draft_steps": ph["S_prime"], "refine_steps": ph["S"] - ph["S_prime"],
                 "l2": "inputs larger than L2 (2.6 GB weights), no flush"}
+    if variant == "wan14":
+        return {"workload": f"wan2.1-14B draft pool: N={n}, 480x832 (1560 tokens), 10 of 50 "
+                            "steps, 1/4 of the blocks skipped per step, on odd steps every "
+                            "remaining block the previous step computed proxied; the drafts "
+                            "only (no refine); random-init weights drawn on the GPU",
+                "n_candidates": n, "tokens": cfg.tokens, "dim": cfg.dim, "depth": cfg.depth,
+                "draft_steps": S_DRAFT, "refine_steps": 0,
+                "l2": "inputs larger than L2 (28 GB weights), no flush"}
     if variant == "full50":
         return {"workload": f"wan2.1-1.3B: N={n}, 480x832 (1560 tokens), all 50 steps, every "
                             "block computed (sampling without the paper's acceleration)",
@@ -308,7 +325,7 @@ def run_gb300(args):
     cfg, sched, skip, proxy, s_draft = plan_for(args.variant)
     NC = n_candidates(args.variant)
     t_setup = time.time()
-    w = synth.make_weights(cfg)
+    w = synth.make_weights_device(cfg) if args.variant == "wan14" else synth.make_weights(cfg)
     model = fb.Model(cfg, w)
     # the split schedule: step k's refine on a small SM partition beside step k + 1's
     # draft on the rest (green contexts); a second model instance serves the refine
@@ -323,6 +340,7 @@ def run_gb300(args):
     if split:
         model_r = fb.Model(cfg.with_(max_n=2), w)
     del w
+    torch.cuda.empty_cache()  # the generator's buffers (56 GB for the 14B weights)
     stream = torch.cuda.Stream()
     model.set_stream(stream)
     # each rank drafts its own candidates (weak scaling, no collective on the path)
@@ -532,7 +550,7 @@ def run_gb300(args):
     launches = sum(s["launches"] for s in launch_stats.values())
     passes = 2 if args.variant == "cfg" else 1
     algo_flops = passes * (NC * computed_blocks(skip, proxy) * block_flops(cfg) +
-                           (S_TOTAL - s_draft) * cfg.depth * block_flops(cfg))
+                           (len(tail) - 1) * cfg.depth * block_flops(cfg))
     out = {"metric": METRIC, "value": value, "unit": "candidates/s", "n_gpus": ws,
            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_step,
            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",

@@ -74,10 +74,12 @@ fb_status fb_weights_entry(const fb_cfg* cfg, int idx, const char** name,
                            size_t* offset, size_t* numel);
 
 /* ---- model --------------------------------------------------------------------
- * fb_init_model: validates cfg, copies the packed fp32 host weights to the device as
- * bf16 (matrices) and fp32 (biases, norm scales, modulation tables), allocates the
- * activation buffers for max_n candidates. *out is NULL on failure. The denoiser is
- * the black-box f_theta of §3 (a DiT); the block follows Eq. 7. */
+ * fb_init_model: validates cfg, copies the packed fp32 weights to the device as bf16
+ * (matrices) and fp32 (biases, norm scales, modulation tables), allocates the
+ * activation buffers for max_n candidates. weights_host may be host memory or this
+ * device's memory (read through unified addressing; the caller keeps it). *out is NULL
+ * on failure. The denoiser is the black-box f_theta of §3 (a DiT); the block follows
+ * Eq. 7. */
 fb_status fb_init_model(const fb_cfg* cfg, const float* weights_host, fb_model** out);
 void fb_free(fb_model* m);
 /* stream: a cudaStream_t (NULL = the model's own stream). */

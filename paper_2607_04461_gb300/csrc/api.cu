@@ -943,7 +943,7 @@ fb_status fb_init_model(const fb_cfg* cfg, const float* weights_host, fb_model**
       dst = reinterpret_cast<bf16*>(m->wmat) + mo;
       mo += e.numel;
       fb_stream_op_not_kernel();
-      if (cudaMemcpyAsync(stage, src, e.numel * 4, cudaMemcpyHostToDevice, m->st) != cudaSuccess ||
+      if (cudaMemcpyAsync(stage, src, e.numel * 4, cudaMemcpyDefault, m->st) != cudaSuccess ||
           f32_to_bf16(stage, reinterpret_cast<bf16*>(dst), e.numel, m->st) != cudaSuccess ||
           cudaStreamSynchronize(m->st) != cudaSuccess)
         return bail(fail(FB_ECUDA, "weight upload failed (%s)", e.name.c_str()));
@@ -956,7 +956,7 @@ fb_status fb_init_model(const fb_cfg* cfg, const float* weights_host, fb_model**
         dst = reinterpret_cast<float*>(m->wvec) + vo;
         vo += e.numel;
       }
-      if (cudaMemcpyAsync(dst, src, e.numel * 4, cudaMemcpyHostToDevice, m->st) != cudaSuccess)
+      if (cudaMemcpyAsync(dst, src, e.numel * 4, cudaMemcpyDefault, m->st) != cudaSuccess)
         return bail(fail(FB_ECUDA, "weight upload failed (%s)", e.name.c_str()));
     }
     ptr[e.name] = dst;

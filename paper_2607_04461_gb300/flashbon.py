@@ -142,12 +142,27 @@ def make_cfg(cfg: synth.Cfg) -> fb_cfg:
     return c
 
 
-def pack_weights(cfg: synth.Cfg, weights: dict) -> np.ndarray:
-    """Packs named weights into the library's fp32 layout (fb_weights_entry order)."""
+def pack_weights(cfg: synth.Cfg, weights: dict):
+    """Packs named weights into the library's fp32 layout (fb_weights_entry order): a
+    numpy buffer, or a CUDA tensor when the weights are CUDA tensors."""
     L = load_library()
     c = make_cfg(cfg)
     count, total = ctypes.c_int(), ctypes.c_size_t()
     _check(L.fb_weights_count(ctypes.byref(c), ctypes.byref(count), ctypes.byref(total)))
+    first = next(iter(weights.values()))
+    if getattr(first, "is_cuda", False):
+        import torch
+        buf = torch.empty(total.value, dtype=torch.float32, device=first.device)
+        name, off, numel = ctypes.c_char_p(), ctypes.c_size_t(), ctypes.c_size_t()
+        for i in range(count.value):
+            _check(L.fb_weights_entry(ctypes.byref(c), i, ctypes.byref(name),
+                                      ctypes.byref(off), ctypes.byref(numel)))
+            w = weights[name.value.decode()].reshape(-1)
+            if w.numel() != numel.value:
+                raise ValueError(f"{name.value.decode()}: {w.numel()} elements, "
+                                 f"expected {numel.value}")
+            buf[off.value: off.value + numel.value].copy_(w)
+        return buf
     buf = np.empty(total.value, np.float32)
     name, off, numel = ctypes.c_char_p(), ctypes.c_size_t(), ctypes.c_size_t()
     for i in range(count.value):
@@ -165,7 +180,8 @@ def pack_weights(cfg: synth.Cfg, weights: dict) -> np.ndarray:
 def fb_init_model(cfg: synth.Cfg, weights) -> int:
     """weights: dict of named arrays, or an already packed fp32 buffer."""
     L = load_library()
-    packed = weights if isinstance(weights, np.ndarray) else pack_weights(cfg, weights)
+    packed = weights if isinstance(weights, np.ndarray) or hasattr(weights, "data_ptr") \
+        else pack_weights(cfg, weights)
     c = make_cfg(cfg)
     h = ctypes.c_void_p()
     _check(L.fb_init_model(ctypes.byref(c), _ptr(packed, np.float32), ctypes.byref(h)))

@@ -144,6 +144,21 @@ def make_weights(cfg: Cfg, seed: int = 0, std: float = 0.02, norm_std: float = 0
     return out
 
 
+def make_weights_device(cfg: Cfg, seed: int = 0, std: float = 0.02,
+                        norm_std: float = 0.02) -> dict:
+    """make_weights' distributions drawn on the current CUDA device (torch, one seeded
+    stream per tensor, values rounded to bf16): random-init weights for shapes whose
+    host generation takes minutes (the 14B model). Not the host generator's numbers."""
+    import torch
+    out = {}
+    for idx, (name, shape, kind) in enumerate(weight_specs(cfg)):
+        g = torch.Generator(device="cuda").manual_seed(seed * 1_000_003 + idx)
+        x = torch.randn(shape, generator=g, device="cuda", dtype=torch.float32)
+        x = 1.0 + norm_std * x if kind == "norm" else std * x
+        out[name] = x.to(torch.bfloat16).to(torch.float32)
+    return out
+
+
 def make_latents(cfg: Cfg, n: int, seed_base: int = 1000, first: int = 0) -> np.ndarray:
     """z_T for candidates first..first+n-1; candidate j is N(0, I) from seed seed_base + j."""
     z = np.empty((n, cfg.latent_c, cfg.latent_h, cfg.latent_w), dtype=np.float32)

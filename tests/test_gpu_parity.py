@@ -356,6 +356,24 @@ def test_wan13_refine_on_a_partition_matches_the_whole_gpu(wan13_pool):
     assert e <= 1e-2, f"displacement {e:.3e}"
 
 
+def test_model_from_device_weights_equals_host_weights():
+    """fb_init_model reads device-resident weights as it reads host ones."""
+    cfg = synth.SMALL
+    wd = synth.make_weights_device(cfg, seed=3)
+    wh = {k: v.cpu().numpy() for k, v in wd.items()}
+    z = synth.make_latents(cfg, 2)
+    ctx = synth.make_text(cfg)
+    sched = synth.make_schedule(3)
+    skip, proxy = synth.empty_plan(3, cfg.depth)
+    outs = []
+    for w in (wd, wh):
+        with fb.Model(cfg, w) as m:
+            a = cuda(z)
+            m.draft(a, ctx, sched, skip, proxy)
+            outs.append(a)
+    assert torch.equal(outs[0], outs[1])
+
+
 # ---- NEXT rows: classifier-free guidance and SDE steps -------------------------------
 
 @pytest.fixture(scope="module")
