@@ -26,7 +26,6 @@ import json
 import os
 import subprocess
 import sys
-import threading
 import time
 
 import numpy as np
@@ -378,34 +377,23 @@ def run_gb300(args):
 
         def pipe_step(z_in, z_buf, zr_bufs, ctx_in, to_dev):
             """Draft of a new pool (large part) while candidate 0 of the previous pool is
-            refined (small part, another host thread); both finished on return."""
+            refined (small part) on a worker thread of the library
+            (fb_pipeline_step); both finished on return."""
             k = pipe["k"]
-            err = []
-
-            def ref():
-                try:
-                    model_r.refine(zr_bufs[(k - 1) % 2], ctx_in, tail, opts=opts_r)
-                except BaseException as e:  # re-raised on the main thread
-                    err.append(e)
-            th = threading.Thread(target=ref) if k > 0 else None
-            if th:
-                th.start()
-            if to_dev:
+            if to_dev:  # on the drafter's stream, ahead of its draft
                 with torch.cuda.stream(t_dr):
                     z_buf.copy_(z_in)
             else:
                 z_buf.copy_(z_in)
-            model.draft(z_buf, ctx_in, draft_sched, skip, proxy, opts=opts_d)
+            fb.fb_pipeline_step(model.handle, z_buf, z_buf.shape[0], ctx_in, draft_sched, skip,
+                                proxy, model_r.handle if k > 0 else None,
+                                zr_bufs[(k - 1) % 2] if k > 0 else None, tail, opts_d, opts_r)
             if to_dev:
                 with torch.cuda.stream(t_dr):
                     zr_bufs[k % 2].copy_(z_buf[0])
                 t_dr.synchronize()
             else:
                 zr_bufs[k % 2].copy_(z_buf[0])
-            if th:
-                th.join()
-            if err:
-                raise err[0]
             pipe["k"] = k + 1
         use_split()
 

@@ -187,6 +187,23 @@ fb_status fb_draft_ex(fb_model* m, float* latents, int n, const float* text_ctx,
 fb_status fb_refine_ex(fb_model* m, float* latent, const float* text_ctx,
                        const float* full_schedule, int n_steps, const fb_sampler_opts* opts);
 
+/* fb_pipeline_step: one step of a draft/refine pipeline in one call (§4.2 Stages 1 and
+ * 3): refine_latent, the selected candidate of the previous pool, is refined with
+ * `refiner` (as fb_refine_ex) on a worker thread while `drafter` drafts `latents` (as
+ * fb_draft_ex) on the calling thread; the call returns when both are done. The two
+ * models should run on the two parts of an fb_sm_split (fb_set_stream and
+ * fb_set_sm_budget on each). refine_latent NULL: the draft alone (the first step).
+ * The refine must not read `latents`: copy the selected candidate out before the next
+ * step. Errors: FB_EINVAL for a NULL drafter, or a refine without a model of its own;
+ * otherwise the draft's status if it failed, else the refine's, with its message
+ * (prefixed "draft: " or "refine: ") in fb_last_error on the calling thread. */
+fb_status fb_pipeline_step(fb_model* drafter, float* latents, int n, const float* text_ctx,
+                           const float* draft_schedule, int n_draft_steps,
+                           const uint8_t* skip_mask, const int32_t* proxy_plan,
+                           const fb_sampler_opts* draft_opts, fb_model* refiner,
+                           float* refine_latent, const float* refine_schedule,
+                           int n_refine_steps, const fb_sampler_opts* refine_opts);
+
 /* ---- cached-state offload (§4.2 Stage 3; §8 NEXT row 4) -----------------------------
  * The paper moves the cached tensors to host memory during drafting and brings only the
  * selected candidate back for refinement; the copies are part of the wall-clock.

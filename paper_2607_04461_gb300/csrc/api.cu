@@ -18,6 +18,7 @@
 #include <cstring>
 #include <map>
 #include <mutex>
+#include <thread>
 #include <string>
 #include <vector>
 
@@ -1403,6 +1404,39 @@ fb_status fb_set_op_repeat(fb_model* m, int n) {
 }
 
 }  // extern "C"
+
+// ---- draft / refine pipeline step -------------------------------------------------
+extern "C" fb_status fb_pipeline_step(fb_model* drafter, float* latents, int n,
+                                      const float* text_ctx, const float* draft_schedule,
+                                      int n_draft_steps, const uint8_t* skip_mask,
+                                      const int32_t* proxy_plan,
+                                      const fb_sampler_opts* draft_opts, fb_model* refiner,
+                                      float* refine_latent, const float* refine_schedule,
+                                      int n_refine_steps,
+                                      const fb_sampler_opts* refine_opts) {
+  if (!drafter) return fail(FB_EINVAL, "drafter is NULL");
+  if (refine_latent && (!refiner || refiner == drafter))
+    return fail(FB_EINVAL, "the refine needs its own model");
+  // the refine on a worker thread (its own model and stream), the draft on this one;
+  // the worker's status and message come back to this thread (errors are per thread)
+  fb_status rs = FB_OK;
+  std::string rmsg;
+  std::thread worker;
+  if (refine_latent) {
+    worker = std::thread([&] {
+      rs = fb_refine_ex(refiner, refine_latent, text_ctx, refine_schedule, n_refine_steps,
+                        refine_opts);
+      if (rs != FB_OK) rmsg = g_last_error;
+    });
+  }
+  const fb_status ds = fb_draft_ex(drafter, latents, n, text_ctx, draft_schedule,
+                                   n_draft_steps, skip_mask, proxy_plan, draft_opts);
+  const std::string dmsg = ds != FB_OK ? g_last_error : std::string();
+  if (worker.joinable()) worker.join();
+  if (ds != FB_OK) return fail(ds, "draft: %s", dmsg.c_str());
+  if (rs != FB_OK) return fail(rs, "refine: %s", rmsg.c_str());
+  return FB_OK;
+}
 
 // ---- SM partitions (green contexts) ------------------------------------------------
 // The driver's green-context calls are looked up at run time (as cuTensorMapEncodeTiled

@@ -54,7 +54,7 @@ EXPORTS = ["fb_weights_count", "fb_weights_entry", "fb_init_model", "fb_free", "
            "fb_op_gemm", "fb_op_attention", "fb_draft_ex", "fb_refine_ex", "fb_select_elo",
            "fb_set_op_repeat", "fb_gemm_streamk_noalloc", "fb_state_bytes", "fb_state_offload",
            "fb_state_wait", "fb_set_sm_budget", "fb_sm_split_create", "fb_sm_split_info",
-           "fb_sm_split_free"]
+           "fb_sm_split_free", "fb_pipeline_step"]
 
 PAIR_VERIFIER = ctypes.CFUNCTYPE(ctypes.c_int, ctypes.c_void_p, ctypes.c_int, ctypes.c_int,
                                  ctypes.POINTER(ctypes.c_int))
@@ -103,6 +103,8 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
         "fb_sm_split_create": (I, [I, ctypes.POINTER(P)]),
         "fb_sm_split_info": (I, [P, I, ctypes.POINTER(P), ctypes.POINTER(I)]),
         "fb_sm_split_free": (None, [P]),
+        "fb_pipeline_step": (I, [P, P, I, P, P, I, P, P, ctypes.POINTER(fb_sampler_opts),
+                                 P, P, P, I, ctypes.POINTER(fb_sampler_opts)]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(L, name)
@@ -300,6 +302,24 @@ def fb_refine_ex(model: int, latent, text_ctx, full_schedule, opts=None) -> None
     _check(load_library().fb_refine_ex(model, _ptr(latent, np.float32),
                                        _ptr(text_ctx, np.float32), _ptr(sched), len(sched) - 1,
                                        None if opts is None else ctypes.byref(opts)))
+
+
+def fb_pipeline_step(drafter: int, latents, n: int, text_ctx, draft_schedule, skip_mask,
+                     proxy_plan, refiner=None, refine_latent=None, refine_schedule=None,
+                     draft_opts=None, refine_opts=None) -> None:
+    """Drafts `latents` with `drafter` while `refiner` refines `refine_latent` (the
+    previous pool's selected candidate) on a worker thread of the library; returns when
+    both are done. refine_latent None: the draft alone."""
+    ds = np.ascontiguousarray(draft_schedule, np.float32)
+    sk = None if skip_mask is None else np.ascontiguousarray(skip_mask, np.uint8)
+    px = None if proxy_plan is None else np.ascontiguousarray(proxy_plan, np.int32)
+    rsched = (np.zeros(1, np.float32) if refine_schedule is None
+              else np.ascontiguousarray(refine_schedule, np.float32))
+    _check(load_library().fb_pipeline_step(
+        drafter, _ptr(latents, np.float32), n, _ptr(text_ctx, np.float32), _ptr(ds),
+        len(ds) - 1, _ptr(sk), _ptr(px), None if draft_opts is None else ctypes.byref(draft_opts),
+        refiner, _ptr(refine_latent, np.float32), _ptr(rsched), len(rsched) - 1,
+        None if refine_opts is None else ctypes.byref(refine_opts)))
 
 
 def fb_select_elo(scores, compare, rho1=0.5, rho2=0.5, kappa=1.5, k_base=32.0):

@@ -648,6 +648,49 @@ def test_stream_k_on_a_partition():
     assert rel_max(outs[0].cpu().double().numpy(), want) <= 1e-4
 
 
+def test_pipeline_step_equals_the_calls_one_after_the_other():
+    """fb_pipeline_step (draft of a new pool on one partition while the previous pool's
+    candidate 0 is refined on the other, a library worker thread) gives what the same
+    two calls give one after the other, bit for bit."""
+    cfg = synth.SMALL
+    w = synth.make_weights(cfg, bf16=True, norm_std=0.2)
+    ctx = synth.make_text(cfg)
+    sched = synth.make_schedule(8)
+    dsched, rsched = sched[:4], sched[3:]
+    skip, proxy = synth.random_plan(3, cfg.depth, 1 / 3, 0.5, seed=5)
+    z_a, z_b = synth.make_latents(cfg, 3), synth.make_latents(cfg, 3, first=3)
+    with fb.Model(cfg, w) as md, fb.Model(cfg.with_(max_n=2), w) as mr, \
+            fb.SmSplit(40) as sp:
+        mr.set_stream(sp.streams[0]); mr.set_sm_budget(sp.sms[0])
+        md.set_stream(sp.streams[1]); md.set_sm_budget(sp.sms[1])
+        # pipelined: pool a alone, then pool b beside the refine of a's candidate 0
+        pa, pb = cuda(z_a), cuda(z_b)
+        fb.fb_pipeline_step(md.handle, pa, 3, ctx, dsched, skip, proxy)
+        torch.cuda.synchronize()
+        ra = pa[0].clone()
+        fb.fb_pipeline_step(md.handle, pb, 3, ctx, dsched, skip, proxy, mr.handle, ra, rsched)
+        torch.cuda.synchronize()
+        # the same calls one after the other
+        qa, qb = cuda(z_a), cuda(z_b)
+        md.draft(qa, ctx, dsched, skip, proxy)
+        torch.cuda.synchronize()
+        ra2 = qa[0].clone()
+        md.draft(qb, ctx, dsched, skip, proxy)
+        mr.refine(ra2, ctx, rsched)
+        torch.cuda.synchronize()
+        with pytest.raises(fb.FlashBonError) as e:   # the refine needs a model of its own
+            fb.fb_pipeline_step(md.handle, cuda(z_b), 3, ctx, dsched, skip, proxy, md.handle,
+                                ra.clone(), rsched)
+        assert e.value.status == fb.FB_EINVAL
+        pc = cuda(z_b)                                # (this call still drafts pc)
+        with pytest.raises(fb.FlashBonError) as e:   # a refine error comes back, prefixed
+            fb.fb_pipeline_step(md.handle, pc, 3, ctx, dsched, skip, proxy, mr.handle,
+                                ra.clone(), np.array([0.5, 0.7], np.float32))  # increasing
+        assert "refine:" in str(e.value)
+        md.set_stream(None); mr.set_stream(None)
+    assert torch.equal(pa, qa) and torch.equal(pb, qb) and torch.equal(ra, ra2)
+
+
 def test_sm_budget_and_split_reject_bad_sizes():
     with fb.Model(synth.TINY, synth.make_weights(synth.TINY)) as m:
         for n in (1, 100000):
