@@ -81,6 +81,9 @@ fb_status fb_weights_entry(const fb_cfg* cfg, int idx, const char** name,
  * on failure. The denoiser is the black-box f_theta of §3 (a DiT); the block follows
  * Eq. 7. */
 fb_status fb_init_model(const fb_cfg* cfg, const float* weights_host, fb_model** out);
+/* fb_free: waits for the model's stream and its offload copies, then releases what the
+ * model owns (device memory, its own streams, events, the pinned error word). NULL is
+ * allowed. A stream given with fb_set_stream stays the caller's. */
 void fb_free(fb_model* m);
 /* stream: a cudaStream_t (NULL = the model's own stream). */
 fb_status fb_set_stream(fb_model* m, void* stream);
@@ -257,6 +260,8 @@ fb_status fb_select_elo(const int32_t* scores, int M, double rho1, double rho2,
  * text context of the last fb_encode_text (FB_ESTATE without one). */
 fb_status fb_block_forward(fb_model* m, int layer, float* h, int n, float t);
 
+/* fb_last_error: the message of the calling thread's last failed call (each thread has
+ * its own; the string stays valid until that thread's next failing call). */
 const char* fb_last_error(void);
 
 /* ---- statistics ----------------------------------------------------------------
@@ -279,6 +284,11 @@ typedef struct fb_kstat {
   uint64_t launches;
   double ms, flops, bytes;
 } fb_kstat;
+/* fb_set_timing: `on` is a bit mask; bit k records CUDA events around every launch of
+ * class k (FB_K_*), 0 stops timing. fb_get_stats waits for the model's stream and
+ * copies the FB_K_COUNT counters (launch counts and algorithmic work are always kept,
+ * times only for timed classes); fb_reset_stats zeroes them; fb_kernel_name gives a
+ * class's name ("?" outside [0, FB_K_COUNT)). FB_EINVAL for a NULL model or output. */
 fb_status fb_set_timing(fb_model* m, int on);
 fb_status fb_get_stats(fb_model* m, fb_kstat* out /* [FB_K_COUNT] */);
 fb_status fb_reset_stats(fb_model* m);
