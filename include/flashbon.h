@@ -151,7 +151,7 @@ fb_status fb_draft(fb_model* m, float* latents, int n, const float* text_ctx,
 fb_status fb_refine(fb_model* m, float* latent, const float* text_ctx,
                     const float* full_schedule, int n_steps);
 
-/* ---- sampler options (§8 NEXT rows: guidance and the SDE step) -----------------
+/* ---- sampler options: classifier-free guidance and the SDE step (App. A.1) -------
  * guidance / text_uncond: classifier-free guidance. When text_uncond is not NULL every
  * step also runs an unconditional pass (text_uncond, [text_len][text_dim] fp32, host or
  * device) through the same plan with its own proxy cache, and uses
@@ -168,8 +168,8 @@ typedef struct fb_sampler_opts {
   const float* text_uncond;
   float sde_a;
   const float* noise;
-  /* §8 NEXT row 4, the cached state of Stage 3 (§4.2: "the layer activations ... for
-   * warm-starting activation proxies"), read as each layer's contribution
+  /* The cached state of Stage 3 (§4.2): per-layer activations kept with the latent so
+   * that the refine can warm-start its activation proxies, read as each layer's contribution
    * Delta_l = B_l(h) - h from its last computed draft step (with that step's t):
    * keep_state (fb_draft_ex): != 0 keeps every candidate's state in the model after the
    *   call, for fb_state_offload (conditional rows under guidance);
@@ -207,7 +207,7 @@ fb_status fb_pipeline_step(fb_model* drafter, float* latents, int n, const float
                            float* refine_latent, const float* refine_schedule,
                            int n_refine_steps, const fb_sampler_opts* refine_opts);
 
-/* ---- cached-state offload (§4.2 Stage 3; §8 NEXT row 4) -----------------------------
+/* ---- cached-state offload (§4.2 Stage 3) --------------------------------------------
  * The paper moves the cached tensors to host memory during drafting and brings only the
  * selected candidate back for refinement; the copies are part of the wall-clock.
  * State layout of one candidate (fb_state_bytes bytes): depth fp32 values t_l (NaN: the

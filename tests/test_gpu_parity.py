@@ -374,7 +374,7 @@ def test_model_from_device_weights_equals_host_weights():
     assert torch.equal(outs[0], outs[1])
 
 
-# ---- NEXT rows: classifier-free guidance and SDE steps -------------------------------
+# ---- classifier-free guidance and SDE steps (App. A.1) -------------------------------
 
 @pytest.fixture(scope="module")
 def small4():
@@ -473,7 +473,7 @@ def test_pipeline_draft_select_refine(small4):
     check_latents(r.cpu().numpy(), want, drafts[win], label="refine of the selected draft")
 
 
-# ---- NEXT row 4: cached-state offload and a warm-started refine (§4.2 Stage 3) --------
+# ---- cached-state offload and a warm-started refine (§4.2 Stage 3) --------------------
 
 def _parse_state(cfg, buf):
     """(t per layer, Delta per layer as fp32 [tokens][dim]) from a state buffer."""

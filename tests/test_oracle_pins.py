@@ -278,6 +278,126 @@ def test_block_matches_library_composition():
     np.testing.assert_allclose(out, x.numpy(), rtol=1e-9, atol=1e-11)
 
 
+def test_time_embed_matches_library_composition():
+    """temb = Linear(SiLU(Linear(emb(1000 t)))) and mod = Linear(SiLU(temb)) as [6, D],
+    restated with torch library routines at several t."""
+    cfg, w = _tiny()
+    m = O.OracleModel(cfg, w)
+    T = {k: t64(v) for k, v in w.items()}
+    for t in (1.0, 0.7, 0.13):
+        temb, mod = m.time_embed(t)
+        e = t64(O.timestep_embedding(t, cfg.freq_dim))
+        want_t = Fn.linear(Fn.silu(Fn.linear(e, T["time.w1"], T["time.b1"])),
+                           T["time.w2"], T["time.b2"])
+        want_m = Fn.linear(Fn.silu(want_t), T["mod.w"], T["mod.b"]).reshape(6, cfg.dim)
+        np.testing.assert_allclose(temb, want_t.numpy(), rtol=1e-12, atol=1e-13)
+        np.testing.assert_allclose(mod, want_m.numpy(), rtol=1e-12, atol=1e-13)
+
+
+def test_head_matches_library_composition():
+    """Head: LayerNorm (no affine) * (1 + table_1 + temb) + table_0 + temb, then
+    Linear(D -> C p p), restated with torch library routines; head.w is non-zero."""
+    cfg, w = _tiny()
+    w = dict(w)
+    w["head.table"] = (rng.standard_normal((2, cfg.dim)) * 0.3).astype(np.float32)
+    m = O.OracleModel(cfg, w)
+    h = rng.standard_normal((cfg.tokens, cfg.dim)) * 2 + 0.5
+    temb, _ = m.time_embed(0.45)
+    got = m.head(h, temb)
+    T = {k: t64(v) for k, v in w.items()}
+    tb = T["head.table"]
+    a = Fn.layer_norm(t64(h), (cfg.dim,), eps=cfg.eps_ln) * (1 + tb[1] + t64(temb)) \
+        + tb[0] + t64(temb)
+    want = Fn.linear(a, T["head.w"], T["head.b"]).numpy()
+    assert np.abs(w["head.w"]).max() > 0 and np.abs(want).max() > 0.1
+    np.testing.assert_allclose(got, want, rtol=1e-12, atol=1e-12)
+
+
+def _hand_cfg(dim, heads=1, head_dim=None):
+    """One token (a 2x2 latent with one channel, patch 2), so RoPE is the identity and
+    attention returns its single value row; LayerNorm eps 0 keeps hand values exact."""
+    return synth.Cfg(depth=1, dim=dim, heads=heads, head_dim=head_dim or dim, ffn=dim,
+                     text_len=1, text_dim=dim, latent_c=1, latent_h=2, latent_w=2,
+                     freq_dim=4, eps_ln=0.0)
+
+
+def _zero_weights(cfg):
+    return {n: np.zeros(s, np.float64) for n, s, _ in synth.weight_specs(cfg)}
+
+
+# logistic sigmoid at the points used below: 1/(1+e^-x)
+SIG2, SIGM1 = 0.8807970779778823, 0.2689414213699951
+
+
+def test_time_embed_hand_values_fix_silu_and_chunk_order():
+    """D = 2, t = 0: the sinusoid is [cos 0, cos 0, sin 0, sin 0] = [1, 1, 0, 0].
+    Case 1 pins the first SiLU and the cos-first order: pre-activation [2, -1] gives
+    temb = [2 sig(2), -sig(-1)]. Case 2 pins the SiLU before the modulation and the
+    row order of the [6, D] split: row k of mod is output features 2k, 2k+1."""
+    cfg = _hand_cfg(2, head_dim=4)
+    w = _zero_weights(cfg)
+    w["time.w1"][0, 0], w["time.w1"][1, 1] = 2.0, -1.0
+    w["time.w2"][:] = np.eye(2)
+    w["mod.b"][:] = np.arange(12)
+    temb, mod = O.OracleModel(cfg, w).time_embed(0.0)
+    np.testing.assert_allclose(temb, [2 * SIG2, -SIGM1], rtol=1e-14)
+    np.testing.assert_allclose(mod, np.arange(12).reshape(6, 2), atol=0)
+    # case 2: temb = b2 = [2, -1] exactly; mod row 2 (the first gate) reads SiLU(temb)
+    w["time.w1"][:] = 0
+    w["time.w2"][:] = 0
+    w["time.b2"][:] = [2.0, -1.0]
+    w["mod.b"][:] = 0
+    w["mod.w"][4] = [1.0, 0.0]          # row 2, feature 0 <- SiLU(temb)_0
+    w["mod.w"][11] = [0.0, 3.0]         # row 5, feature 1 <- 3 SiLU(temb)_1
+    temb, mod = O.OracleModel(cfg, w).time_embed(0.0)
+    np.testing.assert_allclose(temb, [2.0, -1.0], atol=0)
+    want = np.zeros((6, 2))
+    want[2, 0], want[5, 1] = 2 * SIG2, -3 * SIGM1
+    np.testing.assert_allclose(mod, want, rtol=1e-14, atol=1e-300)
+
+
+def test_head_hand_values_fix_shift_and_scale():
+    """D = 2, h = [1, -1] (LayerNorm with eps 0 is the identity on it), table rows
+    [0.5, 0.25] and [1, 2], temb [0.125, 0.5]: scale 1 + [1.125, 2.5], shift
+    [0.625, 0.75], a = [2.75, -2.75]; head rows [1,0], [0,1], [1,1], [1,-1] with bias
+    [0, 0, 0, 1] give v = [2.75, -2.75, 0, 6.5]. Swapping the rows, or dropping temb
+    from either, changes v."""
+    cfg = _hand_cfg(2, head_dim=4)
+    w = _zero_weights(cfg)
+    w["head.table"][:] = [[0.5, 0.25], [1.0, 2.0]]
+    w["head.w"][:] = [[1, 0], [0, 1], [1, 1], [1, -1]]
+    w["head.b"][:] = [0, 0, 0, 1]
+    v = O.OracleModel(cfg, w).head(np.array([[1.0, -1.0]]), np.array([0.125, 0.5]))
+    np.testing.assert_allclose(v, [[2.75, -2.75, 0.0, 6.5]], atol=1e-15)
+
+
+def test_block_hand_values_fix_the_modulation_chunks():
+    """D = 4, one head, one token, h = [1, -1, 1, -1] (its own LayerNorm with eps 0).
+    All matrices are zero except the value part of W_qkv, W_o, W_1 and W_2 (identity),
+    so attention returns v = a and the cross branch adds nothing. Given
+    mod rows s1 = 0.5, c1 = 1, g1 = [1, 2, 3, 4], s2 = 0, c2 = -1, g2 = [10, 20, 30, 40]
+    and b_2 = 1:
+      a1 = LN(h)(1 + c1) + s1 = [2.5, -1.5, 2.5, -1.5];  h1 = h + g1 a1 = [3.5, -4, 8.5, -7]
+      a2 = LN(h1)(1 + c2) + s2 = 0;  FFN = W_2 GELU(0) + b_2 = 1;  h2 = h1 + g2.
+    A swapped shift/scale or a wrong gate row changes the result."""
+    cfg = _hand_cfg(4)
+    w = _zero_weights(cfg)
+    p = "blocks.0."
+    w[p + "attn.wqkv"][8:12] = np.eye(4)
+    w[p + "attn.wo"][:] = np.eye(4)
+    w[p + "ffn.w1"][:] = np.eye(4)
+    w[p + "ffn.w2"][:] = np.eye(4)
+    w[p + "ffn.b2"][:] = 1.0
+    for n in ("attn.norm_q", "attn.norm_k", "cross.norm_q", "cross.norm_k", "norm3.w"):
+        w[p + n][:] = 1.0
+    m = O.OracleModel(cfg, w)
+    mod = np.array([[0.5] * 4, [1.0] * 4, [1, 2, 3, 4], [0.0] * 4, [-1.0] * 4,
+                    [10, 20, 30, 40]], np.float64)
+    kv = (np.zeros((1, 4)), np.zeros((1, 4)))
+    out = m.block(0, np.array([[1.0, -1.0, 1.0, -1.0]]), mod, kv)
+    np.testing.assert_allclose(out, [[13.5, 16.0, 38.5, 33.0]], atol=1e-13)
+
+
 def test_skip_equals_zero_contribution_block():
     """Eq. 6: skipping block l equals running a model whose block l adds nothing."""
     cfg, w = _tiny()
@@ -361,7 +481,7 @@ def test_candidates_are_independent():
     np.testing.assert_array_equal(m.draft(z, ctx, sched, sk, px, candidates=[2])[0], all3[2])
 
 
-# -- NEXT row: the cached state and a warm-started refine (§4.2 Stage 3, R12) -----------------
+# -- the cached state and a warm-started refine (§4.2 Stage 3, reading R12) ------------------
 
 def test_state_holds_each_layers_last_computed_contribution():
     """keep_state returns, per layer, Delta_l = h_after - h_before at the layer's last
@@ -426,7 +546,7 @@ def test_state_proxy_rules():
         O.resolve_plan(skip, proxy, state_layers=(0, 1))       # order 1 from a single anchor
 
 
-# -- NEXT rows: classifier-free guidance and the SDE step (App. A.1) ------------------------
+# -- classifier-free guidance and the SDE step (App. A.1) -----------------------------------
 
 def test_sde_step_hand_value():
     # t = 0.5, t' = 0.4, a = 0.3: sigma = 0.3; drift 2 + 0.09/1.0 * (1 + 0.5*2) = 2.18
@@ -488,7 +608,7 @@ def test_cfg_with_identical_contexts_is_unguided():
     np.testing.assert_allclose(a, b, rtol=1e-12, atol=1e-12)
 
 
-# -- NEXT row: multi-stage Elo selection (§4.2 Stage 2) -------------------------------------
+# -- multi-stage Elo selection (§4.2 Stage 2) ------------------------------------------------
 
 def test_elo_seed_values_from_the_paper():
     assert O.elo_seed(5) == 1500.0 and O.elo_seed(10) == 2000.0 and O.elo_seed(1) == 1100.0
