@@ -348,6 +348,12 @@ fb_status fb_op_attention(fb_model* m, const void* Q, int ldq, const void* K, in
  * them before returning. The error word is cleared at the start of every call. Calls
  * that overlap in time (other host threads, other streams) share these arrays and race:
  * serialise them.
+ * SMs: the grid and the 4-blocks-per-pair rule use the whole device's SM count, and the
+ * split relies on all of the device's SM pairs being resident at once. Do not pass a
+ * stream of an SM partition (fb_sm_split): there completion depends on the order in
+ * which the hardware starts clusters; a finisher of a cut tile whose contributors cannot
+ * start until it leaves waits until the device wait limit (2 s by default) and the call
+ * returns FB_ECUDA.
  * Errors: FB_EINVAL for a NULL pointer, a bad epi, N % 256 != 0, shapes the tcgen05
  * kernel does not take (K % 64, alignment), fewer than 4 K blocks per SM pair
  * (ceil(M / 256) * N / 256 * K / 64 < 4 * pairs) or a device with more than
@@ -357,6 +363,29 @@ fb_status fb_gemm_streamk_noalloc(void* stream, int M, int N, int K, const void*
                                   const void* W, const float* bias, int epi, void* out,
                                   const float* resid, const float* gate, const float* base,
                                   void* delta);
+
+/* ---- testing hooks (engineering entry points; the paper has no counterpart) ---------
+ * fb_set_device_wait_limit: every device-side wait of the library's kernels (mbarrier
+ * phases, stream-K counters) gives up after this many nanoseconds, records
+ * "device wait timed out" in the call's error word, lets its copies in flight land,
+ * frees its TMEM and returns; the call then returns FB_ECUDA and leaves the model
+ * usable. ns = 0 restores the default (2 s). Applies to the current device and to every
+ * model and call on it; tests shorten it to make a wait run out quickly. Not for use
+ * while kernels of the library are running.
+ * fb_test_fail_alloc: host-side failure injection for device allocations. After the call
+ * the library counts its device allocations (every cudaMalloc it makes) from 0; the one
+ * numbered k fails as an out-of-memory cudaMalloc would (the caller sees FB_ENOMEM).
+ * k < 0 disarms. fb_test_alloc_calls: allocations counted since the last
+ * fb_test_fail_alloc. Process-wide; not thread-safe against concurrent model creation.
+ * fb_test_poison_counters: sets the model's stream-K tile counters (m = NULL: those of
+ * fb_gemm_streamk_noalloc) to a large negative value, as a crashed launch could leave
+ * them, so that the next stream-K finisher waits for a count no launch will reach. The
+ * wait runs out at the device wait limit, the call returns FB_ECUDA and clears the
+ * counters; the call after it computes normally. */
+fb_status fb_set_device_wait_limit(unsigned long long ns);
+fb_status fb_test_fail_alloc(long k);
+long fb_test_alloc_calls(void);
+fb_status fb_test_poison_counters(fb_model* m);
 
 #ifdef __cplusplus
 }

@@ -17,6 +17,7 @@
 #include <cstdlib>
 #include <cstring>
 #include <map>
+#include <atomic>
 #include <mutex>
 #include <thread>
 #include <string>
@@ -144,6 +145,7 @@ struct Pending {
 
 struct fb_model {
   fb_cfg c;
+  int dev = 0;  // the device current at fb_init_model; every launch of the model runs there
   int P, PD, gh, gw;
   size_t Mmax;
   int num_sms;      // SMs the model's launches may use (fb_set_sm_budget), <= dev_sms
@@ -210,9 +212,16 @@ struct fb_model {
 namespace {
 
 // ---- allocation helpers -------------------------------------------------------------
+// Host-side failure injection (fb_test_fail_alloc): device allocations are counted from
+// the last arming, and the one whose index equals g_fail_at fails as cudaMalloc would.
+std::atomic<long> g_alloc_calls{0};
+std::atomic<long> g_fail_at{-1};
+
 fb_status dalloc(fb_model* m, void** p, size_t bytes) {
   *p = nullptr;
   if (bytes == 0) bytes = 16;
+  if (g_alloc_calls.fetch_add(1) == g_fail_at.load())
+    return fail(FB_ENOMEM, "cudaMalloc(%zu bytes) failed: injected failure", bytes);
   cudaError_t e = cudaMalloc(p, bytes);
   if (e != cudaSuccess) {
     cudaGetLastError();
@@ -912,6 +921,7 @@ fb_status fb_init_model(const fb_cfg* cfg, const float* weights_host, fb_model**
     cudaGetLastError();
     return bail(fail(FB_ECUDA, "no CUDA device"));
   }
+  m->dev = dev;
   // A blocking stream: its work is ordered after work the caller put on the legacy
   // default stream (e.g. copies that fill the input buffers) and vice versa.
   if (cudaStreamCreateWithFlags(&m->own, cudaStreamDefault) != cudaSuccess)
@@ -1403,6 +1413,43 @@ fb_status fb_set_op_repeat(fb_model* m, int n) {
   return FB_OK;
 }
 
+fb_status fb_set_device_wait_limit(unsigned long long ns) {
+  if (ns == 0) ns = FB_WAIT_LIMIT_NS;
+  CK(gemm_tc_set_wait_limit(ns));
+  CK(attention_tc_set_wait_limit(ns));
+  return FB_OK;
+}
+
+fb_status fb_test_fail_alloc(long k) {
+  g_fail_at.store(-1);
+  g_alloc_calls.store(0);
+  g_fail_at.store(k < 0 ? -1 : k);
+  return FB_OK;
+}
+
+long fb_test_alloc_calls(void) { return g_alloc_calls.load(); }
+
+fb_status fb_test_poison_counters(fb_model* m) {
+  int* ctr = nullptr;
+  size_t n = 0;
+  cudaStream_t st = nullptr;
+  if (m) {
+    ctr = m->sk_ctr;
+    n = (size_t)m->sk_clusters * SK_CTR_PER_CLUSTER;
+    st = m->st;
+  } else {
+    NoAllocDev* d = nullptr;
+    CKS(noalloc_setup(&d));
+    ctr = d->ctr;
+    n = (size_t)FB_NOALLOC_MAX_PAIRS * SK_CTR_PER_CLUSTER;
+  }
+  if (!ctr) return fail(FB_EINVAL, "no stream-K counters");
+  fb_stream_op_not_kernel();
+  CK(cudaMemsetAsync(ctr, 0x80, n * sizeof(int), st));  // every counter 0x80808080 < 0
+  CK(cudaStreamSynchronize(st));
+  return FB_OK;
+}
+
 }  // extern "C"
 
 // ---- draft / refine pipeline step -------------------------------------------------
@@ -1424,6 +1471,13 @@ extern "C" fb_status fb_pipeline_step(fb_model* drafter, float* latents, int n,
   std::thread worker;
   if (refine_latent) {
     worker = std::thread([&] {
+      // a new thread starts on device 0: make the refiner's device current first
+      const cudaError_t e = cudaSetDevice(refiner->dev);
+      if (e != cudaSuccess) {
+        rs = FB_ECUDA;
+        rmsg = std::string("cudaSetDevice failed: ") + cudaGetErrorString(e);
+        return;
+      }
       rs = fb_refine_ex(refiner, refine_latent, text_ctx, refine_schedule, n_refine_steps,
                         refine_opts);
       if (rs != FB_OK) rmsg = g_last_error;

@@ -15,7 +15,11 @@
 //    P = exp2(S * log2(e)/sqrt(d) - m) as bf16 into the swizzled P tile, and rescales its
 //    O row in TMEM only when the max grew by more than 2^8 since the last rescale
 //    (every term of O and l always uses the same m, so the result is exact). At the end
-//    each thread normalises its O row and stores it.
+//    each thread normalises its O row and stores it. The exponent arguments and the row
+//    sum run on key pairs with packed fp32 FMA / add (one instruction per two keys).
+// Ragged ends: the last key tile's S MMA is only as wide as its 32-key chunks of real keys
+// and its PV MMA reads only those keys; in the 256-query kernel a second query tile that
+// lies wholly past Lq is neither loaded nor computed.
 // All waits are bounded; on a timeout the kernel records the error and drains.
 #include <cudaTypedefs.h>
 
@@ -62,6 +66,11 @@ __device__ __forceinline__ uint64_t desc_mn_sw128(uint32_t saddr, uint32_t lbo) 
   return d;
 }
 
+// instruction descriptor of the S MMA with N = 32 * nch keys (N field: N >> 3 at bit 17)
+__device__ __forceinline__ uint32_t idesc_keys(uint32_t idesc128, int nch) {
+  return (idesc128 & ~(0x3Fu << 17)) | ((uint32_t)(4 * nch) << 17);
+}
+
 // three-input maximum (one instruction on sm_100 and later)
 __device__ __forceinline__ float fmax3(float a, float b, float c) {
   float r;
@@ -88,6 +97,26 @@ __device__ __forceinline__ float ex2(float x) {
   float y;
   asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
   return y;
+}
+
+// packed pairs of fp32 (sm_100 and later execute one fma/add on both halves)
+__device__ __forceinline__ uint64_t f2_pack(float lo, float hi) {
+  uint64_t r;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(lo), "f"(hi));
+  return r;
+}
+__device__ __forceinline__ void f2_unpack(uint64_t v, float& lo, float& hi) {
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(v));
+}
+__device__ __forceinline__ uint64_t f2_fma(uint64_t a, uint64_t b, uint64_t c) {
+  uint64_t d;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
+  return d;
+}
+__device__ __forceinline__ uint64_t f2_add(uint64_t a, uint64_t b) {
+  uint64_t d;
+  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
 }
 
 __device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t* r) {
@@ -135,6 +164,9 @@ __global__ void __launch_bounds__(THREADS, 1)
   const int q_row0 = b * p.Lq + qt * TB;
   const int kv_row0 = b * p.kv_batch_rows;
   const int n_kv = (p.Lkv + TB - 1) / TB;
+  // the last key tile holds last_nch 32-key chunks of real keys: its S MMA is that many
+  // chunks wide and its PV MMA reads only those keys
+  const int last_nch = (p.Lkv - (n_kv - 1) * TB + 31) >> 5;
   int* err = p.err;
   bool failed = false;
 
@@ -200,11 +232,21 @@ __global__ void __launch_bounds__(THREADS, 1)
       const uint32_t qa = smem_u32(Qs), pa = smem_u32(Ps);
       auto issue_s = [&](int j) {
         const uint32_t ka = smem_u32(Ks + (j % KSLOT) * K_BYTES);
+        if (j + 1 < n_kv || last_nch == 4) {
 #pragma unroll
-        for (int kk = 0; kk < 8; ++kk) {
-          const uint32_t off = (kk >> 2) * SUB + (kk & 3) * 32;
-          tc_mma_f16(tmem + (j & 1) * TB, desc_k_sw128(qa + off), desc_k_sw128(ka + off), idesc_s,
-                     kk ? 1u : 0u);
+          for (int kk = 0; kk < 8; ++kk) {
+            const uint32_t off = (kk >> 2) * SUB + (kk & 3) * 32;
+            tc_mma_f16(tmem + (j & 1) * TB, desc_k_sw128(qa + off), desc_k_sw128(ka + off),
+                       idesc_s, kk ? 1u : 0u);
+          }
+        } else {
+          const uint32_t idesc = idesc_keys(idesc_s, last_nch);
+#pragma unroll 1
+          for (int kk = 0; kk < 8; ++kk) {
+            const uint32_t off = (kk >> 2) * SUB + (kk & 3) * 32;
+            tc_mma_f16(tmem + (j & 1) * TB, desc_k_sw128(qa + off), desc_k_sw128(ka + off),
+                       idesc, kk ? 1u : 0u);
+          }
         }
         tc_commit(&s_full[j & 1]);
         tc_commit(&k_empty[j % KSLOT]);  // K_j is no longer needed once S_j is done
@@ -222,11 +264,20 @@ __global__ void __launch_bounds__(THREADS, 1)
           if (!mbar_wait(&v_full[j & 1], (j >> 1) & 1, err)) { failed = true; break; }
           tc_fence_after();
           const uint32_t va = smem_u32(Vs + (j & 1) * V_BYTES);
+          if (j + 1 < n_kv || last_nch == 4) {
 #pragma unroll
-          for (int kk = 0; kk < 8; ++kk) {
-            const uint32_t off = (kk >> 2) * SUB + (kk & 3) * 32;
-            tc_mma_f16(tmem + O_COL, desc_k_sw128(pa + off), desc_mn_sw128(va + kk * 2048, SUB),
-                       idesc_pv, (j | kk) ? 1u : 0u);
+            for (int kk = 0; kk < 8; ++kk) {
+              const uint32_t off = (kk >> 2) * SUB + (kk & 3) * 32;
+              tc_mma_f16(tmem + O_COL, desc_k_sw128(pa + off), desc_mn_sw128(va + kk * 2048, SUB),
+                         idesc_pv, (j | kk) ? 1u : 0u);
+            }
+          } else {
+#pragma unroll 1
+            for (int kk = 0; kk < 2 * last_nch; ++kk) {  // 16 keys per step
+              const uint32_t off = (kk >> 2) * SUB + (kk & 3) * 32;
+              tc_mma_f16(tmem + O_COL, desc_k_sw128(pa + off), desc_mn_sw128(va + kk * 2048, SUB),
+                         idesc_pv, (j | kk) ? 1u : 0u);
+            }
           }
           tc_commit(&v_empty[j & 1]);
           tc_commit(o_done);
@@ -291,24 +342,30 @@ __global__ void __launch_bounds__(THREADS, 1)
         }
         tmem_st_wait();
       }
-      float ls[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};  // independent partial sums
+      // exponent arguments and the row sum on key pairs (packed FMA and add)
+      const uint64_t sc2 = f2_pack(p.scale_log2, p.scale_log2);
+      const uint64_t nm2 = f2_pack(-m_used, -m_used);
+      uint64_t ls2[4] = {0ull, 0ull, 0ull, 0ull};  // independent partial sums
 #pragma unroll
       for (int ch = 0; ch < 16; ++ch) {  // 16-byte chunks of 8 keys
-        float e[8];
+        uint32_t w[4];
 #pragma unroll
-        for (int q = 0; q < 8; ++q) {
-          e[q] = ex2(fmaf(s[ch * 8 + q], p.scale_log2, -m_used));
-          ls[q] += e[q];
+        for (int q = 0; q < 4; ++q) {
+          float t0, t1;
+          f2_unpack(f2_fma(f2_pack(s[ch * 8 + 2 * q], s[ch * 8 + 2 * q + 1]), sc2, nm2), t0, t1);
+          const float e0 = ex2(t0), e1 = ex2(t1);
+          ls2[q] = f2_add(ls2[q], f2_pack(e0, e1));
+          w[q] = pack_bf16x2(e0, e1);
         }
-        uint4 v;
-        v.x = pack_bf16x2(e[0], e[1]);
-        v.y = pack_bf16x2(e[2], e[3]);
-        v.z = pack_bf16x2(e[4], e[5]);
-        v.w = pack_bf16x2(e[6], e[7]);
         const int sub = ch >> 3, c16 = (ch & 7) ^ (r & 7);
-        *reinterpret_cast<uint4*>(prow + sub * SUB + c16 * 16) = v;
+        *reinterpret_cast<uint4*>(prow + sub * SUB + c16 * 16) = make_uint4(w[0], w[1], w[2], w[3]);
       }
-      l += ((ls[0] + ls[1]) + (ls[2] + ls[3])) + ((ls[4] + ls[5]) + (ls[6] + ls[7]));
+      {
+        float a0, a1, b0, b1;
+        f2_unpack(f2_add(ls2[0], ls2[1]), a0, a1);
+        f2_unpack(f2_add(ls2[2], ls2[3]), b0, b1);
+        l += (a0 + a1) + (b0 + b1);
+      }
       fence_async_smem();  // P visible to the tensor core (async proxy)
       tc_fence_before();
       __syncwarp();
@@ -436,8 +493,10 @@ __global__ void __launch_bounds__(THREADS2, 1)
     // ---------------- TMA producers: lane 0 Q and K, lane 1 V ----------------
     const int xq = h * 128;
     if (lane == 0) {
-      mbar_expect_tx(q_full, 2 * Q_BYTES);
-      for (int g = 0; g < 2; ++g) {
+      // a second query tile with no query in range (the ragged end of Lq) does no work
+      const int ngroups = qb * 2 * TB + TB < p.Lq ? 2 : 1;
+      mbar_expect_tx(q_full, ngroups * Q_BYTES);
+      for (int g = 0; g < ngroups; ++g) {
         tma_load_2d(Qs + g * Q_BYTES, &tmQ, q_full, xq, q_row0 + g * TB);
         tma_load_2d(Qs + g * Q_BYTES + SUB, &tmQ, q_full, xq + 64, q_row0 + g * TB);
       }
@@ -467,27 +526,50 @@ __global__ void __launch_bounds__(THREADS2, 1)
                                ((uint32_t)(TB >> 4) << 24);
       const uint32_t idesc_pv = idesc_s | (1u << 16);
       const uint32_t qa = smem_u32(Qs);
+      const int two = qb * 2 * TB + TB < p.Lq;  // both tiles hold queries (as for the Q load)
+      // real keys of the last key tile, in 32-key chunks (see attn_tc_kernel)
+      const int last_nch = (p.Lkv - (n_kv - 1) * TB + 31) >> 5;
+      // full key tiles take the constant-folded loops; the last tile of a ragged Lkv
+      // (last_nch < 4 chunks of 32 keys) issues S with N = 32 * last_nch and PV over those
+      // keys only
       auto issue_s = [&](int g, int j) {
         const uint32_t ka = smem_u32(Ks + (j % KSLOT) * K_BYTES);
         const uint32_t qg = qa + g * Q_BYTES;
+        if (j + 1 < n_kv || last_nch == 4) {
 #pragma unroll
-        for (int kk = 0; kk < 8; ++kk) {
-          const uint32_t off = (kk >> 2) * SUB + (kk & 3) * 32;
-          tc_mma_f16(tmem + g * TB, desc_k_sw128(qg + off), desc_k_sw128(ka + off), idesc_s,
-                     kk ? 1u : 0u);
+          for (int kk = 0; kk < 8; ++kk) {
+            const uint32_t off = (kk >> 2) * SUB + (kk & 3) * 32;
+            tc_mma_f16(tmem + g * TB, desc_k_sw128(qg + off), desc_k_sw128(ka + off), idesc_s,
+                       kk ? 1u : 0u);
+          }
+        } else {
+          const uint32_t idesc = idesc_keys(idesc_s, last_nch);
+#pragma unroll 1
+          for (int kk = 0; kk < 8; ++kk) {
+            const uint32_t off = (kk >> 2) * SUB + (kk & 3) * 32;
+            tc_mma_f16(tmem + g * TB, desc_k_sw128(qg + off), desc_k_sw128(ka + off), idesc,
+                       kk ? 1u : 0u);
+          }
         }
         tc_commit(&s_full[g]);
-        if (g == 1) tc_commit(&k_empty[j % KSLOT]);  // both tiles' S_j done: K_j is free
+        if (g == 1 || two == 0) tc_commit(&k_empty[j % KSLOT]);  // every tile's S_j done
       };
       auto issue_pv = [&](int g, int j) {
         const uint32_t va = smem_u32(Vs + (j & 1) * V_BYTES);
+        if (j + 1 < n_kv || last_nch == 4) {
 #pragma unroll
-        for (int kk = 0; kk < 8; ++kk)
-          tc_mma_f16_ts(tmem + O_COL + g * TB, tmem + g * TB + kk * 8,
-                        desc_mn_sw128(va + kk * 2048, SUB), idesc_pv, (j | kk) ? 1u : 0u);
+          for (int kk = 0; kk < 8; ++kk)
+            tc_mma_f16_ts(tmem + O_COL + g * TB, tmem + g * TB + kk * 8,
+                          desc_mn_sw128(va + kk * 2048, SUB), idesc_pv, (j | kk) ? 1u : 0u);
+        } else {
+#pragma unroll 1
+          for (int kk = 0; kk < 2 * last_nch; ++kk)  // 16 keys per step
+            tc_mma_f16_ts(tmem + O_COL + g * TB, tmem + g * TB + kk * 8,
+                          desc_mn_sw128(va + kk * 2048, SUB), idesc_pv, (j | kk) ? 1u : 0u);
+        }
       };
       bool ok = mbar_wait(q_full, 0, err) && mbar_wait(&k_full[0], 0, err);
-      if (ok) {
+      if (ok && two) {
         tc_fence_after();
         issue_s(0, 0);
         issue_s(1, 0);
@@ -508,8 +590,24 @@ __global__ void __launch_bounds__(THREADS2, 1)
           tc_commit(&v_empty[j & 1]);
           if (more) issue_s(1, j + 1);
         }
-        if (ok) tc_commit(o_done);
+      } else if (ok) {
+        // one tile (the second lies past Lq): the same chain without the other group
+        tc_fence_after();
+        issue_s(0, 0);
+        for (int j = 0; j < n_kv && ok; ++j) {
+          if (!(ok = mbar_wait(&p_full[0], j & 1, err))) break;
+          if (!(ok = mbar_wait(&v_full[j & 1], (j >> 1) & 1, err))) break;
+          tc_fence_after();
+          issue_pv(0, j);
+          tc_commit(&v_empty[j & 1]);
+          if (j + 1 < n_kv) {
+            if (!(ok = mbar_wait(&k_full[(j + 1) % KSLOT], ((j + 1) / KSLOT) & 1, err))) break;
+            tc_fence_after();
+            issue_s(0, j + 1);
+          }
+        }
       }
+      if (ok) tc_commit(o_done);
       failed = !ok;
     }
   } else {
@@ -520,93 +618,106 @@ __global__ void __launch_bounds__(THREADS2, 1)
     const uint32_t lane_base = tmem + ((uint32_t)(quarter * 32) << 16);
     const uint32_t s_col = g * TB, o_col = O_COL + g * TB;
     float m_used = -INFINITY, l = 0.f;
-    for (int j = 0; j < n_kv && !failed; ++j) {
-      const bool ok = mbar_wait(&s_full[g], j & 1, err);
-      if (!__all_sync(0xffffffffu, ok)) { failed = true; break; }
-      tc_fence_after();
-      float s[128];
-      {
-        // all four loads in flight, one wait; scores stay unscaled (the scale is > 0, so the
-        // row max commutes with it and is scaled once)
-        uint32_t u[128];
-#pragma unroll
-        for (int c = 0; c < 4; ++c) tmem_ld32(lane_base + s_col + c * 32, u + c * 32);
-        tmem_ld_wait();
-#pragma unroll
-        for (int c = 0; c < 4; ++c) reg_fence32(u + c * 32);
-#pragma unroll
-        for (int i = 0; i < 128; ++i) s[i] = __uint_as_float(u[i]);
-      }
-      const int valid = p.Lkv - j * TB;  // keys of this tile that exist
-      if (valid < TB) {
-#pragma unroll
-        for (int i = 0; i < 128; ++i)
-          if (i >= valid) s[i] = -INFINITY;
-      }
-      const float mx = rowmax128(s) * p.scale_log2;
-      if (j == 0) {
-        m_used = mx;
-      } else if (__any_sync(0xffffffffu, mx > m_used + 8.f)) {
-        const float m_new = fmaxf(m_used, mx);
-        const float alpha = ex2(m_used - m_new);
-        m_used = m_new;
-        l *= alpha;
-#pragma unroll 1
-        for (int c = 0; c < 4; ++c) {
-          uint32_t u[32];
-          tmem_ld32(lane_base + o_col + c * 32, u);
-          tmem_ld_wait();
-          reg_fence32(u);
-#pragma unroll
-          for (int i = 0; i < 32; ++i) u[i] = __float_as_uint(__uint_as_float(u[i]) * alpha);
-          tmem_st32(lane_base + o_col + c * 32, u);
-        }
-      }
-      float ls[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};  // independent partial sums
-#pragma unroll
-      for (int c = 0; c < 2; ++c) {
-        uint32_t u[32];
-#pragma unroll
-        for (int i = 0; i < 32; ++i) {
-          const float e0 = ex2(fmaf(s[c * 64 + 2 * i], p.scale_log2, -m_used));
-          const float e1 = ex2(fmaf(s[c * 64 + 2 * i + 1], p.scale_log2, -m_used));
-          ls[(2 * i) & 7] += e0;
-          ls[(2 * i + 1) & 7] += e1;
-          u[i] = pack_bf16x2(e0, e1);
-        }
-        tmem_st32(lane_base + s_col + c * 32, u);
-      }
-      l += ((ls[0] + ls[1]) + (ls[2] + ls[3])) + ((ls[4] + ls[5]) + (ls[6] + ls[7]));
-      tmem_st_wait();
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&p_full[g]);
-    }
-    if (!failed) {
-      const bool ok = mbar_wait(o_done, 0, err);
-      if (__all_sync(0xffffffffu, ok)) {
+    // a tile with no query in range (the ragged end of Lq) has no MMAs and no softmax
+    if (qb * 2 * TB + g * TB < p.Lq) {
+      for (int j = 0; j < n_kv && !failed; ++j) {
+        const bool ok = mbar_wait(&s_full[g], j & 1, err);
+        if (!__all_sync(0xffffffffu, ok)) { failed = true; break; }
         tc_fence_after();
-        const float inv = 1.f / l;
-        const int qrow = qb * 2 * TB + g * TB + r;
-        bf16* orow = p.O + (size_t)(q_row0 + g * TB + r) * p.ldo + h * 128;
-#pragma unroll 1
-        for (int c = 0; c < 4; ++c) {
-          uint32_t u[32];
-          tmem_ld32(lane_base + o_col + c * 32, u);
+        float s[128];
+        {
+          // all four loads in flight, one wait; scores stay unscaled (the scale is > 0, so the
+          // row max commutes with it and is scaled once)
+          uint32_t u[128];
+#pragma unroll
+          for (int c = 0; c < 4; ++c) tmem_ld32(lane_base + s_col + c * 32, u + c * 32);
           tmem_ld_wait();
-          reg_fence32(u);
-          if (qrow < p.Lq) {
 #pragma unroll
-            for (int q = 0; q < 4; ++q) {
-              float v[8];
+          for (int c = 0; c < 4; ++c) reg_fence32(u + c * 32);
 #pragma unroll
-              for (int i = 0; i < 8; ++i) v[i] = __uint_as_float(u[q * 8 + i]) * inv;
-              store_bf16x8(orow + c * 32 + q * 8, v);
-            }
+          for (int i = 0; i < 128; ++i) s[i] = __uint_as_float(u[i]);
+        }
+        const int valid = p.Lkv - j * TB;  // keys of this tile that exist
+        if (valid < TB) {
+#pragma unroll
+          for (int i = 0; i < 128; ++i)
+            if (i >= valid) s[i] = -INFINITY;
+        }
+        const float mx = rowmax128(s) * p.scale_log2;
+        if (j == 0) {
+          m_used = mx;
+        } else if (__any_sync(0xffffffffu, mx > m_used + 8.f)) {
+          const float m_new = fmaxf(m_used, mx);
+          const float alpha = ex2(m_used - m_new);
+          m_used = m_new;
+          l *= alpha;
+#pragma unroll 1
+          for (int c = 0; c < 4; ++c) {
+            uint32_t u[32];
+            tmem_ld32(lane_base + o_col + c * 32, u);
+            tmem_ld_wait();
+            reg_fence32(u);
+#pragma unroll
+            for (int i = 0; i < 32; ++i) u[i] = __float_as_uint(__uint_as_float(u[i]) * alpha);
+            tmem_st32(lane_base + o_col + c * 32, u);
           }
         }
-      } else {
-        failed = true;
+        // exponent arguments and the row sum on key pairs: one packed FMA and one packed
+        // add per two keys
+        const uint64_t sc2 = f2_pack(p.scale_log2, p.scale_log2);
+        const uint64_t nm2 = f2_pack(-m_used, -m_used);
+        uint64_t ls2[4] = {0ull, 0ull, 0ull, 0ull};  // independent partial sums
+#pragma unroll
+        for (int c = 0; c < 2; ++c) {
+          uint32_t u[32];
+#pragma unroll
+          for (int i = 0; i < 32; ++i) {
+            float t0, t1;
+            f2_unpack(f2_fma(f2_pack(s[c * 64 + 2 * i], s[c * 64 + 2 * i + 1]), sc2, nm2), t0,
+                      t1);
+            const float e0 = ex2(t0), e1 = ex2(t1);
+            ls2[i & 3] = f2_add(ls2[i & 3], f2_pack(e0, e1));
+            u[i] = pack_bf16x2(e0, e1);
+          }
+          tmem_st32(lane_base + s_col + c * 32, u);
+        }
+        {
+          float a0, a1, b0, b1;
+          f2_unpack(f2_add(ls2[0], ls2[1]), a0, a1);
+          f2_unpack(f2_add(ls2[2], ls2[3]), b0, b1);
+          l += (a0 + a1) + (b0 + b1);
+        }
+        tmem_st_wait();
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&p_full[g]);
+      }
+      if (!failed) {
+        const bool ok = mbar_wait(o_done, 0, err);
+        if (__all_sync(0xffffffffu, ok)) {
+          tc_fence_after();
+          const float inv = 1.f / l;
+          const int qrow = qb * 2 * TB + g * TB + r;
+          bf16* orow = p.O + (size_t)(q_row0 + g * TB + r) * p.ldo + h * 128;
+#pragma unroll 1
+          for (int c = 0; c < 4; ++c) {
+            uint32_t u[32];
+            tmem_ld32(lane_base + o_col + c * 32, u);
+            tmem_ld_wait();
+            reg_fence32(u);
+            if (qrow < p.Lq) {
+#pragma unroll
+              for (int q = 0; q < 4; ++q) {
+                float v[8];
+#pragma unroll
+                for (int i = 0; i < 8; ++i) v[i] = __uint_as_float(u[q * 8 + i]) * inv;
+                store_bf16x8(orow + c * 32 + q * 8, v);
+              }
+            }
+          }
+        } else {
+          failed = true;
+        }
       }
     }
   }
@@ -652,6 +763,10 @@ bool map_128x64(CUtensorMap* m, const bf16* ptr, int rows, int cols, int ld) {
 }
 
 }  // namespace
+
+cudaError_t attention_tc_set_wait_limit(unsigned long long ns) {
+  return fb_set_wait_limit_tu(ns);
+}
 
 bool attention_tc_supported(const AttnArgs& a) {
   auto al16 = [](const void* q) { return (reinterpret_cast<uintptr_t>(q) & 15) == 0; };

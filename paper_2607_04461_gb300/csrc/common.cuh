@@ -11,8 +11,17 @@ typedef __nv_bfloat16 bf16;
 enum { FB_DEVERR_NONE = 0, FB_DEVERR_WAIT_TIMEOUT = 1, FB_DEVERR_BAD_ARG = 2 };
 
 // Time limit of one device-side wait (ns); a wait that runs past it reports
-// FB_DEVERR_WAIT_TIMEOUT and makes the kernel give up.
+// FB_DEVERR_WAIT_TIMEOUT and makes the kernel give up. Each translation unit that waits
+// holds its own copy of the limit (no relocatable device code); fb_set_wait_limit_tu
+// sets the copy of the calling unit on the current device.
 #define FB_WAIT_LIMIT_NS 2000000000ull
+static __device__ unsigned long long g_fb_wait_limit_ns = FB_WAIT_LIMIT_NS;
+__device__ __forceinline__ unsigned long long fb_wait_limit() {
+  return *(volatile unsigned long long*)&g_fb_wait_limit_ns;
+}
+static inline cudaError_t fb_set_wait_limit_tu(unsigned long long ns) {
+  return cudaMemcpyToSymbol(g_fb_wait_limit_ns, &ns, sizeof(ns));
+}
 
 __device__ __forceinline__ uint64_t fb_globaltimer() {
   uint64_t t;
@@ -145,7 +154,7 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, int* e
     if (mbar_try(a, parity)) return true;
     if ((i & 63u) == 0) {
       if (*(volatile int*)err != 0) return false;
-      if (fb_globaltimer() - t0 > FB_WAIT_LIMIT_NS) {
+      if (fb_globaltimer() - t0 > fb_wait_limit()) {
         atomicExch(err, FB_DEVERR_WAIT_TIMEOUT);
         return false;
       }

@@ -144,7 +144,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             const uint32_t a = smem_u32(&full[s]);
             const uint64_t t0 = fb_globaltimer();
             while (!mbar_try(a, (issued[s] - 1) & 1u) &&
-                   fb_globaltimer() - t0 < FB_WAIT_LIMIT_NS) {
+                   fb_globaltimer() - t0 < fb_wait_limit()) {
             }
           }
       }
@@ -579,7 +579,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
             const uint64_t t0 = fb_globaltimer();
             while (*(volatile int*)ctr < n_c - 1) {
               if (*(volatile int*)err != 0) { ok2 = false; break; }
-              if (fb_globaltimer() - t0 > FB_WAIT_LIMIT_NS) {
+              if (fb_globaltimer() - t0 > fb_wait_limit()) {
                 atomicExch(err, FB_DEVERR_WAIT_TIMEOUT);
                 ok2 = false;
                 break;
@@ -931,6 +931,8 @@ bool gemm_tc_supported(const GemmArgs& g) {
          (g.kind < EPI_RESID || al16(g.epi.resid)) && (g.kind != EPI_RESID_DELTA || g.epi.resid) &&
          (g.kind != EPI_RESID_DELTA || (al16(g.epi.base) && al16(g.epi.delta)));
 }
+
+cudaError_t gemm_tc_set_wait_limit(unsigned long long ns) { return fb_set_wait_limit_tu(ns); }
 
 cudaError_t gemm_tc(const GemmArgs& g, int* err, int num_sms, cudaStream_t st, bool force_1sm) {
   if (!gemm_tc_supported(g)) return cudaErrorInvalidValue;

@@ -32,6 +32,8 @@ constexpr int SK_CTR_PER_CLUSTER = 16;
 bool gemm_tc_supported(const GemmArgs& g);
 cudaError_t gemm_tc(const GemmArgs& g, int* err, int num_sms, cudaStream_t st,
                     bool force_1sm = false);
+// Sets the gemm_tc unit's device wait limit on the current device (ns; see common.cuh).
+cudaError_t gemm_tc_set_wait_limit(unsigned long long ns);
 // CUDA-core path: requires N % 8 == 0.
 cudaError_t gemm_simt(const GemmArgs& g, cudaStream_t st);
 
@@ -51,6 +53,8 @@ cudaError_t attention(const AttnArgs& a, cudaStream_t st);
 // tcgen05/TMEM kernel: head_dim 128, 16-byte aligned rows.
 bool attention_tc_supported(const AttnArgs& a);
 cudaError_t attention_tc(const AttnArgs& a, int* err, cudaStream_t st);
+// Sets the attention_tc unit's device wait limit on the current device (ns).
+cudaError_t attention_tc_set_wait_limit(unsigned long long ns);
 
 // ---- pointwise / small kernels ------------------------------------------------------
 // out[r][:] = bf16(LN(x[r][:]) * (mul_base + mul[:]) + add[:]), x fp32 [rows][D].

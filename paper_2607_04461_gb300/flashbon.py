@@ -54,7 +54,8 @@ EXPORTS = ["fb_weights_count", "fb_weights_entry", "fb_init_model", "fb_free", "
            "fb_op_gemm", "fb_op_attention", "fb_draft_ex", "fb_refine_ex", "fb_select_elo",
            "fb_set_op_repeat", "fb_gemm_streamk_noalloc", "fb_state_bytes", "fb_state_offload",
            "fb_state_wait", "fb_set_sm_budget", "fb_sm_split_create", "fb_sm_split_info",
-           "fb_sm_split_free", "fb_pipeline_step"]
+           "fb_sm_split_free", "fb_pipeline_step", "fb_set_device_wait_limit",
+           "fb_test_fail_alloc", "fb_test_alloc_calls", "fb_test_poison_counters"]
 
 PAIR_VERIFIER = ctypes.CFUNCTYPE(ctypes.c_int, ctypes.c_void_p, ctypes.c_int, ctypes.c_int,
                                  ctypes.POINTER(ctypes.c_int))
@@ -105,6 +106,10 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
         "fb_sm_split_free": (None, [P]),
         "fb_pipeline_step": (I, [P, P, I, P, P, I, P, P, ctypes.POINTER(fb_sampler_opts),
                                  P, P, P, I, ctypes.POINTER(fb_sampler_opts)]),
+        "fb_set_device_wait_limit": (I, [ctypes.c_ulonglong]),
+        "fb_test_fail_alloc": (I, [ctypes.c_long]),
+        "fb_test_alloc_calls": (ctypes.c_long, []),
+        "fb_test_poison_counters": (I, [P]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(L, name)
@@ -360,6 +365,27 @@ def fb_set_timing(model: int, mask: int) -> None:
 
 def fb_set_op_repeat(model: int, n: int) -> None:
     _check(load_library().fb_set_op_repeat(model, int(n)))
+
+
+def fb_set_device_wait_limit(ns: int) -> None:
+    """Device-side wait limit in nanoseconds (0 = the default 2 s); a testing hook."""
+    _check(load_library().fb_set_device_wait_limit(int(ns)))
+
+
+def fb_test_fail_alloc(k: int) -> None:
+    """Makes the library's k-th device allocation from now fail (k < 0 disarms)."""
+    _check(load_library().fb_test_fail_alloc(int(k)))
+
+
+def fb_test_alloc_calls() -> int:
+    """Device allocations the library made since the last fb_test_fail_alloc."""
+    return int(load_library().fb_test_alloc_calls())
+
+
+def fb_test_poison_counters(model) -> None:
+    """Sets the stream-K counters of `model` (None: the allocation-free entry point's) to
+    a large negative value, so the next stream-K finisher's wait cannot complete."""
+    _check(load_library().fb_test_poison_counters(model))
 
 
 def fb_get_stats(model: int) -> dict:

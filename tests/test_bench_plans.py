@@ -9,6 +9,8 @@ import pytest
 ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 sys.path.insert(0, ROOT)
 import bench  # noqa: E402
+from _plans import knob_plan  # noqa: E402
+from oracle import flashbon_oracle as O  # noqa: E402
 
 
 def test_base_plan_is_the_draft_pool():
@@ -48,3 +50,11 @@ def test_full50_computes_every_block():
 def test_split_schedule_variants():
     assert set(bench.SPLIT_VARIANTS) == {"base", "sde"}
     assert bench.REFINE_SMS % 8 == 0
+
+
+def test_knob_plans_use_every_proxy_order():
+    """The plans above really forecast at the orders named (anchor counts per proxy)."""
+    an = O.resolve_plan(*knob_plan("1k"))
+    assert an[(3, 0)] == [2, 1, 0] and an[(3, 1)] == [2, 1] and an[(4, 2)] == [3, 1]
+    an = O.resolve_plan(*knob_plan("14b"))
+    assert an[(1, 0)] == [0] and an[(3, 1)] == [2, 1, 0] and an[(3, 2)] == [2]

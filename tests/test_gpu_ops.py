@@ -218,6 +218,10 @@ ATTN_CASES = [
     # grids of more than one wave of 128-query CTAs take the 256-query kernel (P in TMEM)
     (4, 1560, 1560, 12, 128, False),
     (9, 600, 512, 12, 128, True),     # last CTA: tile A partly valid, tile B past Lq
+    # the last key tile's MMAs cover only its 32-key chunks of real keys
+    (2, 384, 192, 2, 128, False),     # 64 keys in the last tile; tile B starts at Lq
+    (1, 300, 240, 2, 128, True),      # 112 keys: four chunks, the last one partial
+    (2, 100, 193, 2, 128, False),     # 65 keys: three chunks
 ]
 
 

@@ -3,6 +3,8 @@
 Small shapes are compared in full; the Wan2.1-1.3B-shaped workloads are run at full
 size in the configuration the benchmark uses and checked on sampled candidates the
 oracle computes one by one, plus properties that hold at any size."""
+import os
+
 import numpy as np
 import pytest
 import torch
@@ -10,7 +12,8 @@ import torch
 from oracle import flashbon_oracle as O
 from paper_2607_04461_gb300 import flashbon as fb
 from paper_2607_04461_gb300 import synth
-from _metrics import BLOCK_TOL, check_latents, rel_max
+from _metrics import BLOCK_TOL, COS_MIN, check_latents, cosine, rel_max
+from _plans import knob_plan
 
 pytestmark = pytest.mark.gpu
 
@@ -282,6 +285,55 @@ def test_wan13_draft_pool_full_size(wan13_pool):
     ref = O.OracleModel(cfg, w)
     want = ref.draft(z[:1], ctx, sched[:3], skip[:2], proxy[:2])
     check_latents(two.cpu().numpy()[0], want[0], z[0], label="wan13 cand 0, 2 steps")
+
+
+GOLD13 = os.path.join(os.path.dirname(os.path.abspath(__file__)), "golden", "wan13_pool_cand0.npz")
+
+
+def test_wan13_pool_whole_trajectory_matches_oracle(wan13_pool):
+    """The benchmark's whole path at full size against the oracle's trajectory of
+    candidate 0 (stored by tests/golden/make_wan13_trajectory.py, which calls only the
+    oracle): the 32-candidate draft over 10 of 50 steps with a third of the blocks
+    skipped per step and half of the rest proxied on odd steps (§4.1, Eqs. 3-7), then
+    candidate 0's draft latent refined over the remaining 40 steps with phi_full (§4.2
+    Stage 3) on the 40-SM partition the benchmark refines on. Checked after the draft,
+    after 20 refine steps and at the end."""
+    g = np.load(GOLD13)
+    cfg, w, m = wan13_pool
+    n, S = 32, 10
+    sched = synth.make_schedule(50)
+    skip, proxy = synth.random_plan(S, cfg.depth, 1 / 3, 0.5, seed=7)
+    assert np.array_equal(skip, g["skip"]) and np.array_equal(proxy, g["proxy"])
+    assert np.array_equal(sched, g["schedule"])
+    mid = int(g["refine_mid_step"])
+    z = synth.make_latents(cfg, n)
+    ctx = synth.make_text(cfg)
+    a = cuda(z)
+    m.draft(a, ctx, sched[:S + 1], skip, proxy)
+    zd = a[0].clone()
+    zd_h = zd.cpu().numpy()
+    check_latents(zd_h, g["z_draft"], z[0], label="draft, 10 steps")
+    try:
+        sp = fb.SmSplit(40)
+    except fb.FlashBonError:
+        sp = None                        # no SM partitions from the driver: whole GPU
+    try:
+        if sp is not None:
+            m.set_stream(sp.streams[0])
+            m.set_sm_budget(sp.sms[0])
+        m.refine(zd, ctx, sched[S:mid + 1])
+        zm_h = zd.cpu().numpy()
+        m.refine(zd, ctx, sched[mid:])
+        zr_h = zd.cpu().numpy()
+    finally:
+        m.set_stream(None)
+        m.set_sm_budget(0)
+        if sp is not None:
+            sp.close()
+    check_latents(zm_h, g["z_refine_mid"], z[0], label=f"refine to step {mid}")
+    check_latents(zr_h, g["z_refine"], z[0], label="refine, 40 steps")
+    # the refine's own displacement, each side from its own draft latent
+    assert cosine(zr_h - zd_h, g["z_refine"] - g["z_draft"]) >= COS_MIN
 
 
 # ---- the other shapes of the scope table: Wan2.1-14B width, 4096 tokens ---------------
@@ -701,3 +753,42 @@ def test_sm_budget_and_split_reject_bad_sizes():
         with pytest.raises(fb.FlashBonError) as e:
             fb.SmSplit(n)
         assert e.value.status == fb.FB_EINVAL
+
+
+# ---- multi-step plans with the method's knobs at the larger shapes (§4.1, Eqs. 3-7) ----
+# Three-block models keep the oracle's cost to a minute while every step mixes computed,
+# skipped and proxied blocks.
+
+def test_wan13_4096_tokens_knob_plan_matches_oracle():
+    """Wan2.1-1.3B dims at 1024x1024 (4096 tokens per candidate, 32 key tiles), three
+    blocks, N=2, five steps of a plan with skips and order-1/2 proxies: both candidates."""
+    cfg = synth.WAN13_1K.with_(depth=3, max_n=2)
+    w = synth.make_weights(cfg)
+    ctx = synth.make_text(cfg)
+    sched = synth.make_schedule(50)[:6]
+    skip, proxy = knob_plan("1k")
+    z = synth.make_latents(cfg, 2)
+    with fb.Model(cfg, w) as m:
+        a = cuda(z)
+        m.draft(a, ctx, sched, skip, proxy)
+        got = a.cpu().numpy()
+    want = O.OracleModel(cfg, w).draft(z, ctx, sched, skip, proxy)
+    for j in range(2):
+        check_latents(got[j], want[j], z[j], label=f"4096 tokens cand {j}")
+
+
+def test_wan14_width_knob_plan_matches_oracle():
+    """Wan2.1-14B dims (hidden 5120, 40 heads, FFN 13824), three blocks, four steps with
+    skips, order-0 proxies and an order-2 forecast; candidate 0 of N=2."""
+    cfg = synth.WAN14.with_(depth=3, max_n=2)
+    w = synth.make_weights(cfg)
+    ctx = synth.make_text(cfg)
+    sched = synth.make_schedule(50)[:5]
+    skip, proxy = knob_plan("14b")
+    z = synth.make_latents(cfg, 2)
+    with fb.Model(cfg, w) as m:
+        a = cuda(z)
+        m.draft(a, ctx, sched, skip, proxy)
+        got = a.cpu().numpy()
+    want = O.OracleModel(cfg, w).draft(z[:1], ctx, sched, skip, proxy)
+    check_latents(got[0], want[0], z[0], label="14B width cand 0")

@@ -80,3 +80,30 @@ def test_noalloc_rejects_what_it_cannot_run(M, N, K):
     with pytest.raises(fb.FlashBonError) as e:
         fb.fb_gemm_streamk_noalloc(None, M, N, K, None, W, None, 0, out)
     assert e.value.status == fb.FB_EINVAL
+
+
+def test_noalloc_wait_timeout_clears_its_counters(model):
+    """With the static tile counters poisoned (a large negative count, as a crashed launch
+    could leave them) a finisher waits for a count no launch reaches. With a short device
+    wait limit the call returns FB_ECUDA "device wait timed out"; it must leave the
+    counters at zero, so the next two calls match fb_op_gemm impl 4 bit for bit."""
+    M, N, K, epi = 1560, 1536, 8960, 2
+    A, W = randn((M, K), 31), randn((N, K), 32, scale=K ** -0.5)
+    bias, gate = randn((N,), 33, dtype=torch.float32), randn((N,), 34, dtype=torch.float32)
+    resid = randn((M, N), 35, dtype=torch.float32)
+    ref = torch.empty((M, N), dtype=torch.float32, device="cuda")
+    fb.fb_op_gemm(model.handle, M, N, K, A, W, bias, epi, ref, resid, gate, None, None, 4)
+    out = torch.zeros((M, N), dtype=torch.float32, device="cuda")
+    fb.fb_test_poison_counters(None)
+    fb.fb_set_device_wait_limit(20_000_000)
+    try:
+        with pytest.raises(fb.FlashBonError) as e:
+            fb.fb_gemm_streamk_noalloc(None, M, N, K, A, W, bias, epi, out, resid, gate)
+    finally:
+        fb.fb_set_device_wait_limit(0)
+    assert e.value.status == fb.FB_ECUDA and "device wait timed out" in str(e.value)
+    for _ in range(2):
+        o = torch.empty((M, N), dtype=torch.float32, device="cuda")
+        fb.fb_gemm_streamk_noalloc(None, M, N, K, A, W, bias, epi, o, resid, gate)
+        torch.cuda.synchronize()
+        assert torch.equal(o, ref)
