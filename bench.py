@@ -89,6 +89,7 @@ VARIANTS = {
     "phi_star": "",
     "full50": "",
     "wan14": "",
+    "sweep": "",
 }
 
 
@@ -242,22 +243,24 @@ def read_peaks():
     return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}, "fallback"
 
 
-def gemm_traffic_ratio():
-    """DRAM traffic / algorithmic bytes of the tcgen05 GEMM from the committed ncu summary,
-    if it was taken on the current kernel source (else None)."""
+def gemm_traffic():
+    """DRAM traffic of the tcgen05 GEMM per algorithmic byte, from the committed ncu
+    captures (profiles/gemm_tc_traffic.json), if they were taken on the current kernel
+    source; else None. Returns (combined ratio, {probe: ratio})."""
     src = os.path.join(ROOT, "paper_2607_04461_gb300", "csrc", "gemm_tc.cu")
-    summ = os.path.join(ROOT, "profiles", "gemm_tc_ffn_wan13.md")
+    summ = os.path.join(ROOT, "profiles", "gemm_tc_traffic.json")
     if not os.path.exists(summ):
         return None
     sha = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
-    vals = {}
-    for line in open(summ):
-        if line.startswith("bench-key "):
-            k, _, v = line[len("bench-key "):].partition(":")
-            vals[k.strip()] = v.strip()
-    if vals.get("kernel_sha") != sha or "traffic_ratio_to_algorithmic" not in vals:
+    with open(summ) as fh:
+        d = json.load(fh)
+    if d.get("kernel_sha") != sha:
         return None
-    return float(vals["traffic_ratio_to_algorithmic"])
+    probes = d["probes"]
+    tot_t = sum(v["dram_read_bytes"] + v["dram_write_bytes"] for v in probes.values())
+    tot_a = sum(v["algorithmic_bytes"] for v in probes.values())
+    return tot_t / tot_a, {k: (v["dram_read_bytes"] + v["dram_write_bytes"]) /
+                           v["algorithmic_bytes"] for k, v in probes.items()}
 
 
 def aggregate(ms_local, n_local, world, reduce_max=None):
@@ -471,12 +474,13 @@ def run_gb300(args):
         for k in by_phase[ph]:
             by_phase[ph][k] += cur[k] - last[0][k]
         last[0] = cur
-    e2.record(stream)
-    for _ in range(args.steps):
-        dev_step(after)
-    finish()
-    e3.record(stream)
-    torch.cuda.synchronize()
+    with ClockSampler(local) as clk2s:
+        e2.record(stream)
+        for _ in range(args.steps):
+            dev_step(after)
+        finish()
+        e3.record(stream)
+        torch.cuda.synchronize()
     stats = model.stats()
     model.set_timing(0)
     ms_instrumented = e2.elapsed_time(e3)
@@ -533,8 +537,18 @@ def run_gb300(args):
     g = stats["gemm_tc"]
     achieved = g["flops"] / (g["ms"] / 1e3) / 1e12 if g["ms"] > 0 else None
     peak = peaks["bf16_tflops_sustained"]
-    ratio = gemm_traffic_ratio()
+    tr = gemm_traffic()
+    ratio, per_probe = tr if tr else (None, None)
     traffic = ratio * g["bytes"] / g["launches"] if (ratio and g["launches"]) else None
+    n_sm = torch.cuda.get_device_properties(local).multi_processor_count
+    clk2 = clk2s.summary()
+
+    def per_clock(tflops, mhz):
+        """MACs per SM clock per SM: independent of the clock the work ran at."""
+        return tflops * 1e12 / 2 / (mhz * 1e6 * n_sm) if (tflops and mhz) else None
+    # the measured peak's own rate per clock: the sustained cuBLAS loop at its median clock
+    peak_mhz = (peaks.get("clocks_under_load") or {}).get("sm_mhz_median")
+    peak_pc = per_clock(peak, peak_mhz)
     launches = sum(s["launches"] for s in launch_stats.values())
     passes = 2 if args.variant == "cfg" else 1
     algo_flops = passes * (NC * computed_blocks(skip, proxy) * block_flops(cfg) +
@@ -553,10 +567,25 @@ def run_gb300(args):
                         "projections)", "achieved": achieved, "peak": peak,
                         "unit": "TFLOP/s", "frac": (achieved / peak) if achieved else None,
                         "peak_kind": f"bf16 sustained, {peak_kind}",
+                        "frac_burst": (achieved / peaks["bf16_tflops"]) if achieved else None,
+                        "per_clock": {
+                            "sm_mhz": clk2.get("sm_mhz"),
+                            "mac_per_clk_per_sm": per_clock(achieved, clk2.get("sm_mhz")),
+                            "peak_mac_per_clk_per_sm": peak_pc, "peak_sm_mhz": peak_mhz,
+                            "frac": (per_clock(achieved, clk2.get("sm_mhz")) / peak_pc
+                                     if (achieved and peak_pc and clk2.get("sm_mhz"))
+                                     else None),
+                            "note": "the GEMM launches' MACs per SM clock (median SM clock "
+                                    "sampled during this pass) against the sustained cuBLAS "
+                                    "loop's at its own median clock"},
                         "traffic": traffic,
-                        "traffic_note": "DRAM bytes per launch: ncu traffic/algorithmic ratio "
-                                        "of the FFN probes x this run's algorithmic bytes "
-                                        "per GEMM launch (profiles/gemm_tc_ffn_wan13.md)",
+                        "traffic_kind": "estimated" if traffic else None,
+                        "traffic_note": "DRAM bytes per launch estimated as the ncu "
+                                        "traffic/algorithmic ratio of three 8192-row probes "
+                                        "(profiles/gemm_tc_traffic.json) x this run's "
+                                        "algorithmic bytes per GEMM launch; null when the "
+                                        "kernel source differs from the captured one",
+                        "traffic_ratio_by_probe": per_probe,
                         "launches": g["launches"], "ms": g["ms"] / args.steps,
                         "measured_in": "timed pass 2 (same steps, one after the other on "
                                        "the whole GPU, per-launch CUDA events on the "
@@ -566,7 +595,10 @@ def run_gb300(args):
                                           "achieved": (v["flops"] / (v["ms"] / 1e3) / 1e12
                                                        if v["ms"] > 0 else None),
                                           "frac": (v["flops"] / (v["ms"] / 1e3) / 1e12 / peak
-                                                   if v["ms"] > 0 else None)}
+                                                   if v["ms"] > 0 else None),
+                                          "frac_burst": (v["flops"] / (v["ms"] / 1e3) / 1e12
+                                                         / peaks["bf16_tflops"]
+                                                         if v["ms"] > 0 else None)}
                                      for ph, v in by_phase.items()}},
            "step_tflops": algo_flops / (ms_step / 1e3) / 1e12,
            "step_frac_of_peak": algo_flops / (ms_step / 1e3) / 1e12 / peak,
@@ -606,7 +638,8 @@ def run_probe(args):
     (8192 x 1536 -> 8960, GELU epilogue); gemm_resid = FFN down (8192 x 8960 -> 1536,
     gated residual + contribution write); gemm_out = attention output projection
     (8192 x 1536 -> 1536, gated fp32 residual); attn = self-attention over 1560 tokens,
-    4 candidates x 12 heads x 128."""
+    4 candidates x 12 heads x 128; attn_pool = the same for the draft pool's 32
+    candidates."""
     import torch
     from paper_2607_04461_gb300 import flashbon as fb
     torch.cuda.set_device(0)
@@ -614,6 +647,9 @@ def run_probe(args):
     m = fb.Model(cfg, synth.make_weights(cfg))
     g = torch.Generator().manual_seed(0)
     rnd = lambda *s, dt=torch.bfloat16: (torch.randn(*s, generator=g) * 0.5).to(dt).cuda()  # noqa
+    if args.probe == "pointwise":
+        m.close()
+        return probe_pointwise(args)
     if args.probe in ("gemm_shapes", "attn_shapes", "breakdown"):
         call = None
     elif args.probe in ("gemm_refine_out", "gemm_refine_down"):
@@ -647,7 +683,7 @@ def run_probe(args):
             dl = torch.empty(M, D, dtype=torch.bfloat16, device="cuda")
             call = lambda: fb.fb_op_gemm(m.handle, M, D, F, A, W, b, 3, h, hb, gt, h, dl)  # noqa
     else:
-        n, P, H, dh = 4, 1560, 12, 128
+        n, P, H, dh = (32 if args.probe == "attn_pool" else 4), 1560, 12, 128
         qkv, o = rnd(n * P, 3 * H * dh), torch.empty(n * P, H * dh, dtype=torch.bfloat16, device="cuda")
         base, D = qkv.data_ptr(), H * dh
         call = lambda: fb.fb_op_attention(m.handle, base, 3 * D, base + 2 * D, 3 * D,  # noqa
@@ -799,6 +835,112 @@ def probe_breakdown(args):
     return 0
 
 
+def probe_pointwise(args):
+    """The HBM-bound kernels on a case sized for an ncu capture: a 16-candidate
+    Wan2.1-1.3B draft (24960 rows, the fp32 residual stream 153 MB, above L2) over the
+    first two steps of the bench plan (step 1 proxies), `steps` times."""
+    import torch
+    from paper_2607_04461_gb300 import flashbon as fb
+    torch.cuda.set_device(0)
+    n = 16
+    cfg, sched, skip, proxy = workload()
+    cfg = cfg.with_(max_n=n)
+    model = fb.Model(cfg, synth.make_weights(cfg))
+    z0 = torch.from_numpy(synth.make_latents(cfg, n)).cuda()
+    ctx = torch.from_numpy(synth.make_text(cfg)).cuda()
+    z = torch.empty_like(z0)
+    model.reset_stats()
+    model.set_timing((1 << len(fb.KERNEL_KINDS)) - 1)
+    for _ in range(args.steps):
+        z.copy_(z0)
+        model.draft(z, ctx, sched[:3], skip[:2], proxy[:2])
+    torch.cuda.synchronize()
+    st = {k: {"launches": v["launches"], "ms": round(v["ms"], 3),
+              "gbs": round(v["bytes"] / v["ms"] / 1e6, 1) if v["ms"] else None,
+              "bytes_per_launch": v["bytes"] / v["launches"]}
+          for k, v in model.stats().items() if v["launches"]}
+    print(json.dumps({"probe": "pointwise", "candidates": n, "stats": st}))
+    model.close()
+    return 0
+
+
+SWEEP_N = (1, 4, 16, 64)
+SWEEP_SKIP = (0.0, 0.25, 0.5)
+SWEEP_PROXY = (0.0, 0.5)
+
+
+def run_sweep(args):
+    """The 4096-token throughput sweep: Wan2.1-1.3B dims at 1024x1024 (16 x 128 x 128 latent,
+    4096 tokens), 10 draft steps of the 50-step schedule, N in SWEEP_N, a seeded fraction
+    of the blocks skipped per step (SWEEP_SKIP) and, on odd steps, a fraction of the
+    remaining blocks proxied from the previous step (SWEEP_PROXY). One JSON line per point:
+    candidates/s from `steps` timed drafts (CUDA events, inputs resident), then one draft
+    with per-launch events for the GEMM and attention rates."""
+    import torch
+    from paper_2607_04461_gb300 import flashbon as fb
+    torch.cuda.set_device(0)
+    peaks, peak_kind = read_peaks()
+    cfg = synth.WAN13_1K.with_(max_n=max(SWEEP_N))
+    model = fb.Model(cfg, synth.make_weights(cfg))
+    ctx = torch.from_numpy(synth.make_text(cfg)).cuda()
+    sched = synth.make_schedule(S_TOTAL)[: S_DRAFT + 1]
+    stream = torch.cuda.Stream()
+    model.set_stream(stream)
+    kinds = (1 << fb.K["gemm_tc"]) | (1 << fb.K["attn_self"]) | (1 << fb.K["attn_cross"])
+    for n in SWEEP_N:
+        z0 = torch.from_numpy(synth.make_latents(cfg, n)).cuda()
+        z = torch.empty_like(z0)
+        for sf in SWEEP_SKIP:
+            for pf in SWEEP_PROXY:
+                skip, proxy = synth.random_plan(S_DRAFT, cfg.depth, sf, pf, seed=PLAN_SEED)
+
+                def draft():
+                    with torch.cuda.stream(stream):
+                        z.copy_(z0)
+                    model.draft(z, ctx, sched, skip, proxy)
+                for _ in range(args.warmup):
+                    draft()
+                torch.cuda.synchronize()
+                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                with ClockSampler(0) as clk:
+                    e0.record(stream)
+                    for _ in range(args.steps):
+                        draft()
+                    e1.record(stream)
+                    torch.cuda.synchronize()
+                ms = e0.elapsed_time(e1) / args.steps
+                model.reset_stats()
+                model.set_timing(kinds)
+                draft()
+                model.set_timing(0)
+                st = model.stats()
+                flops = n * computed_blocks(skip, proxy) * block_flops(cfg)
+
+                def rate(*ks):
+                    f = sum(st[k]["flops"] for k in ks)
+                    t = sum(st[k]["ms"] for k in ks)
+                    return (f / (t / 1e3) / 1e12, t) if t else (None, 0.0)
+                g, g_ms = rate("gemm_tc")
+                a, a_ms = rate("attn_self", "attn_cross")
+                print(json.dumps({
+                    "variant": "sweep", "metric": "draft candidates/sec", "unit": "candidates/s",
+                    "value": n / (ms / 1e3), "ms_per_draft": ms, "n_candidates": n,
+                    "skip_frac": sf, "proxy_frac": pf, "tokens": cfg.tokens,
+                    "draft_steps": S_DRAFT, "computed_blocks": computed_blocks(skip, proxy),
+                    "algorithmic_tflop": flops / 1e12,
+                    "step_tflops": flops / (ms / 1e3) / 1e12,
+                    "gemm": {"tflops": g, "ms": g_ms,
+                             "frac_burst": g / peaks["bf16_tflops"] if g else None},
+                    "attention": {"tflops": a, "ms": a_ms,
+                                  "frac_burst": a / peaks["bf16_tflops"] if a else None},
+                    "peak_kind": f"bf16 burst, {peak_kind}", "clocks": clk.summary()}),
+                    flush=True)
+        del z0, z
+    model.set_stream(None)
+    model.close()
+    return 0
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -817,13 +959,16 @@ def main():
                          "or SDE steps")
     ap.add_argument("--probe", choices=["gemm", "gemm_resid", "gemm_out", "gemm_refine_out",
                                         "gemm_refine_down", "attn", "attn_mma", "gemm_shapes",
-                                        "attn_shapes", "breakdown"],
+                                        "attn_shapes", "breakdown", "pointwise",
+                                        "attn_pool"],
                     default=None)
     args = ap.parse_args()
     if args.probe:
         return run_probe(args)
     if args.impl == "reference":
         return run_reference(args)
+    if args.variant == "sweep":
+        return run_sweep(args)
     return run_gb300(args)
 
 

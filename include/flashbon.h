@@ -326,8 +326,10 @@ fb_status fb_op_gemm(fb_model* m, int M, int N, int K, const void* A, const void
  * h*head_dim; likewise K, V (kv_batch_rows = 0 shares one K/V across the batch,
  * otherwise the row offset between batches); O row stride ldo. impl: 0 = automatic
  * (the tcgen05 kernel for head_dim 128, the mma.sync kernel for 64), 1 = force the
- * mma.sync kernel, 2 / 3 = force the tcgen05 kernel with 128- / 256-query CTAs
- * (head_dim 128 only, else FB_EINVAL). */
+ * mma.sync kernel, 2 / 3 = force the tcgen05 kernel with 128- / 256-query CTAs, 4 = force
+ * the persistent 256-query kernel (at most one CTA per SM looping over the (batch, head,
+ * query-tile pair) items; the automatic choice when 256-query CTAs exceed one wave)
+ * (2-4: head_dim 128 only, else FB_EINVAL). */
 fb_status fb_op_attention(fb_model* m, const void* Q, int ldq, const void* K, int ldk,
                           const void* V, int ldv, void* O, int ldo, int batch, int Lq,
                           int Lkv, int kv_batch_rows, int heads, int head_dim, int impl);

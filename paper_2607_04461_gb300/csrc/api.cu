@@ -412,12 +412,14 @@ fb_status encode_text(fb_model* m, const float* ctx, bf16* kv_dst) {
 }
 
 // ---- per-step conditioning: temb, mod, per-layer modulation, head modulation ---------
-fb_status time_embed(fb_model* m, float t) {
+// have_emb: m->emb already holds the sinusoid of t (written by the previous step's
+// Euler kernel)
+fb_status time_embed(fb_model* m, float t, bool have_emb = false) {
   const fb_cfg& c = m->c;
   const int D = c.dim;
   KTimer k(m, FB_K_SMALL, 2.0 * D * (c.freq_dim + D + 6.0 * D),
-           2.0 * D * (c.freq_dim + D + 6.0 * D), 5);
-  CK(timestep_sincos(t, c.freq_dim, m->emb, m->st));
+           2.0 * D * (c.freq_dim + D + 6.0 * D), have_emb ? 4 : 5);
+  if (!have_emb) CK(timestep_sincos(t, c.freq_dim, m->emb, m->st));
   CK(gemv(m->time_w1, m->time_b1, m->emb, m->th1, D, c.freq_dim, 0, 1, m->st));
   CK(gemv(m->time_w2, m->time_b2, m->th1, m->temb, D, D, 0, 0, m->st));
   CK(gemv(m->mod_w, m->mod_b, m->temb, m->mod, 6 * D, D, 1, 0, m->st));
@@ -696,16 +698,23 @@ fb_status sample(fb_model* m, float* z, int n, const float* sched, int S, const 
   CKS(ensure_anchors(m, need));
   const int M = nr * m->P;
   const size_t zn = (size_t)n * c.latent_c * c.latent_h * c.latent_w;
+  // with the tensor-core head, each step's Euler kernel also writes the next step's
+  // sinusoidal embedding and patch rows (step 0 computes its own)
+  const bool fused_next = m->vbuf && m->patch_a;
   for (int k = 0; k < S; ++k) {
     const float t = sched[k], t1 = sched[k + 1];
-    CKS(time_embed(m, t));
+    const bool from_prev = fused_next && k > 0;
+    CKS(time_embed(m, t, from_prev));
     for (int u = 0; u < (so.guided ? 2 : 1); ++u) {
       float* hu = m->hA + (size_t)u * n * m->P * c.dim;
+      const bool rows_ready = from_prev || u > 0;
       KTimer kt(m, FB_K_EMBED, 2.0 * n * m->P * (double)c.dim * m->PD,
-                4.0 * n * m->P * (double)(c.dim + m->PD), m->patch_a ? 2 : 1);
+                (rows_ready ? 2.0 : 4.0) * n * m->P * (double)(c.dim + m->PD),
+                m->patch_a ? (rows_ready ? 1 : 2) : 1);
       if (m->patch_a) {
         // tensor cores: bf16 patch rows, then h = patches W_p^T + b_p (fp32, no residual)
-        CK(patchify(z, n, c.latent_c, c.latent_h, c.latent_w, c.patch, m->patch_a, m->st));
+        if (!rows_ready)
+          CK(patchify(z, n, c.latent_c, c.latent_h, c.latent_w, c.patch, m->patch_a, m->st));
         const GemmArgs g = gemm_args(n * m->P, c.dim, m->PD, m->patch_a, m->patch_w, m->patch_b,
                                      EPI_RESID, hu);
         CK(gemm_tc(g, m->derr, m->num_sms, m->st));
@@ -755,6 +764,12 @@ fb_status sample(fb_model* m, float* z, int n, const float* sched, int S, const 
         const GemmArgs g = gemm_args(M, m->npad, c.dim, m->act, m->head_wp, m->head_bp, EPI_RESID,
                                      m->vbuf);
         CK(gemm_tc(g, m->derr, m->num_sms, m->st));
+        if (k + 1 < S && m->patch_a) {
+          hs.patch_next = m->patch_a;
+          hs.emb_next = m->emb;
+          hs.t_next = t1;
+          hs.freq_dim = c.freq_dim;
+        }
         CK(euler_step(m->vbuf, m->npad, n, c.latent_c, c.latent_h, c.latent_w, c.patch, hs, z,
                       m->st));
       } else {
@@ -1306,7 +1321,7 @@ fb_status fb_op_attention(fb_model* m, const void* Q, int ldq, const void* K, in
                           const void* V, int ldv, void* O, int ldo, int batch, int Lq, int Lkv,
                           int kv_batch_rows, int heads, int head_dim, int impl) {
   if (!m || !Q || !K || !V || !O) return fail(FB_EINVAL, "null argument");
-  if (impl < 0 || impl > 3) return fail(FB_EINVAL, "impl must be 0 .. 3");
+  if (impl < 0 || impl > 4) return fail(FB_EINVAL, "impl must be 0 .. 4");
   if (batch < 1 || Lq < 1 || Lkv < 1 || heads < 1 || (head_dim != 64 && head_dim != 128))
     return fail(FB_EINVAL, "bad sizes");
   AttnArgs a{};

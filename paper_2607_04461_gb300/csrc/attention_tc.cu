@@ -45,6 +45,7 @@ struct Params {
   int ldo;
   float scale_log2;
   int* err;
+  int batch, heads;  // the persistent kernel's item count
 };
 
 __device__ __forceinline__ uint64_t desc_k_sw128(uint32_t saddr) {
@@ -734,6 +735,344 @@ __global__ void __launch_bounds__(THREADS2, 1)
   }
 }
 
+// ---- persistent 256-query kernel ----------------------------------------------------
+// attn_tc2_kernel's computation with at most one CTA per SM, each looping over items
+// (batch b, head h, query-tile pair qb), qb fastest so that the CTAs running at the same
+// time share their K/V tiles in L2. Per CTA the work of consecutive items overlaps:
+//  * the producer loads the next item's Q as soon as the current item's last S MMAs are
+//    done (q_empty) and carries on through the K/V rings, whose slots and phases count
+//    across items;
+//  * the MMA issuer starts the next item's S MMAs right after the current item's last PV
+//    (the tensor pipe runs in order, so S_g overwrites P_g only after PV_g has read it);
+//  * each softmax group stores its O rows (o_done, one phase per item of the group) while
+//    those S MMAs run; its first P of the next item is announced only after those TMEM
+//    reads, so the first PV of the next item (accumulate = 0) cannot overwrite O early.
+// Group B has no work in items whose second query tile lies past Lq; the issuer and the
+// group count the phases of their own barriers.
+__global__ void __launch_bounds__(THREADS2, 1)
+    attn_tc2p_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
+                     const __grid_constant__ CUtensorMap tmV, Params p) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint8_t* Qs = smem;                  // [2 tiles][2 sub-tiles]
+  uint8_t* Ks = smem + 2 * Q_BYTES;
+  uint8_t* Vs = Ks + KSLOT * K_BYTES;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(Vs + VSLOT * V_BYTES);
+  uint64_t* q_full = bars;
+  uint64_t* q_empty = bars + 1;
+  uint64_t* k_full = bars + 2;         // [3]
+  uint64_t* k_empty = bars + 5;        // [3]
+  uint64_t* v_full = bars + 8;         // [2]
+  uint64_t* v_empty = bars + 10;       // [2]
+  uint64_t* s_full = bars + 12;        // [2 groups]
+  uint64_t* p_full = bars + 14;        // [2 groups]
+  uint64_t* o_done = bars + 16;        // [2 groups]
+  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(bars + 18);
+
+  const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+  const int n_kv = (p.Lkv + TB - 1) / TB;
+  const int nqb = (p.Lq + 2 * TB - 1) / (2 * TB);
+  const int n_items = nqb * p.heads * p.batch;
+  int* err = p.err;
+  bool failed = false;
+
+  if (threadIdx.x == 0) {
+    mbar_init(q_full, 1);
+    mbar_init(q_empty, 1);
+    for (int s = 0; s < KSLOT; ++s) {
+      mbar_init(&k_full[s], 1);
+      mbar_init(&k_empty[s], 1);
+    }
+    for (int s = 0; s < 2; ++s) {
+      mbar_init(&v_full[s], 1);
+      mbar_init(&v_empty[s], 1);
+      mbar_init(&s_full[s], 1);
+      mbar_init(&p_full[s], 4);
+      mbar_init(&o_done[s], 1);
+    }
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    tma_prefetch_desc(&tmQ);
+    tma_prefetch_desc(&tmK);
+    tma_prefetch_desc(&tmV);
+  }
+  if (warp == 1) tmem_alloc(tmem_holder, TMEM_COLS);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_holder;
+  griddep_wait();
+  griddep_launch();
+
+  if (warp == 0) {
+    // ---------------- TMA producers: lane 0 Q and K, lane 1 V ----------------
+    if (lane == 0) {
+      uint32_t kt = 0;  // K tiles loaded by this CTA
+      int it = 0;
+      for (int item = blockIdx.x; item < n_items && !failed; item += gridDim.x, ++it) {
+        const int qb = item % nqb, bh = item / nqb, h = bh % p.heads, b = bh / p.heads;
+        const int xq = h * 128, q_row0 = b * p.Lq + qb * 2 * TB, kv_row0 = b * p.kv_batch_rows;
+        const int ng = qb * 2 * TB + TB < p.Lq ? 2 : 1;
+        if (!mbar_wait(q_empty, (it & 1) ^ 1u, err)) { failed = true; break; }
+        mbar_expect_tx(q_full, ng * Q_BYTES);
+        for (int g = 0; g < ng; ++g) {
+          tma_load_2d(Qs + g * Q_BYTES, &tmQ, q_full, xq, q_row0 + g * TB);
+          tma_load_2d(Qs + g * Q_BYTES + SUB, &tmQ, q_full, xq + 64, q_row0 + g * TB);
+        }
+        for (int j = 0; j < n_kv; ++j, ++kt) {
+          const int s = kt % KSLOT;
+          if (!mbar_wait(&k_empty[s], ((kt / KSLOT) & 1) ^ 1u, err)) { failed = true; break; }
+          uint8_t* st = Ks + s * K_BYTES;
+          const int y = kv_row0 + j * TB;
+          mbar_expect_tx(&k_full[s], K_BYTES);
+          tma_load_2d(st, &tmK, &k_full[s], xq, y);
+          tma_load_2d(st + SUB, &tmK, &k_full[s], xq + 64, y);
+        }
+      }
+    } else if (lane == 1) {
+      uint32_t vt = 0;  // V tiles loaded by this CTA
+      for (int item = blockIdx.x; item < n_items && !failed; item += gridDim.x) {
+        const int bh = item / nqb, h = bh % p.heads, b = bh / p.heads;
+        const int xq = h * 128, kv_row0 = b * p.kv_batch_rows;
+        for (int j = 0; j < n_kv; ++j, ++vt) {
+          const int s = vt & 1;
+          if (!mbar_wait(&v_empty[s], ((vt >> 1) & 1) ^ 1u, err)) { failed = true; break; }
+          uint8_t* st = Vs + s * V_BYTES;
+          const int y = kv_row0 + j * TB;
+          mbar_expect_tx(&v_full[s], V_BYTES);
+          tma_load_2d(st, &tmV, &v_full[s], xq, y);
+          tma_load_2d(st + SUB, &tmV, &v_full[s], xq + 64, y);
+        }
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      const uint32_t idesc_s = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(TB >> 3) << 17) |
+                               ((uint32_t)(TB >> 4) << 24);
+      const uint32_t idesc_pv = idesc_s | (1u << 16);
+      const uint32_t qa = smem_u32(Qs);
+      const int last_nch = (p.Lkv - (n_kv - 1) * TB + 31) >> 5;
+      uint32_t kb = 0, vb = 0, pc[2] = {0u, 0u};  // K, V tiles and P tiles (per group) consumed
+      bool ok = true;
+      int it = 0;
+      // S_g of key tile j (K ring slot of tile kb + j); the last group's S of a tile frees
+      // its K slot, and of the last tile also the Q buffer
+      auto issue_s = [&](int g, int j, int ng) {
+        const uint32_t kt = kb + j;
+        const uint32_t ka = smem_u32(Ks + (kt % KSLOT) * K_BYTES);
+        const uint32_t qg = qa + g * Q_BYTES;
+        if (j + 1 < n_kv || last_nch == 4) {
+#pragma unroll
+          for (int kk = 0; kk < 8; ++kk) {
+            const uint32_t off = (kk >> 2) * SUB + (kk & 3) * 32;
+            tc_mma_f16(tmem + g * TB, desc_k_sw128(qg + off), desc_k_sw128(ka + off), idesc_s,
+                       kk ? 1u : 0u);
+          }
+        } else {
+          const uint32_t idesc = idesc_keys(idesc_s, last_nch);
+#pragma unroll 1
+          for (int kk = 0; kk < 8; ++kk) {
+            const uint32_t off = (kk >> 2) * SUB + (kk & 3) * 32;
+            tc_mma_f16(tmem + g * TB, desc_k_sw128(qg + off), desc_k_sw128(ka + off), idesc,
+                       kk ? 1u : 0u);
+          }
+        }
+        tc_commit(&s_full[g]);
+        if (g == ng - 1) {
+          tc_commit(&k_empty[kt % KSLOT]);
+          if (j == n_kv - 1) tc_commit(q_empty);
+        }
+      };
+      auto issue_pv = [&](int g, int j) {
+        const uint32_t va = smem_u32(Vs + ((vb + j) & 1) * V_BYTES);
+        if (j + 1 < n_kv || last_nch == 4) {
+#pragma unroll
+          for (int kk = 0; kk < 8; ++kk)
+            tc_mma_f16_ts(tmem + O_COL + g * TB, tmem + g * TB + kk * 8,
+                          desc_mn_sw128(va + kk * 2048, SUB), idesc_pv, (j | kk) ? 1u : 0u);
+        } else {
+#pragma unroll 1
+          for (int kk = 0; kk < 2 * last_nch; ++kk)
+            tc_mma_f16_ts(tmem + O_COL + g * TB, tmem + g * TB + kk * 8,
+                          desc_mn_sw128(va + kk * 2048, SUB), idesc_pv, (j | kk) ? 1u : 0u);
+        }
+      };
+      for (int item = blockIdx.x; item < n_items && ok; item += gridDim.x, ++it) {
+        const int qb = item % nqb;
+        const int ng = qb * 2 * TB + TB < p.Lq ? 2 : 1;
+        if (!(ok = mbar_wait(q_full, it & 1, err))) break;
+        if (!(ok = mbar_wait(&k_full[kb % KSLOT], (kb / KSLOT) & 1, err))) break;
+        tc_fence_after();
+        for (int g = 0; g < ng; ++g) issue_s(g, 0, ng);
+        for (int j = 0; j < n_kv && ok; ++j) {
+          const bool more = j + 1 < n_kv;
+          const uint32_t vt = vb + j;
+          if (!(ok = mbar_wait(&p_full[0], pc[0]++ & 1, err))) break;
+          if (!(ok = mbar_wait(&v_full[vt & 1], (vt >> 1) & 1, err))) break;
+          tc_fence_after();
+          issue_pv(0, j);
+          if (ng == 1) tc_commit(&v_empty[vt & 1]);
+          if (more) {
+            const uint32_t kt = kb + j + 1;
+            if (!(ok = mbar_wait(&k_full[kt % KSLOT], (kt / KSLOT) & 1, err))) break;
+            tc_fence_after();
+            issue_s(0, j + 1, ng);
+          }
+          if (ng == 1) continue;
+          if (!(ok = mbar_wait(&p_full[1], pc[1]++ & 1, err))) break;
+          tc_fence_after();
+          issue_pv(1, j);
+          tc_commit(&v_empty[vt & 1]);
+          if (more) issue_s(1, j + 1, ng);
+        }
+        if (!ok) break;
+        for (int g = 0; g < ng; ++g) tc_commit(&o_done[g]);
+        kb += n_kv;
+        vb += n_kv;
+      }
+      failed = !ok;
+    }
+  } else {
+    // ---------------- softmax groups: warps 2-5 -> tile A, warps 6-9 -> tile B ----------
+    const int g = (warp - 2) >> 2;
+    const int quarter = warp & 3;
+    const int r = quarter * 32 + lane;
+    const uint32_t lane_base = tmem + ((uint32_t)(quarter * 32) << 16);
+    const uint32_t s_col = g * TB, o_col = O_COL + g * TB;
+    uint32_t cnt = 0;  // items this group has worked on
+    for (int item = blockIdx.x; item < n_items && !failed; item += gridDim.x) {
+      const int qb = item % nqb;
+      if (qb * 2 * TB + g * TB >= p.Lq) continue;  // this tile lies past Lq: no work
+      float m_used = -INFINITY, l = 0.f;
+      for (int j = 0; j < n_kv; ++j) {
+        const bool ok = mbar_wait(&s_full[g], (cnt * (uint32_t)n_kv + j) & 1, err);
+        if (!__all_sync(0xffffffffu, ok)) { failed = true; break; }
+        tc_fence_after();
+        float s[128];
+        {
+          uint32_t u[128];
+#pragma unroll
+          for (int c = 0; c < 4; ++c) tmem_ld32(lane_base + s_col + c * 32, u + c * 32);
+          tmem_ld_wait();
+#pragma unroll
+          for (int c = 0; c < 4; ++c) reg_fence32(u + c * 32);
+#pragma unroll
+          for (int i = 0; i < 128; ++i) s[i] = __uint_as_float(u[i]);
+        }
+        const int valid = p.Lkv - j * TB;
+        if (valid < TB) {
+#pragma unroll
+          for (int i = 0; i < 128; ++i)
+            if (i >= valid) s[i] = -INFINITY;
+        }
+        const float mx = rowmax128(s) * p.scale_log2;
+        if (j == 0) {
+          m_used = mx;
+        } else if (__any_sync(0xffffffffu, mx > m_used + 8.f)) {
+          const float m_new = fmaxf(m_used, mx);
+          const float alpha = ex2(m_used - m_new);
+          m_used = m_new;
+          l *= alpha;
+#pragma unroll 1
+          for (int c = 0; c < 4; ++c) {
+            uint32_t u[32];
+            tmem_ld32(lane_base + o_col + c * 32, u);
+            tmem_ld_wait();
+            reg_fence32(u);
+#pragma unroll
+            for (int i = 0; i < 32; ++i) u[i] = __float_as_uint(__uint_as_float(u[i]) * alpha);
+            tmem_st32(lane_base + o_col + c * 32, u);
+          }
+        }
+        const uint64_t sc2 = f2_pack(p.scale_log2, p.scale_log2);
+        const uint64_t nm2 = f2_pack(-m_used, -m_used);
+        uint64_t ls2[2] = {0ull, 0ull};  // independent partial sums
+        // keys 0-63 from the registers; P of those keys fills TMEM columns 0-31 only, so
+        // keys 64-127 are read again from their S columns instead of staying live in
+        // registers through the first half (register room for the item loop)
+#pragma unroll
+        for (int c = 0; c < 2; ++c) {
+          float h[64];
+          if (c == 0) {
+#pragma unroll
+            for (int i = 0; i < 64; ++i) h[i] = s[i];
+          } else {
+            uint32_t u2[64];
+            tmem_ld32(lane_base + s_col + 64, u2);
+            tmem_ld32(lane_base + s_col + 96, u2 + 32);
+            tmem_ld_wait();
+            reg_fence32(u2);
+            reg_fence32(u2 + 32);
+#pragma unroll
+            for (int i = 0; i < 64; ++i) h[i] = __uint_as_float(u2[i]);
+            if (valid < TB) {
+#pragma unroll
+              for (int i = 0; i < 64; ++i)
+                if (64 + i >= valid) h[i] = -INFINITY;
+            }
+          }
+          uint32_t u[32];
+#pragma unroll
+          for (int i = 0; i < 32; ++i) {
+            float t0, t1;
+            f2_unpack(f2_fma(f2_pack(h[2 * i], h[2 * i + 1]), sc2, nm2), t0, t1);
+            const float e0 = ex2(t0), e1 = ex2(t1);
+            ls2[i & 1] = f2_add(ls2[i & 1], f2_pack(e0, e1));
+            u[i] = pack_bf16x2(e0, e1);
+          }
+          tmem_st32(lane_base + s_col + c * 32, u);
+        }
+        {
+          float a0, a1;
+          f2_unpack(f2_add(ls2[0], ls2[1]), a0, a1);
+          l += a0 + a1;
+        }
+        tmem_st_wait();
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&p_full[g]);
+      }
+      if (failed) break;
+      // the item's O rows: PV_g of its last key tile done
+      const bool ok = mbar_wait(&o_done[g], cnt & 1, err);
+      if (!__all_sync(0xffffffffu, ok)) { failed = true; break; }
+      tc_fence_after();
+      const int bh = item / nqb, h = bh % p.heads, b = bh / p.heads;
+      const float inv = 1.f / l;
+      const int qrow = qb * 2 * TB + g * TB + r;
+      bf16* orow = p.O + (size_t)(b * p.Lq + qrow) * p.ldo + h * 128;
+#pragma unroll 1
+      for (int c = 0; c < 4; ++c) {
+        uint32_t u[32];
+        tmem_ld32(lane_base + o_col + c * 32, u);
+        tmem_ld_wait();
+        reg_fence32(u);
+        if (qrow < p.Lq) {
+#pragma unroll
+          for (int q = 0; q < 4; ++q) {
+            float v[8];
+#pragma unroll
+            for (int i = 0; i < 8; ++i) v[i] = __uint_as_float(u[q * 8 + i]) * inv;
+            store_bf16x8(orow + c * 32 + q * 8, v);
+          }
+        }
+      }
+      ++cnt;
+    }
+  }
+
+  if (failed || *(volatile int*)err != 0) {
+    const uint64_t t0 = fb_globaltimer();
+    while (fb_globaltimer() - t0 < 100000ull) __nanosleep(1000);
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, TMEM_COLS);
+  }
+}
+
 PFN_cuTensorMapEncodeTiled_v12000 encoder() {
   // looked up once; a function-local static is initialised thread-safely (the bench
   // drives two models from two host threads)
@@ -795,15 +1134,28 @@ cudaError_t attention_tc(const AttnArgs& a, int* err, cudaStream_t st) {
   p.ldo = a.ldo;
   p.scale_log2 = 1.4426950408889634f / sqrtf(128.f);
   p.err = err;
+  p.batch = a.batch;
+  p.heads = a.heads;
   // 256-query CTAs share each K/V tile between two query tiles and overlap one tile's
-  // softmax with the other's MMAs; one costs about 1.7 times a 128-query CTA in steady
-  // state (one CTA per SM either way). The choice compares waves: on 152 SMs, 1 x 1560
-  // queries x 12 heads is 2 waves of 128-query CTAs (156) or 1 of 256-query CTAs (84,
-  // 18 % faster); on a 40-SM partition it is 4 waves against 3 (1.7 x 3 > 4).
+  // softmax with the other's MMAs; one costs about 1.4 times a 128-query CTA (measured:
+  // 4 x 1560 queries x 12 heads, 5 waves of 128-query CTAs 93.8 us, 3 waves of 256-query
+  // CTAs 79.8 us). The choice compares waves (for the persistent kernel, items per CTA):
+  // on 152 SMs, 1 x 1560 queries x 12 heads is 2 waves of 128-query CTAs (156) or 1 of
+  // 256-query CTAs (84); on a 40-SM partition it is 4 waves against 3 (1.4 x 3 > 4).
   const long ctas1 = (long)((a.Lq + TB - 1) / TB) * a.heads * a.batch;
   const long ctas2 = (long)((a.Lq + 2 * TB - 1) / (2 * TB)) * a.heads * a.batch;
   const long w1 = (ctas1 + sms - 1) / sms, w2 = (ctas2 + sms - 1) / sms;
-  const bool two = a.tc_variant == 2 || (a.tc_variant == 0 && 10 * w1 >= 17 * w2);
+  const bool two = a.tc_variant >= 2 || (a.tc_variant == 0 && 10 * w1 >= 14 * w2);
+  // more than one wave of 256-query CTAs: one persistent CTA per SM loops over them
+  if (a.tc_variant == 3 || (two && a.tc_variant == 0 && ctas2 > sms)) {
+    cudaError_t e = cudaFuncSetAttribute(attn_tc2p_kernel,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM2_BYTES);
+    if (e != cudaSuccess) return e;
+    const int grid = (int)(ctas2 < sms ? ctas2 : sms);
+    e = launch_k(attn_tc2p_kernel, dim3(grid), dim3(THREADS2), SMEM2_BYTES, st, mq, mk, mv, p);
+    if (e != cudaSuccess) return e;
+    return cudaGetLastError();
+  }
   if (two) {
     cudaError_t e = cudaFuncSetAttribute(attn_tc2_kernel,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM2_BYTES);

@@ -45,7 +45,8 @@ struct AttnArgs {
   int batch, Lq, Lkv;
   int kv_batch_rows;       // row offset of batch b's K/V (0 = shared)
   int heads, head_dim;
-  int tc_variant;          // tcgen05 kernel: 0 automatic, 1 128-query CTAs, 2 256-query CTAs
+  int tc_variant;          // tcgen05 kernel: 0 automatic, 1 128-query CTAs, 2 256-query CTAs,
+                           // 3 the persistent 256-query kernel
   int sms;                 // SMs the launch may use (its choice of CTA size); 0: the device's
 };
 // mma.sync (warp-level) kernel: head_dim 64 or 128.
@@ -85,6 +86,13 @@ struct HeadStep {
   float dt, t, w, sde_c, nscale;
   int uncond_rows;        // 0: no guidance
   const float* noise;     // null: ODE step
+  // euler_step only: the next step's conditioning, written from the updated z (null: last
+  // step). patch_next: bf16 patch rows (as patchify writes them); emb_next: the sinusoidal
+  // embedding of t_next (as timestep_sincos writes it, freq_dim entries).
+  bf16* patch_next;
+  float* emb_next;
+  float t_next;
+  int freq_dim;
 };
 cudaError_t head_euler(const bf16* a, int n, int C, int H, int W, int p, const bf16* Wh,
                        const float* bh, int D, const HeadStep& hs, float* z, cudaStream_t st);
@@ -93,7 +101,9 @@ cudaError_t head_euler(const bf16* a, int n, int C, int H, int W, int p, const b
 cudaError_t patchify(const float* z, int n, int C, int H, int W, int p, bf16* out,
                      cudaStream_t st);
 // The guidance combination and step of head_euler, with v[row][o] (fp32, leading dimension
-// ldv >= C p p) the head output a Wh^T + bh computed by the tensor-core GEMM.
+// ldv >= C p p) the head output a Wh^T + bh computed by the tensor-core GEMM; with
+// hs.patch_next / hs.emb_next also the next step's patch rows and timestep embedding
+// (C p p % 8 == 0).
 cudaError_t euler_step(const float* v, int ldv, int n, int C, int H, int W, int p,
                        const HeadStep& hs, float* z, cudaStream_t st);
 // y[o] = act_out(b[o] + sum_k W[o][k] act_in(x[k])), act: 0 none, 1 SiLU.

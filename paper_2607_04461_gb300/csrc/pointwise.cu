@@ -241,35 +241,56 @@ __global__ void __launch_bounds__(256) patchify_kernel(const float* __restrict__
 }
 
 // euler_step: the guidance combination and the ODE / SDE step of head_euler, from the
-// head output v[row][o] (bias included) of the tensor-core head GEMM. Thread -> one
-// element (b, ch, y, x) of z, which reads output o = (ch, y % p, x % p) of token
-// (y / p, x / p) of candidate b.
+// head output v[row][o] (bias included) of the tensor-core head GEMM, fused with the next
+// step's conditioning inputs: the bf16 patch rows of the updated z (the A operand of the
+// next patch embedding) and the sinusoidal embedding of the next t. One block per token
+// row (p latent rows) of one candidate: threads walk the latent in memory order (each
+// element reads output o = (ch, y % p, x % p) of token x / p), then the updated values
+// leave through a shared-memory tile [token][o] as whole 16-byte patch-row chunks.
+__device__ __forceinline__ void sincos_entry(float t, int k, int half, float* emb) {
+  // f_k = 10000^(-k/half); the argument is formed in double for accuracy at 1000 t
+  const double f = exp(-9.210340371976184 * (double)k / (double)half);
+  const double arg = 1000.0 * (double)t * f;
+  emb[k] = (float)cos(arg);
+  emb[half + k] = (float)sin(arg);
+}
+
 __global__ void __launch_bounds__(256) euler_step_kernel(const float* __restrict__ v, int ldv,
                                                          int n, int C, int H, int W, int p,
                                                          HeadStep hs, float* __restrict__ z) {
+  extern __shared__ float tile[];  // [W / p tokens][C p p] when hs.patch_next
   griddep_wait();
   griddep_launch();
-  const int gw = W / p, P = (H / p) * gw;
-  const size_t total = (size_t)n * C * H * W;
-  for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < total;
-       i += (size_t)gridDim.x * blockDim.x) {
-    const int x = (int)(i % W);
-    size_t t = i / W;
-    const int y = (int)(t % H);
-    t /= H;
-    const int ch = (int)(t % C), b = (int)(t / C);
-    const size_t tok = (size_t)b * P + (y / p) * gw + x / p;
-    const int o = (ch * p + y % p) * p + x % p;
-    float vv = v[tok * ldv + o];
+  const int PD = C * p * p, gw = W / p, gh = H / p, P = gh * gw;
+  const int r = blockIdx.x % gh, b = blockIdx.x / gh;  // token row r of candidate b
+  if (hs.emb_next && blockIdx.x == 0) {
+    const int half = hs.freq_dim / 2;
+    for (int k = threadIdx.x; k < half; k += blockDim.x)
+      sincos_entry(hs.t_next, k, half, hs.emb_next);
+  }
+  const size_t tok0 = (size_t)b * P + (size_t)r * gw;  // first token of the row
+  const int row_elems = C * p * W;                      // (ch, dy, x) of the p latent rows
+  for (int e = threadIdx.x; e < row_elems; e += blockDim.x) {
+    const int x = e % W, dy = (e / W) % p, ch = e / (W * p);
+    const size_t zi = (((size_t)b * C + ch) * H + (size_t)r * p + dy) * W + x;
+    const int tok = x / p, o = (ch * p + dy) * p + x % p;
+    float vv = v[(tok0 + tok) * ldv + o];
     if (hs.uncond_rows) {
-      const float vu = v[(tok + hs.uncond_rows) * ldv + o];
+      const float vu = v[(tok0 + tok + hs.uncond_rows) * ldv + o];
       vv = vu + hs.w * (vv - vu);
     }
-    const float zo = z[i];
-    if (hs.noise)
-      z[i] = zo + (vv + hs.sde_c * (zo + (1.f - hs.t) * vv)) * hs.dt + hs.nscale * hs.noise[i];
-    else
-      z[i] = zo + hs.dt * vv;
+    const float zo = z[zi];
+    const float zn = hs.noise ? zo + (vv + hs.sde_c * (zo + (1.f - hs.t) * vv)) * hs.dt +
+                                    hs.nscale * hs.noise[zi]
+                              : zo + hs.dt * vv;
+    z[zi] = zn;
+    if (hs.patch_next) tile[tok * PD + o] = zn;
+  }
+  if (!hs.patch_next) return;
+  __syncthreads();
+  for (int c = threadIdx.x; c < gw * (PD / 8); c += blockDim.x) {
+    const int tok = c / (PD / 8), o0 = (c % (PD / 8)) * 8;
+    store_bf16x8(hs.patch_next + (tok0 + tok) * PD + o0, tile + tok * PD + o0);
   }
 }
 
@@ -379,13 +400,7 @@ __global__ void timestep_sincos_kernel(float t, int dim, float* emb) {
   griddep_wait();
   griddep_launch();
   const int half = dim / 2;
-  for (int k = threadIdx.x; k < half; k += blockDim.x) {
-    // f_k = 10000^(-k/half); the argument is formed in double for accuracy at 1000 t
-    const double f = exp(-9.210340371976184 * (double)k / (double)half);
-    const double arg = 1000.0 * (double)t * f;
-    emb[k] = (float)cos(arg);
-    emb[half + k] = (float)sin(arg);
-  }
+  for (int k = threadIdx.x; k < half; k += blockDim.x) sincos_entry(t, k, half, emb);
 }
 
 __global__ void mod_prepare_kernel(const float* __restrict__ mod,
@@ -472,11 +487,13 @@ cudaError_t patchify(const float* z, int n, int C, int H, int W, int p, bf16* ou
 
 cudaError_t euler_step(const float* v, int ldv, int n, int C, int H, int W, int p,
                        const HeadStep& hs, float* z, cudaStream_t st) {
-  if (H % p || W % p || ldv < C * p * p) return cudaErrorInvalidValue;
-  const size_t work = (size_t)n * C * H * W;
-  if (work == 0) return cudaSuccess;
-  return launch_k(euler_step_kernel, dim3(grid_for(work, 256)), dim3(256), 0, st, v, ldv, n, C, H,
-                  W, p, hs, z);
+  const int PD = C * p * p;
+  if (H % p || W % p || ldv < PD || PD % 8) return cudaErrorInvalidValue;
+  const size_t smem = hs.patch_next ? (size_t)(W / p) * PD * sizeof(float) : 0;
+  if (smem > 48 * 1024) return cudaErrorInvalidValue;  // one token row's tile
+  if (n == 0) return cudaSuccess;
+  return launch_k(euler_step_kernel, dim3(n * (H / p)), dim3(256), smem, st, v, ldv, n, C, H, W, p,
+                  hs, z);
 }
 
 cudaError_t proxy_add(float* h, size_t n_elems, const ProxyTerms& t, cudaStream_t st) {

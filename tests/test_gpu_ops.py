@@ -222,10 +222,13 @@ ATTN_CASES = [
     (2, 384, 192, 2, 128, False),     # 64 keys in the last tile; tile B starts at Lq
     (1, 300, 240, 2, 128, True),      # 112 keys: four chunks, the last one partial
     (2, 100, 193, 2, 128, False),     # 65 keys: three chunks
+    # persistent 256-query CTAs: several items per CTA, one- and two-tile items mixed
+    (12, 1560, 1560, 12, 128, False),
+    (8, 300, 240, 12, 128, True),
 ]
 
 
-@pytest.mark.parametrize("impl", [0, 3], ids=["auto", "tc_q256"])
+@pytest.mark.parametrize("impl", [0, 3, 4], ids=["auto", "tc_q256", "tc_q256_persistent"])
 def test_attention_large_logits(model, impl):
     """Scores spanning many powers of two exercise the rescaling of O."""
     batch, L, heads, dh = 2, 400, 2, 128
@@ -244,7 +247,8 @@ def test_attention_large_logits(model, impl):
         assert rel_max(on[sl], want) <= 2e-2
 
 
-@pytest.mark.parametrize("impl", [0, 1, 2, 3], ids=["auto", "mma_sync", "tc_q128", "tc_q256"])
+@pytest.mark.parametrize("impl", [0, 1, 2, 3, 4],
+                         ids=["auto", "mma_sync", "tc_q128", "tc_q256", "tc_q256_persistent"])
 @pytest.mark.parametrize("batch,Lq,Lkv,heads,dh,shared", ATTN_CASES)
 def test_attention(model, batch, Lq, Lkv, heads, dh, shared, impl):
     D = heads * dh
