@@ -120,6 +120,7 @@ __device__ __forceinline__ uint64_t f2_add(uint64_t a, uint64_t b) {
   return d;
 }
 
+
 __device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t* r) {
   asm volatile(
       "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], "
@@ -139,9 +140,60 @@ __device__ __forceinline__ void fence_async_smem() {
   asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
 
+__device__ __forceinline__ void tma_store_3d(const CUtensorMap* map, uint32_t src, int x, int y,
+                                             int z) {
+  asm volatile("cp.async.bulk.tensor.3d.global.shared::cta.bulk_group [%0, {%2, %3, %4}], [%1];"
+               ::"l"(reinterpret_cast<uint64_t>(map)), "r"(src), "r"(x), "r"(y), "r"(z)
+               : "memory");
+}
+
+// The O rows of one warp (lane = row y0 + lane of batch b, its 128 columns at TMEM address
+// t_o) to global memory: scaled by inv, rounded to bf16, written into a 4 KB staging tile
+// (32 rows x 64 columns in the TMA 128-byte swizzle: 16-byte chunk c of row r at chunk
+// position c ^ (r & 7), so a warp's writes fall in distinct banks) and stored by two 3-D
+// TMA stores (64 columns each) that drop rows at or past Lq. Whole 128-byte row segments
+// reach memory instead of one 16-byte piece per row per store instruction. Lane 0 waits
+// until the first store has read the tile before it is refilled; the caller waits for the
+// stores (bulk_wait) before the CTA exits or before the tile is used again.
+__device__ __forceinline__ void store_o_warp(uint8_t* stage, const CUtensorMap* tmO, uint32_t t_o,
+                                             float inv, int x0, int y0, int b, int Lq, int lane) {
+  if (y0 >= Lq) return;  // every row of this warp lies past Lq
+#pragma unroll 1
+  for (int half = 0; half < 2; ++half) {
+    uint32_t u[64];
+    tmem_ld32(t_o + half * 64, u);
+    tmem_ld32(t_o + half * 64 + 32, u + 32);
+    tmem_ld_wait();
+    reg_fence32(u);
+    reg_fence32(u + 32);
+    if (half == 1) {
+      if (lane == 0) bulk_wait_read<0>();
+      __syncwarp();
+    }
+    uint8_t* row = stage + lane * 128;
+#pragma unroll
+    for (int c = 0; c < 8; ++c) {
+      uint4 w;
+      w.x = pack_bf16x2(__uint_as_float(u[8 * c + 0]) * inv, __uint_as_float(u[8 * c + 1]) * inv);
+      w.y = pack_bf16x2(__uint_as_float(u[8 * c + 2]) * inv, __uint_as_float(u[8 * c + 3]) * inv);
+      w.z = pack_bf16x2(__uint_as_float(u[8 * c + 4]) * inv, __uint_as_float(u[8 * c + 5]) * inv);
+      w.w = pack_bf16x2(__uint_as_float(u[8 * c + 6]) * inv, __uint_as_float(u[8 * c + 7]) * inv);
+      *reinterpret_cast<uint4*>(row + ((c ^ (lane & 7)) * 16)) = w;
+    }
+    fence_async_smem();
+    __syncwarp();
+    if (lane == 0) {
+      tma_store_3d(tmO, smem_u32(stage), x0 + half * 64, y0, b);
+      bulk_commit();
+    }
+  }
+}
+
+
 __global__ void __launch_bounds__(THREADS, 1)
     attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
-                   const __grid_constant__ CUtensorMap tmV, Params p) {
+                   const __grid_constant__ CUtensorMap tmV,
+                   const __grid_constant__ CUtensorMap tmO, Params p) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -376,25 +428,10 @@ __global__ void __launch_bounds__(THREADS, 1)
       const bool ok = mbar_wait(o_done, (n_kv - 1) & 1, err);
       if (__all_sync(0xffffffffu, ok)) {
         tc_fence_after();
-        const float inv = 1.f / l;
-        const int qrow = qt * TB + r;
-        bf16* orow = p.O + (size_t)q_row0 * p.ldo + (size_t)r * p.ldo + h * 128;
-#pragma unroll 1
-        for (int c = 0; c < 4; ++c) {
-          uint32_t u[32];
-          tmem_ld32(lane_base + O_COL + c * 32, u);
-          tmem_ld_wait();
-          reg_fence32(u);
-          if (qrow < p.Lq) {
-#pragma unroll
-            for (int g = 0; g < 4; ++g) {
-              float v[8];
-#pragma unroll
-              for (int i = 0; i < 8; ++i) v[i] = __uint_as_float(u[g * 8 + i]) * inv;
-              store_bf16x8(orow + c * 32 + g * 8, v);
-            }
-          }
-        }
+        // every MMA is done: the P tile is free for the O staging tiles (4 KB per warp)
+        store_o_warp(Ps + (warp - 2) * 4096, &tmO, lane_base + O_COL, 1.f / l, h * 128,
+                     qt * TB + quarter * 32, b, p.Lq, lane);
+        if (lane == 0) bulk_wait<0>();
       } else {
         failed = true;
       }
@@ -438,7 +475,8 @@ __device__ __forceinline__ void tc_mma_f16_ts(uint32_t d_tmem, uint32_t a_tmem, 
 
 __global__ void __launch_bounds__(THREADS2, 1)
     attn_tc2_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
-                    const __grid_constant__ CUtensorMap tmV, Params p) {
+                    const __grid_constant__ CUtensorMap tmV,
+                   const __grid_constant__ CUtensorMap tmO, Params p) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -663,30 +701,48 @@ __global__ void __launch_bounds__(THREADS2, 1)
             tmem_st32(lane_base + o_col + c * 32, u);
           }
         }
-        // exponent arguments and the row sum on key pairs: one packed FMA and one packed
-        // add per two keys
         const uint64_t sc2 = f2_pack(p.scale_log2, p.scale_log2);
         const uint64_t nm2 = f2_pack(-m_used, -m_used);
-        uint64_t ls2[4] = {0ull, 0ull, 0ull, 0ull};  // independent partial sums
+        uint64_t ls2[2] = {0ull, 0ull};  // independent partial sums
+        // keys 0-63 from the registers; P of those keys fills TMEM columns 0-31 only, so
+        // keys 64-127 are read again from their S columns instead of staying live in
+        // registers through the first half (register room for the item loop)
 #pragma unroll
         for (int c = 0; c < 2; ++c) {
+          float h[64];
+          if (c == 0) {
+#pragma unroll
+            for (int i = 0; i < 64; ++i) h[i] = s[i];
+          } else {
+            uint32_t u2[64];
+            tmem_ld32(lane_base + s_col + 64, u2);
+            tmem_ld32(lane_base + s_col + 96, u2 + 32);
+            tmem_ld_wait();
+            reg_fence32(u2);
+            reg_fence32(u2 + 32);
+#pragma unroll
+            for (int i = 0; i < 64; ++i) h[i] = __uint_as_float(u2[i]);
+            if (valid < TB) {
+#pragma unroll
+              for (int i = 0; i < 64; ++i)
+                if (64 + i >= valid) h[i] = -INFINITY;
+            }
+          }
           uint32_t u[32];
 #pragma unroll
           for (int i = 0; i < 32; ++i) {
             float t0, t1;
-            f2_unpack(f2_fma(f2_pack(s[c * 64 + 2 * i], s[c * 64 + 2 * i + 1]), sc2, nm2), t0,
-                      t1);
+            f2_unpack(f2_fma(f2_pack(h[2 * i], h[2 * i + 1]), sc2, nm2), t0, t1);
             const float e0 = ex2(t0), e1 = ex2(t1);
-            ls2[i & 3] = f2_add(ls2[i & 3], f2_pack(e0, e1));
+            ls2[i & 1] = f2_add(ls2[i & 1], f2_pack(e0, e1));
             u[i] = pack_bf16x2(e0, e1);
           }
           tmem_st32(lane_base + s_col + c * 32, u);
         }
         {
-          float a0, a1, b0, b1;
+          float a0, a1;
           f2_unpack(f2_add(ls2[0], ls2[1]), a0, a1);
-          f2_unpack(f2_add(ls2[2], ls2[3]), b0, b1);
-          l += (a0 + a1) + (b0 + b1);
+          l += a0 + a1;
         }
         tmem_st_wait();
         tc_fence_before();
@@ -697,25 +753,10 @@ __global__ void __launch_bounds__(THREADS2, 1)
         const bool ok = mbar_wait(o_done, 0, err);
         if (__all_sync(0xffffffffu, ok)) {
           tc_fence_after();
-          const float inv = 1.f / l;
-          const int qrow = qb * 2 * TB + g * TB + r;
-          bf16* orow = p.O + (size_t)(q_row0 + g * TB + r) * p.ldo + h * 128;
-#pragma unroll 1
-          for (int c = 0; c < 4; ++c) {
-            uint32_t u[32];
-            tmem_ld32(lane_base + o_col + c * 32, u);
-            tmem_ld_wait();
-            reg_fence32(u);
-            if (qrow < p.Lq) {
-#pragma unroll
-              for (int q = 0; q < 4; ++q) {
-                float v[8];
-#pragma unroll
-                for (int i = 0; i < 8; ++i) v[i] = __uint_as_float(u[q * 8 + i]) * inv;
-                store_bf16x8(orow + c * 32 + q * 8, v);
-              }
-            }
-          }
+          // every MMA is done: the Q tiles are free for the O staging tiles (4 KB per warp)
+          store_o_warp(Qs + (warp - 2) * 4096, &tmO, lane_base + o_col, 1.f / l, h * 128,
+                       qb * 2 * TB + g * TB + quarter * 32, b, p.Lq, lane);
+          if (lane == 0) bulk_wait<0>();
         } else {
           failed = true;
         }
@@ -749,20 +790,25 @@ __global__ void __launch_bounds__(THREADS2, 1)
 //    reads, so the first PV of the next item (accumulate = 0) cannot overwrite O early.
 // Group B has no work in items whose second query tile lies past Lq; the issuer and the
 // group count the phases of their own barriers.
+template <bool TMA_O>
 __global__ void __launch_bounds__(THREADS2, 1)
     attn_tc2p_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
-                     const __grid_constant__ CUtensorMap tmV, Params p) {
+                     const __grid_constant__ CUtensorMap tmV,
+                   const __grid_constant__ CUtensorMap tmO, Params p) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* Qs = smem;                  // [2 tiles][2 sub-tiles]
+  // K ring: 3 slots, or 2 and 32 KB of O staging tiles (4 KB per softmax warp)
+  constexpr int KS = TMA_O ? 2 : KSLOT;
   uint8_t* Ks = smem + 2 * Q_BYTES;
-  uint8_t* Vs = Ks + KSLOT * K_BYTES;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(Vs + VSLOT * V_BYTES);
+  uint8_t* Vs = Ks + KS * K_BYTES;
+  uint8_t* Os = Vs + VSLOT * V_BYTES;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(Os + (TMA_O ? 8 * 4096 : 0));
   uint64_t* q_full = bars;
   uint64_t* q_empty = bars + 1;
-  uint64_t* k_full = bars + 2;         // [3]
-  uint64_t* k_empty = bars + 5;        // [3]
+  uint64_t* k_full = bars + 2;         // [KS]
+  uint64_t* k_empty = bars + 5;        // [KS]
   uint64_t* v_full = bars + 8;         // [2]
   uint64_t* v_empty = bars + 10;       // [2]
   uint64_t* s_full = bars + 12;        // [2 groups]
@@ -780,7 +826,7 @@ __global__ void __launch_bounds__(THREADS2, 1)
   if (threadIdx.x == 0) {
     mbar_init(q_full, 1);
     mbar_init(q_empty, 1);
-    for (int s = 0; s < KSLOT; ++s) {
+    for (int s = 0; s < KS; ++s) {
       mbar_init(&k_full[s], 1);
       mbar_init(&k_empty[s], 1);
     }
@@ -820,8 +866,8 @@ __global__ void __launch_bounds__(THREADS2, 1)
           tma_load_2d(Qs + g * Q_BYTES + SUB, &tmQ, q_full, xq + 64, q_row0 + g * TB);
         }
         for (int j = 0; j < n_kv; ++j, ++kt) {
-          const int s = kt % KSLOT;
-          if (!mbar_wait(&k_empty[s], ((kt / KSLOT) & 1) ^ 1u, err)) { failed = true; break; }
+          const int s = kt % KS;
+          if (!mbar_wait(&k_empty[s], ((kt / KS) & 1) ^ 1u, err)) { failed = true; break; }
           uint8_t* st = Ks + s * K_BYTES;
           const int y = kv_row0 + j * TB;
           mbar_expect_tx(&k_full[s], K_BYTES);
@@ -859,7 +905,7 @@ __global__ void __launch_bounds__(THREADS2, 1)
       // its K slot, and of the last tile also the Q buffer
       auto issue_s = [&](int g, int j, int ng) {
         const uint32_t kt = kb + j;
-        const uint32_t ka = smem_u32(Ks + (kt % KSLOT) * K_BYTES);
+        const uint32_t ka = smem_u32(Ks + (kt % KS) * K_BYTES);
         const uint32_t qg = qa + g * Q_BYTES;
         if (j + 1 < n_kv || last_nch == 4) {
 #pragma unroll
@@ -879,7 +925,7 @@ __global__ void __launch_bounds__(THREADS2, 1)
         }
         tc_commit(&s_full[g]);
         if (g == ng - 1) {
-          tc_commit(&k_empty[kt % KSLOT]);
+          tc_commit(&k_empty[kt % KS]);
           if (j == n_kv - 1) tc_commit(q_empty);
         }
       };
@@ -901,7 +947,7 @@ __global__ void __launch_bounds__(THREADS2, 1)
         const int qb = item % nqb;
         const int ng = qb * 2 * TB + TB < p.Lq ? 2 : 1;
         if (!(ok = mbar_wait(q_full, it & 1, err))) break;
-        if (!(ok = mbar_wait(&k_full[kb % KSLOT], (kb / KSLOT) & 1, err))) break;
+        if (!(ok = mbar_wait(&k_full[kb % KS], (kb / KS) & 1, err))) break;
         tc_fence_after();
         for (int g = 0; g < ng; ++g) issue_s(g, 0, ng);
         for (int j = 0; j < n_kv && ok; ++j) {
@@ -914,7 +960,7 @@ __global__ void __launch_bounds__(THREADS2, 1)
           if (ng == 1) tc_commit(&v_empty[vt & 1]);
           if (more) {
             const uint32_t kt = kb + j + 1;
-            if (!(ok = mbar_wait(&k_full[kt % KSLOT], (kt / KSLOT) & 1, err))) break;
+            if (!(ok = mbar_wait(&k_full[kt % KS], (kt / KS) & 1, err))) break;
             tc_fence_after();
             issue_s(0, j + 1, ng);
           }
@@ -1038,27 +1084,35 @@ __global__ void __launch_bounds__(THREADS2, 1)
       if (!__all_sync(0xffffffffu, ok)) { failed = true; break; }
       tc_fence_after();
       const int bh = item / nqb, h = bh % p.heads, b = bh / p.heads;
-      const float inv = 1.f / l;
-      const int qrow = qb * 2 * TB + g * TB + r;
-      bf16* orow = p.O + (size_t)(b * p.Lq + qrow) * p.ldo + h * 128;
+      if constexpr (TMA_O) {
+        if (lane == 0) bulk_wait_read<0>();  // the previous item's stores have read the tile
+        __syncwarp();
+        store_o_warp(Os + (warp - 2) * 4096, &tmO, lane_base + o_col, 1.f / l, h * 128,
+                     qb * 2 * TB + g * TB + quarter * 32, b, p.Lq, lane);
+      } else {
+        const float inv = 1.f / l;
+        const int qrow = qb * 2 * TB + g * TB + r;
+        bf16* orow = p.O + (size_t)(b * p.Lq + qrow) * p.ldo + h * 128;
 #pragma unroll 1
-      for (int c = 0; c < 4; ++c) {
-        uint32_t u[32];
-        tmem_ld32(lane_base + o_col + c * 32, u);
-        tmem_ld_wait();
-        reg_fence32(u);
-        if (qrow < p.Lq) {
+        for (int c = 0; c < 4; ++c) {
+          uint32_t u[32];
+          tmem_ld32(lane_base + o_col + c * 32, u);
+          tmem_ld_wait();
+          reg_fence32(u);
+          if (qrow < p.Lq) {
 #pragma unroll
-          for (int q = 0; q < 4; ++q) {
-            float v[8];
+            for (int q = 0; q < 4; ++q) {
+              float v[8];
 #pragma unroll
-            for (int i = 0; i < 8; ++i) v[i] = __uint_as_float(u[q * 8 + i]) * inv;
-            store_bf16x8(orow + c * 32 + q * 8, v);
+              for (int i = 0; i < 8; ++i) v[i] = __uint_as_float(u[q * 8 + i]) * inv;
+              store_bf16x8(orow + c * 32 + q * 8, v);
+            }
           }
         }
       }
       ++cnt;
     }
+    if (TMA_O && lane == 0) bulk_wait<0>();  // this warp's O stores complete before exit
   }
 
   if (failed || *(volatile int*)err != 0) {
@@ -1101,7 +1155,23 @@ bool map_128x64(CUtensorMap* m, const bf16* ptr, int rows, int cols, int ld) {
              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// O as a 3-D tensor [batch][Lq][cols] (row stride ld, batch stride Lq ld): a TMA store box
+// of 32 rows x 64 columns (128-byte swizzle) stops at each batch's Lq
+bool map_o(CUtensorMap* m, const bf16* ptr, int batch, int Lq, int cols, int ld) {
+  auto enc = encoder();
+  if (!enc) return false;
+  cuuint64_t dims[3] = {(cuuint64_t)cols, (cuuint64_t)Lq, (cuuint64_t)batch};
+  cuuint64_t strides[2] = {(cuuint64_t)ld * sizeof(bf16), (cuuint64_t)Lq * ld * sizeof(bf16)};
+  cuuint32_t box[3] = {64, 32, 1};
+  cuuint32_t estr[3] = {1, 1, 1};
+  return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<bf16*>(ptr), dims, strides, box,
+             estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+             CU_TENSOR_MAP_L2_PROMOTION_L2_128B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 }  // namespace
+
+static int n_kv_of(const AttnArgs& a) { return (a.Lkv + TB - 1) / TB; }
 
 cudaError_t attention_tc_set_wait_limit(unsigned long long ns) {
   return fb_set_wait_limit_tu(ns);
@@ -1118,9 +1188,10 @@ cudaError_t attention_tc(const AttnArgs& a, int* err, cudaStream_t st) {
   if (!attention_tc_supported(a)) return cudaErrorInvalidValue;
   const int cols = a.heads * 128;
   const int kv_rows = a.kv_batch_rows ? (a.batch - 1) * a.kv_batch_rows + a.Lkv : a.Lkv;
-  CUtensorMap mq, mk, mv;
+  CUtensorMap mq, mk, mv, mo;
   if (!map_128x64(&mq, a.Q, a.batch * a.Lq, cols, a.ldq) ||
-      !map_128x64(&mk, a.K, kv_rows, cols, a.ldk) || !map_128x64(&mv, a.V, kv_rows, cols, a.ldv))
+      !map_128x64(&mk, a.K, kv_rows, cols, a.ldk) || !map_128x64(&mv, a.V, kv_rows, cols, a.ldv) ||
+      !map_o(&mo, a.O, a.batch, a.Lq, cols, a.ldo))
     return cudaErrorInvalidValue;
   int dev = 0, sms = a.sms;
   if (sms <= 0 && (cudaGetDevice(&dev) != cudaSuccess ||
@@ -1148,11 +1219,13 @@ cudaError_t attention_tc(const AttnArgs& a, int* err, cudaStream_t st) {
   const bool two = a.tc_variant >= 2 || (a.tc_variant == 0 && 10 * w1 >= 14 * w2);
   // more than one wave of 256-query CTAs: one persistent CTA per SM loops over them
   if (a.tc_variant == 3 || (two && a.tc_variant == 0 && ctas2 > sms)) {
-    cudaError_t e = cudaFuncSetAttribute(attn_tc2p_kernel,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM2_BYTES);
+    // items of at most 4 key tiles store O through TMA (see attn_tc2p_kernel)
+    auto kern = n_kv_of(a) <= 4 ? attn_tc2p_kernel<true> : attn_tc2p_kernel<false>;
+    cudaError_t e =
+        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM2_BYTES);
     if (e != cudaSuccess) return e;
     const int grid = (int)(ctas2 < sms ? ctas2 : sms);
-    e = launch_k(attn_tc2p_kernel, dim3(grid), dim3(THREADS2), SMEM2_BYTES, st, mq, mk, mv, p);
+    e = launch_k(kern, dim3(grid), dim3(THREADS2), SMEM2_BYTES, st, mq, mk, mv, mo, p);
     if (e != cudaSuccess) return e;
     return cudaGetLastError();
   }
@@ -1161,14 +1234,14 @@ cudaError_t attention_tc(const AttnArgs& a, int* err, cudaStream_t st) {
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM2_BYTES);
     if (e != cudaSuccess) return e;
     dim3 grid((a.Lq + 2 * TB - 1) / (2 * TB), a.heads, a.batch);
-    e = launch_k(attn_tc2_kernel, grid, dim3(THREADS2), SMEM2_BYTES, st, mq, mk, mv, p);
+    e = launch_k(attn_tc2_kernel, grid, dim3(THREADS2), SMEM2_BYTES, st, mq, mk, mv, mo, p);
     if (e != cudaSuccess) return e;
   } else {
     cudaError_t e = cudaFuncSetAttribute(attn_tc_kernel,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
     if (e != cudaSuccess) return e;
     dim3 grid((a.Lq + TB - 1) / TB, a.heads, a.batch);
-    e = launch_k(attn_tc_kernel, grid, dim3(THREADS), SMEM_BYTES, st, mq, mk, mv, p);
+    e = launch_k(attn_tc_kernel, grid, dim3(THREADS), SMEM_BYTES, st, mq, mk, mv, mo, p);
     if (e != cudaSuccess) return e;
   }
   return cudaGetLastError();
