@@ -650,6 +650,13 @@ def run_probe(args):
     if args.probe == "pointwise":
         m.close()
         return probe_pointwise(args)
+    if args.probe == "mma_rate":
+        res = {f"N{n}/issuers{k}": round(fb.fb_probe_mma_rate(k, n), 1)
+               for n in (64, 128, 256) for k in (1, 2, 4) if k * n <= 512}
+        print(json.dumps({"probe": "mma_rate", "unit": "MAC per SM clock",
+                          "nominal": 4096, "res": res}))
+        m.close()
+        return 0
     if args.probe in ("gemm_shapes", "attn_shapes", "breakdown"):
         call = None
     elif args.probe in ("gemm_refine_out", "gemm_refine_down"):
@@ -960,7 +967,7 @@ def main():
     ap.add_argument("--probe", choices=["gemm", "gemm_resid", "gemm_out", "gemm_refine_out",
                                         "gemm_refine_down", "attn", "attn_mma", "gemm_shapes",
                                         "attn_shapes", "breakdown", "pointwise",
-                                        "attn_pool"],
+                                        "attn_pool", "mma_rate"],
                     default=None)
     args = ap.parse_args()
     if args.probe:

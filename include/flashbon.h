@@ -384,6 +384,14 @@ fb_status fb_gemm_streamk_noalloc(void* stream, int M, int N, int K, const void*
  * them, so that the next stream-K finisher waits for a count no launch will reach. The
  * wait runs out at the device wait limit, the call returns FB_ECUDA and clears the
  * counters; the call after it computes normally. */
+/* fb_probe_mma_rate: the tensor pipe's sustained rate on the current device, in MACs per SM
+ * clock: every SM times (clock64) `reps` tcgen05.mma kind::f16 instructions of M = 128,
+ * K = 16 and width n (64, 128 or 256) issued by each of `issuers` warps (1-4,
+ * issuers * n <= 512 TMEM columns) into accumulators of their own; *mac_per_clk is
+ * computed from the slowest SM. Allocates and
+ * frees two small device buffers and synchronises the device. FB_EINVAL for arguments
+ * outside those ranges, FB_ECUDA on a CUDA error. */
+fb_status fb_probe_mma_rate(int issuers, int n, int reps, double* mac_per_clk);
 fb_status fb_set_device_wait_limit(unsigned long long ns);
 fb_status fb_test_fail_alloc(long k);
 long fb_test_alloc_calls(void);

@@ -18,7 +18,7 @@ CSRC = os.path.join(PKG, "csrc")
 BUILD = os.path.join(ROOT, "_build")
 LIB = os.path.join(PKG, "libflashbon.so")
 SOURCES = ["api.cu", "gemm_tc.cu", "gemm_simt.cu", "attention.cu", "attention_tc.cu",
-           "pointwise.cu", "select.cu"]
+           "pointwise.cu", "select.cu", "probe.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

@@ -1444,6 +1444,40 @@ fb_status fb_test_fail_alloc(long k) {
 
 long fb_test_alloc_calls(void) { return g_alloc_calls.load(); }
 
+fb_status fb_probe_mma_rate(int issuers, int n, int reps, double* mac_per_clk) {
+  if (!mac_per_clk || issuers < 1 || issuers > 4 || (n != 64 && n != 128 && n != 256) ||
+      issuers * n > 512 || reps < 1)
+    return fail(FB_EINVAL, "issuers 1..4, n 64/128/256, issuers * n <= 512 TMEM columns, "
+                           "reps >= 1, non-NULL output");
+  int dev = 0, sms = 0;
+  CK(cudaGetDevice(&dev));
+  CK(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
+  unsigned long long* cyc = nullptr;
+  int* err = nullptr;
+  CK(cudaMalloc(&cyc, sizeof(unsigned long long) * sms));
+  if (cudaMalloc(&err, sizeof(int)) != cudaSuccess) {
+    cudaFree(cyc);
+    return fail(FB_ENOMEM, "cudaMalloc failed");
+  }
+  std::vector<unsigned long long> h(sms);
+  int herr = 0;
+  cudaError_t e = cudaMemset(err, 0, sizeof(int));
+  if (e == cudaSuccess) e = cudaMemset(cyc, 0, sizeof(unsigned long long) * sms);
+  fb_stream_op_not_kernel();
+  if (e == cudaSuccess) e = mma_rate_probe(issuers, n, reps, sms, cyc, err, nullptr);
+  if (e == cudaSuccess) e = cudaDeviceSynchronize();
+  if (e == cudaSuccess)
+    e = cudaMemcpy(h.data(), cyc, sizeof(unsigned long long) * sms, cudaMemcpyDeviceToHost);
+  if (e == cudaSuccess) e = cudaMemcpy(&herr, err, sizeof(int), cudaMemcpyDeviceToHost);
+  cudaFree(cyc);
+  cudaFree(err);
+  if (e != cudaSuccess) return fail(FB_ECUDA, "probe failed: %s", cudaGetErrorString(e));
+  if (herr != 0) return fail(FB_ECUDA, "device wait timed out");
+  const unsigned long long slowest = *std::max_element(h.begin(), h.end());
+  *mac_per_clk = 128.0 * n * 16 * (double)issuers * reps / (double)slowest;
+  return FB_OK;
+}
+
 fb_status fb_test_poison_counters(fb_model* m) {
   int* ctr = nullptr;
   size_t n = 0;

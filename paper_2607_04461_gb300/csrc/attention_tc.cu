@@ -1218,7 +1218,8 @@ cudaError_t attention_tc(const AttnArgs& a, int* err, cudaStream_t st) {
   const long w1 = (ctas1 + sms - 1) / sms, w2 = (ctas2 + sms - 1) / sms;
   const bool two = a.tc_variant >= 2 || (a.tc_variant == 0 && 10 * w1 >= 14 * w2);
   // more than one wave of 256-query CTAs: one persistent CTA per SM loops over them
-  if (a.tc_variant == 3 || (two && a.tc_variant == 0 && ctas2 > sms)) {
+  const bool persistent = a.tc_variant >= 3 || (two && a.tc_variant == 0 && ctas2 > sms);
+  if (persistent) {
     // items of at most 4 key tiles store O through TMA (see attn_tc2p_kernel)
     auto kern = n_kv_of(a) <= 4 ? attn_tc2p_kernel<true> : attn_tc2p_kernel<false>;
     cudaError_t e =

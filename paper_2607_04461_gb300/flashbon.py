@@ -55,7 +55,8 @@ EXPORTS = ["fb_weights_count", "fb_weights_entry", "fb_init_model", "fb_free", "
            "fb_set_op_repeat", "fb_gemm_streamk_noalloc", "fb_state_bytes", "fb_state_offload",
            "fb_state_wait", "fb_set_sm_budget", "fb_sm_split_create", "fb_sm_split_info",
            "fb_sm_split_free", "fb_pipeline_step", "fb_set_device_wait_limit",
-           "fb_test_fail_alloc", "fb_test_alloc_calls", "fb_test_poison_counters"]
+           "fb_test_fail_alloc", "fb_test_alloc_calls", "fb_test_poison_counters",
+           "fb_probe_mma_rate"]
 
 PAIR_VERIFIER = ctypes.CFUNCTYPE(ctypes.c_int, ctypes.c_void_p, ctypes.c_int, ctypes.c_int,
                                  ctypes.POINTER(ctypes.c_int))
@@ -110,6 +111,7 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
         "fb_test_fail_alloc": (I, [ctypes.c_long]),
         "fb_test_alloc_calls": (ctypes.c_long, []),
         "fb_test_poison_counters": (I, [P]),
+        "fb_probe_mma_rate": (I, [I, I, I, ctypes.POINTER(ctypes.c_double)]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(L, name)
@@ -386,6 +388,13 @@ def fb_test_poison_counters(model) -> None:
     """Sets the stream-K counters of `model` (None: the allocation-free entry point's) to
     a large negative value, so the next stream-K finisher's wait cannot complete."""
     _check(load_library().fb_test_poison_counters(model))
+
+
+def fb_probe_mma_rate(issuers: int, n: int, reps: int = 16384) -> float:
+    """Tensor-pipe MACs per SM clock with `issuers` issuing warps and M=128 x n MMAs."""
+    out = ctypes.c_double()
+    _check(load_library().fb_probe_mma_rate(int(issuers), int(n), int(reps), ctypes.byref(out)))
+    return out.value
 
 
 def fb_get_stats(model: int) -> dict:
