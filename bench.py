@@ -689,13 +689,22 @@ def run_probe(args):
             h, hb, gt = rnd(M, D, dt=torch.float32), rnd(M, D, dt=torch.float32), rnd(D, dt=torch.float32)
             dl = torch.empty(M, D, dtype=torch.bfloat16, device="cuda")
             call = lambda: fb.fb_op_gemm(m.handle, M, D, F, A, W, b, 3, h, hb, gt, h, dl)  # noqa
+    elif args.probe == "attn_pool_cross":
+        # the draft pool's cross-attention: 32 candidates x 1560 queries, 512 text keys
+        n, P, H, dh, T = 32, 1560, 12, 128, 512
+        q, kv = rnd(n * P, H * dh), rnd(T, 2 * H * dh)
+        o = torch.empty(n * P, H * dh, dtype=torch.bfloat16, device="cuda")
+        D = H * dh
+        call = lambda: fb.fb_op_attention(m.handle, q, D, kv.data_ptr(), 2 * D,  # noqa
+                                          kv.data_ptr() + 2 * D, 2 * D, o, D, n, P, T, 0, H, dh, 0)
     else:
         n, P, H, dh = (32 if args.probe == "attn_pool" else 4), 1560, 12, 128
         qkv, o = rnd(n * P, 3 * H * dh), torch.empty(n * P, H * dh, dtype=torch.bfloat16, device="cuda")
         base, D = qkv.data_ptr(), H * dh
         call = lambda: fb.fb_op_attention(m.handle, base, 3 * D, base + 2 * D, 3 * D,  # noqa
                                           base + 4 * D, 3 * D, o, D, n, P, P, P, H, dh,
-                                          1 if args.probe == "attn_mma" else 3)
+                                          1 if args.probe == "attn_mma" else
+                                          (0 if args.probe == "attn_pool" else 3))
     if args.probe == "gemm_shapes":
         return probe_gemm_shapes(m, rnd, args)
     if args.probe == "attn_shapes":
@@ -967,7 +976,7 @@ def main():
     ap.add_argument("--probe", choices=["gemm", "gemm_resid", "gemm_out", "gemm_refine_out",
                                         "gemm_refine_down", "attn", "attn_mma", "gemm_shapes",
                                         "attn_shapes", "breakdown", "pointwise",
-                                        "attn_pool", "mma_rate"],
+                                        "attn_pool", "attn_pool_cross", "mma_rate"],
                     default=None)
     args = ap.parse_args()
     if args.probe:
