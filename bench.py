@@ -657,7 +657,7 @@ def run_probe(args):
                           "nominal": 4096, "res": res}))
         m.close()
         return 0
-    if args.probe in ("gemm_shapes", "attn_shapes", "breakdown"):
+    if args.probe in ("gemm_shapes", "gemm_shapes_part", "attn_shapes", "breakdown"):
         call = None
     elif args.probe in ("gemm_refine_out", "gemm_refine_down"):
         # the refine pass's attention output projection / FFN down-projection (one
@@ -705,8 +705,8 @@ def run_probe(args):
                                           base + 4 * D, 3 * D, o, D, n, P, P, P, H, dh,
                                           1 if args.probe == "attn_mma" else
                                           (0 if args.probe == "attn_pool" else 3))
-    if args.probe == "gemm_shapes":
-        return probe_gemm_shapes(m, rnd, args)
+    if args.probe in ("gemm_shapes", "gemm_shapes_part"):
+        return probe_gemm_shapes(m, rnd, args, part=args.probe == "gemm_shapes_part")
     if args.probe == "attn_shapes":
         return probe_attn_shapes(m, rnd, args)
     if args.probe == "breakdown":
@@ -722,10 +722,12 @@ def run_probe(args):
     return 0
 
 
-def probe_gemm_shapes(m, rnd, args):
+def probe_gemm_shapes(m, rnd, args, part=False):
     """Per-launch time of each block GEMM shape at the draft (N=32) and refine (N=1) row
     counts: `reps` back-to-back launches inside one call, timed with CUDA events on the
-    library's stream (fb_get_stats), for the automatic choice and the forced 1-SM kernel."""
+    library's stream (fb_get_stats), for the automatic choice and each forced variant.
+    part: the refine's row count only, on an SM partition of --refine-sms SMs (the split
+    schedule's refine side)."""
     import torch
     from paper_2607_04461_gb300 import flashbon as fb
     D, F = 1536, 8960
@@ -733,7 +735,13 @@ def probe_gemm_shapes(m, rnd, args):
               "cross_out": (D, D, 2), "ffn_up": (F, D, 1), "ffn_down": (D, F, 3)}
     res = {}
     reps = max(5, args.steps)
-    for M in (49920, 1560):
+    split = None
+    if part:
+        split = fb.SmSplit(args.refine_sms)
+        m.set_stream(split.streams[0])
+        m.set_sm_budget(split.sms[0])
+        res["partition_sms"] = split.sms[0]
+    for M in ((1560,) if part else (49920, 1560)):
         for name, (N, K, epi) in shapes.items():
             A, W, b = rnd(M, K), rnd(N, K), rnd(N, dt=torch.float32)
             out = torch.empty(M, N, dtype=torch.bfloat16 if epi < 2 else torch.float32, device="cuda")
@@ -763,6 +771,11 @@ def probe_gemm_shapes(m, rnd, args):
                     "us": round(us, 2), "tflops": round(2 * M * N * K / us / 1e6, 1),
                     "chained_us": round(chain_us, 2)}
             del A, W, out, r, dl
+    if split:
+        torch.cuda.synchronize()
+        m.set_sm_budget(0)
+        m.set_stream(None)
+        split.close()
     print(json.dumps({"probe": "gemm_shapes", "res": res}))
     return 0
 
@@ -974,7 +987,7 @@ def main():
                     help="base: the draft-pool workload; cfg / sde: the same with guidance "
                          "or SDE steps")
     ap.add_argument("--probe", choices=["gemm", "gemm_resid", "gemm_out", "gemm_refine_out",
-                                        "gemm_refine_down", "attn", "attn_mma", "gemm_shapes",
+                                        "gemm_refine_down", "attn", "attn_mma", "gemm_shapes", "gemm_shapes_part",
                                         "attn_shapes", "breakdown", "pointwise",
                                         "attn_pool", "attn_pool_cross", "mma_rate"],
                     default=None)

@@ -100,25 +100,6 @@ __device__ __forceinline__ float ex2(float x) {
   return y;
 }
 
-// packed pairs of fp32 (sm_100 and later execute one fma/add on both halves)
-__device__ __forceinline__ uint64_t f2_pack(float lo, float hi) {
-  uint64_t r;
-  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(lo), "f"(hi));
-  return r;
-}
-__device__ __forceinline__ void f2_unpack(uint64_t v, float& lo, float& hi) {
-  asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(v));
-}
-__device__ __forceinline__ uint64_t f2_fma(uint64_t a, uint64_t b, uint64_t c) {
-  uint64_t d;
-  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
-  return d;
-}
-__device__ __forceinline__ uint64_t f2_add(uint64_t a, uint64_t b) {
-  uint64_t d;
-  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
-  return d;
-}
 
 
 __device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t* r) {
@@ -396,8 +377,8 @@ __global__ void __launch_bounds__(THREADS, 1)
         tmem_st_wait();
       }
       // exponent arguments and the row sum on key pairs (packed FMA and add)
-      const uint64_t sc2 = f2_pack(p.scale_log2, p.scale_log2);
-      const uint64_t nm2 = f2_pack(-m_used, -m_used);
+      const uint64_t sc2 = f2_join(p.scale_log2, p.scale_log2);
+      const uint64_t nm2 = f2_join(-m_used, -m_used);
       uint64_t ls2[4] = {0ull, 0ull, 0ull, 0ull};  // independent partial sums
 #pragma unroll
       for (int ch = 0; ch < 16; ++ch) {  // 16-byte chunks of 8 keys
@@ -405,9 +386,9 @@ __global__ void __launch_bounds__(THREADS, 1)
 #pragma unroll
         for (int q = 0; q < 4; ++q) {
           float t0, t1;
-          f2_unpack(f2_fma(f2_pack(s[ch * 8 + 2 * q], s[ch * 8 + 2 * q + 1]), sc2, nm2), t0, t1);
+          f2_split(f2_fma(f2_join(s[ch * 8 + 2 * q], s[ch * 8 + 2 * q + 1]), sc2, nm2), t0, t1);
           const float e0 = ex2(t0), e1 = ex2(t1);
-          ls2[q] = f2_add(ls2[q], f2_pack(e0, e1));
+          ls2[q] = f2_add(ls2[q], f2_join(e0, e1));
           w[q] = pack_bf16x2(e0, e1);
         }
         const int sub = ch >> 3, c16 = (ch & 7) ^ (r & 7);
@@ -415,8 +396,8 @@ __global__ void __launch_bounds__(THREADS, 1)
       }
       {
         float a0, a1, b0, b1;
-        f2_unpack(f2_add(ls2[0], ls2[1]), a0, a1);
-        f2_unpack(f2_add(ls2[2], ls2[3]), b0, b1);
+        f2_split(f2_add(ls2[0], ls2[1]), a0, a1);
+        f2_split(f2_add(ls2[2], ls2[3]), b0, b1);
         l += (a0 + a1) + (b0 + b1);
       }
       fence_async_smem();  // P visible to the tensor core (async proxy)
@@ -701,8 +682,8 @@ __global__ void __launch_bounds__(THREADS2, 1)
             tmem_st32(lane_base + o_col + c * 32, u);
           }
         }
-        const uint64_t sc2 = f2_pack(p.scale_log2, p.scale_log2);
-        const uint64_t nm2 = f2_pack(-m_used, -m_used);
+        const uint64_t sc2 = f2_join(p.scale_log2, p.scale_log2);
+        const uint64_t nm2 = f2_join(-m_used, -m_used);
         uint64_t ls2[2] = {0ull, 0ull};  // independent partial sums
         // keys 0-63 from the registers; P of those keys fills TMEM columns 0-31 only, so
         // keys 64-127 are read again from their S columns instead of staying live in
@@ -732,16 +713,16 @@ __global__ void __launch_bounds__(THREADS2, 1)
 #pragma unroll
           for (int i = 0; i < 32; ++i) {
             float t0, t1;
-            f2_unpack(f2_fma(f2_pack(h[2 * i], h[2 * i + 1]), sc2, nm2), t0, t1);
+            f2_split(f2_fma(f2_join(h[2 * i], h[2 * i + 1]), sc2, nm2), t0, t1);
             const float e0 = ex2(t0), e1 = ex2(t1);
-            ls2[i & 1] = f2_add(ls2[i & 1], f2_pack(e0, e1));
+            ls2[i & 1] = f2_add(ls2[i & 1], f2_join(e0, e1));
             u[i] = pack_bf16x2(e0, e1);
           }
           tmem_st32(lane_base + s_col + c * 32, u);
         }
         {
           float a0, a1;
-          f2_unpack(f2_add(ls2[0], ls2[1]), a0, a1);
+          f2_split(f2_add(ls2[0], ls2[1]), a0, a1);
           l += a0 + a1;
         }
         tmem_st_wait();
@@ -1030,8 +1011,8 @@ __global__ void __launch_bounds__(THREADS2, 1)
             tmem_st32(lane_base + o_col + c * 32, u);
           }
         }
-        const uint64_t sc2 = f2_pack(p.scale_log2, p.scale_log2);
-        const uint64_t nm2 = f2_pack(-m_used, -m_used);
+        const uint64_t sc2 = f2_join(p.scale_log2, p.scale_log2);
+        const uint64_t nm2 = f2_join(-m_used, -m_used);
         uint64_t ls2[2] = {0ull, 0ull};  // independent partial sums
         // keys 0-63 from the registers; P of those keys fills TMEM columns 0-31 only, so
         // keys 64-127 are read again from their S columns instead of staying live in
@@ -1061,16 +1042,16 @@ __global__ void __launch_bounds__(THREADS2, 1)
 #pragma unroll
           for (int i = 0; i < 32; ++i) {
             float t0, t1;
-            f2_unpack(f2_fma(f2_pack(h[2 * i], h[2 * i + 1]), sc2, nm2), t0, t1);
+            f2_split(f2_fma(f2_join(h[2 * i], h[2 * i + 1]), sc2, nm2), t0, t1);
             const float e0 = ex2(t0), e1 = ex2(t1);
-            ls2[i & 1] = f2_add(ls2[i & 1], f2_pack(e0, e1));
+            ls2[i & 1] = f2_add(ls2[i & 1], f2_join(e0, e1));
             u[i] = pack_bf16x2(e0, e1);
           }
           tmem_st32(lane_base + s_col + c * 32, u);
         }
         {
           float a0, a1;
-          f2_unpack(f2_add(ls2[0], ls2[1]), a0, a1);
+          f2_split(f2_add(ls2[0], ls2[1]), a0, a1);
           l += a0 + a1;
         }
         tmem_st_wait();

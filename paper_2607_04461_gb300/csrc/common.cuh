@@ -112,11 +112,51 @@ __device__ __forceinline__ float tanh_approx(float x) {
   asm("tanh.approx.f32 %0, %1;" : "=f"(y) : "f"(x));
   return y;
 }
-// GELU, tanh form. The hardware tanh (max relative error about 2^-11) is well inside
-// the bf16 rounding of the GEMM output that it feeds.
+// GELU, tanh form: 0.5 x (1 + tanh(sqrt(2/pi) (x + 0.044715 x^3))), evaluated as
+// h + h tanh(x (k0 + k1 x^2)) with h = x / 2 (five fp32 operations and one tanh). The
+// hardware tanh (max relative error about 2^-11) is well inside the bf16 rounding of the
+// GEMM output that it feeds.
 __device__ __forceinline__ float gelu_tanh_f(float x) {
-  const float k0 = 0.7978845608028654f;  // sqrt(2/pi)
-  return 0.5f * x * (1.f + tanh_approx(k0 * (x + 0.044715f * x * x * x)));
+  const float k0 = 0.7978845608028654f;              // sqrt(2/pi)
+  const float k1 = 0.7978845608028654f * 0.044715f;  // sqrt(2/pi) * 0.044715
+  const float h = 0.5f * x;
+  return fmaf(h, tanh_approx(x * fmaf(x * x, k1, k0)), h);
+}
+// packed pairs of fp32 (sm_100 and later execute one fma/add/mul on both halves)
+__device__ __forceinline__ uint64_t f2_join(float lo, float hi) {
+  uint64_t r;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(lo), "f"(hi));
+  return r;
+}
+__device__ __forceinline__ void f2_split(uint64_t v, float& lo, float& hi) {
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(v));
+}
+__device__ __forceinline__ uint64_t f2_add(uint64_t a, uint64_t b) {
+  uint64_t d;
+  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+__device__ __forceinline__ uint64_t f2_mul(uint64_t a, uint64_t b) {
+  uint64_t d;
+  asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+__device__ __forceinline__ uint64_t f2_fma(uint64_t a, uint64_t b, uint64_t c) {
+  uint64_t d;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
+  return d;
+}
+// gelu_tanh_f on a pair, the fp32 arithmetic on packed pairs
+__device__ __forceinline__ void gelu_tanh_f2(float& a, float& b) {
+  const uint64_t x = f2_join(a, b);
+  const uint64_t h = f2_mul(x, f2_join(0.5f, 0.5f));
+  const uint64_t t = f2_fma(f2_mul(x, x), f2_join(0.7978845608028654f * 0.044715f,
+                                                   0.7978845608028654f * 0.044715f),
+                            f2_join(0.7978845608028654f, 0.7978845608028654f));
+  float u0, u1;
+  f2_split(f2_mul(x, t), u0, u1);
+  const uint64_t th = f2_join(tanh_approx(u0), tanh_approx(u1));
+  f2_split(f2_fma(h, th, h), a, b);
 }
 __device__ __forceinline__ float silu_f(float x) { return x / (1.f + expf(-x)); }
 

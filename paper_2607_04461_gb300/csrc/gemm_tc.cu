@@ -722,17 +722,18 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
             // one outstanding group allowed is the other tile's, one chunk ago)
             if (lane == 0) bulk_wait_read<1>();
             __syncwarp();
+            // bias by shuffle; GELU on packed fp32 pairs
 #pragma unroll
             for (int q = 0; q < 4; ++q) {
-              float y[8];
+              uint32_t w[4];
 #pragma unroll
-              for (int i = 0; i < 8; ++i) {
-                y[i] = v[8 * q + i] + __shfl_sync(0xffffffffu, bl, 8 * q + i);
-                if (KIND == EPI_GELU_BF16) y[i] = gelu_tanh_f(y[i]);
+              for (int i = 0; i < 4; ++i) {
+                float y0 = v[8 * q + 2 * i] + __shfl_sync(0xffffffffu, bl, 8 * q + 2 * i);
+                float y1 = v[8 * q + 2 * i + 1] + __shfl_sync(0xffffffffu, bl, 8 * q + 2 * i + 1);
+                if (KIND == EPI_GELU_BF16) gelu_tanh_f2(y0, y1);
+                w[i] = pack_bf16x2(y0, y1);
               }
-              *reinterpret_cast<uint4*>(tile_b + swz64(lane, q)) =
-                  make_uint4(pack_bf16x2(y[0], y[1]), pack_bf16x2(y[2], y[3]),
-                             pack_bf16x2(y[4], y[5]), pack_bf16x2(y[6], y[7]));
+              *reinterpret_cast<uint4*>(tile_b + swz64(lane, q)) = make_uint4(w[0], w[1], w[2], w[3]);
             }
           }
           fence_proxy_async_smem();
