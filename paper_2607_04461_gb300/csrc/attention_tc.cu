@@ -634,7 +634,6 @@ __global__ void __launch_bounds__(THREADS2, 1)
     // ---------------- softmax groups: warps 2-5 -> tile A, warps 6-9 -> tile B ----------
     const int g = (warp - 2) >> 2;
     const int quarter = warp & 3;
-    const int r = quarter * 32 + lane;
     const uint32_t lane_base = tmem + ((uint32_t)(quarter * 32) << 16);
     const uint32_t s_col = g * TB, o_col = O_COL + g * TB;
     float m_used = -INFINITY, l = 0.f;
@@ -767,25 +766,22 @@ __global__ void __launch_bounds__(THREADS2, 1)
 //  * the MMA issuer starts the next item's S MMAs right after the current item's last PV
 //    (the tensor pipe runs in order, so S_g overwrites P_g only after PV_g has read it);
 //  * each softmax group stores its O rows (o_done, one phase per item of the group) while
-//    those S MMAs run; its first P of the next item is announced only after those TMEM
-//    reads, so the first PV of the next item (accumulate = 0) cannot overwrite O early.
+//    those S MMAs run, each thread its row in 32-byte stores (whole sectors); its first P
+//    of the next item is announced only after those TMEM reads, so the first PV of the
+//    next item (accumulate = 0) cannot overwrite O early.
 // Group B has no work in items whose second query tile lies past Lq; the issuer and the
 // group count the phases of their own barriers.
-template <bool TMA_O>
 __global__ void __launch_bounds__(THREADS2, 1)
     attn_tc2p_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
-                     const __grid_constant__ CUtensorMap tmV,
-                   const __grid_constant__ CUtensorMap tmO, Params p) {
+                     const __grid_constant__ CUtensorMap tmV, Params p) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* Qs = smem;                  // [2 tiles][2 sub-tiles]
-  // K ring: 3 slots, or 2 and 32 KB of O staging tiles (4 KB per softmax warp)
-  constexpr int KS = TMA_O ? 2 : KSLOT;
+  constexpr int KS = KSLOT;            // K ring slots
   uint8_t* Ks = smem + 2 * Q_BYTES;
   uint8_t* Vs = Ks + KS * K_BYTES;
-  uint8_t* Os = Vs + VSLOT * V_BYTES;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(Os + (TMA_O ? 8 * 4096 : 0));
+  uint64_t* bars = reinterpret_cast<uint64_t*>(Vs + VSLOT * V_BYTES);
   uint64_t* q_full = bars;
   uint64_t* q_empty = bars + 1;
   uint64_t* k_full = bars + 2;         // [KS]
@@ -1065,15 +1061,12 @@ __global__ void __launch_bounds__(THREADS2, 1)
       if (!__all_sync(0xffffffffu, ok)) { failed = true; break; }
       tc_fence_after();
       const int bh = item / nqb, h = bh % p.heads, b = bh / p.heads;
-      if constexpr (TMA_O) {
-        if (lane == 0) bulk_wait_read<0>();  // the previous item's stores have read the tile
-        __syncwarp();
-        store_o_warp(Os + (warp - 2) * 4096, &tmO, lane_base + o_col, 1.f / l, h * 128,
-                     qb * 2 * TB + g * TB + quarter * 32, b, p.Lq, lane);
-      } else {
+      {
         const float inv = 1.f / l;
         const int qrow = qb * 2 * TB + g * TB + r;
         bf16* orow = p.O + (size_t)(b * p.Lq + qrow) * p.ldo + h * 128;
+        // 32-byte stores (whole sectors) where the rows are 32-byte aligned
+        const bool st32 = ((reinterpret_cast<uintptr_t>(p.O) & 31) | (p.ldo & 15)) == 0;
 #pragma unroll 1
         for (int c = 0; c < 4; ++c) {
           uint32_t u[32];
@@ -1081,19 +1074,30 @@ __global__ void __launch_bounds__(THREADS2, 1)
           tmem_ld_wait();
           reg_fence32(u);
           if (qrow < p.Lq) {
+            if (st32) {
 #pragma unroll
-            for (int q = 0; q < 4; ++q) {
-              float v[8];
+              for (int q = 0; q < 2; ++q) {
+                uint32_t w[8];
 #pragma unroll
-              for (int i = 0; i < 8; ++i) v[i] = __uint_as_float(u[q * 8 + i]) * inv;
-              store_bf16x8(orow + c * 32 + q * 8, v);
+                for (int i = 0; i < 8; ++i)
+                  w[i] = pack_bf16x2(__uint_as_float(u[q * 16 + 2 * i]) * inv,
+                                     __uint_as_float(u[q * 16 + 2 * i + 1]) * inv);
+                store_b32x8(orow + c * 32 + q * 16, w);
+              }
+            } else {
+#pragma unroll
+              for (int q = 0; q < 4; ++q) {
+                float v[8];
+#pragma unroll
+                for (int i = 0; i < 8; ++i) v[i] = __uint_as_float(u[q * 8 + i]) * inv;
+                store_bf16x8(orow + c * 32 + q * 8, v);
+              }
             }
           }
         }
       }
       ++cnt;
     }
-    if (TMA_O && lane == 0) bulk_wait<0>();  // this warp's O stores complete before exit
   }
 
   if (failed || *(volatile int*)err != 0) {
@@ -1152,8 +1156,6 @@ bool map_o(CUtensorMap* m, const bf16* ptr, int batch, int Lq, int cols, int ld)
 
 }  // namespace
 
-static int n_kv_of(const AttnArgs& a) { return (a.Lkv + TB - 1) / TB; }
-
 cudaError_t attention_tc_set_wait_limit(unsigned long long ns) {
   return fb_set_wait_limit_tu(ns);
 }
@@ -1201,13 +1203,12 @@ cudaError_t attention_tc(const AttnArgs& a, int* err, cudaStream_t st) {
   // more than one wave of 256-query CTAs: one persistent CTA per SM loops over them
   const bool persistent = a.tc_variant >= 3 || (two && a.tc_variant == 0 && ctas2 > sms);
   if (persistent) {
-    // items of at most 4 key tiles store O through TMA (see attn_tc2p_kernel)
-    auto kern = n_kv_of(a) <= 4 ? attn_tc2p_kernel<true> : attn_tc2p_kernel<false>;
+    auto kern = attn_tc2p_kernel;
     cudaError_t e =
         cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM2_BYTES);
     if (e != cudaSuccess) return e;
     const int grid = (int)(ctas2 < sms ? ctas2 : sms);
-    e = launch_k(kern, dim3(grid), dim3(THREADS2), SMEM2_BYTES, st, mq, mk, mv, mo, p);
+    e = launch_k(kern, dim3(grid), dim3(THREADS2), SMEM2_BYTES, st, mq, mk, mv, p);
     if (e != cudaSuccess) return e;
     return cudaGetLastError();
   }
