@@ -930,17 +930,20 @@ __global__ void __launch_bounds__(THREADS2, 1)
         for (int j = 0; j < n_kv && ok; ++j) {
           const bool more = j + 1 < n_kv;
           const uint32_t vt = vb + j;
-          if (!(ok = mbar_wait(&p_full[0], pc[0]++ & 1, err))) break;
+          // this step's V and next step's K tiles first: they are normally there already,
+          // and these waits then overlap the tensor pipe's last instructions of the
+          // previous batch instead of following the softmax's hand-off (the pipe holds
+          // about one instruction, so every wait between batches is idle pipe time)
           if (!(ok = mbar_wait(&v_full[vt & 1], (vt >> 1) & 1, err))) break;
-          tc_fence_after();
-          issue_pv(0, j);
-          if (ng == 1) tc_commit(&v_empty[vt & 1]);
           if (more) {
             const uint32_t kt = kb + j + 1;
             if (!(ok = mbar_wait(&k_full[kt % KS], (kt / KS) & 1, err))) break;
-            tc_fence_after();
-            issue_s(0, j + 1, ng);
           }
+          if (!(ok = mbar_wait(&p_full[0], pc[0]++ & 1, err))) break;
+          tc_fence_after();
+          issue_pv(0, j);
+          if (ng == 1) tc_commit(&v_empty[vt & 1]);
+          if (more) issue_s(0, j + 1, ng);
           if (ng == 1) continue;
           if (!(ok = mbar_wait(&p_full[1], pc[1]++ & 1, err))) break;
           tc_fence_after();
