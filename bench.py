@@ -657,6 +657,16 @@ def run_probe(args):
                           "nominal": 4096, "res": res}))
         m.close()
         return 0
+    if args.probe == "pipes":
+        res = {"mma_gap_mac_per_clk": {str(g): round(fb.fb_probe_mma_gap(g), 1)
+                                       for g in (0, 64, 128, 256, 512)},
+               "mufu_per_clk": {name: round(fb.fb_probe_mufu(op), 2)
+                                for op, name in enumerate(("ex2", "tanh", "rcp"))},
+               "tmem_load_128_columns_clocks": {"tensor_idle": round(fb.fb_probe_tmem_load(False), 1),
+                                                "tensor_busy": round(fb.fb_probe_tmem_load(True), 1)}}
+        print(json.dumps({"probe": "pipes", "res": res}))
+        m.close()
+        return 0
     if args.probe in ("gemm_shapes", "gemm_shapes_part", "attn_shapes", "breakdown"):
         call = None
     elif args.probe in ("gemm_refine_out", "gemm_refine_down"):
@@ -987,7 +997,7 @@ def main():
                     help="base: the draft-pool workload; cfg / sde: the same with guidance "
                          "or SDE steps")
     ap.add_argument("--probe", choices=["gemm", "gemm_resid", "gemm_out", "gemm_refine_out",
-                                        "gemm_refine_down", "attn", "attn_mma", "gemm_shapes", "gemm_shapes_part",
+                                        "gemm_refine_down", "attn", "attn_mma", "gemm_shapes", "gemm_shapes_part", "pipes",
                                         "attn_shapes", "breakdown", "pointwise",
                                         "attn_pool", "attn_pool_cross", "mma_rate"],
                     default=None)

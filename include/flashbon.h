@@ -392,6 +392,20 @@ fb_status fb_gemm_streamk_noalloc(void* stream, int M, int N, int K, const void*
  * frees two small device buffers and synchronises the device. FB_EINVAL for arguments
  * outside those ranges, FB_ECUDA on a CUDA error. */
 fb_status fb_probe_mma_rate(int issuers, int n, int reps, double* mac_per_clk);
+/* fb_probe_mma_gap: the same rate (MACs per SM clock, slowest SM) when one thread per SM
+ * issues 2048 batches of 8 instructions (M = N = 128, K = 16) and spins `gap` clocks
+ * (0 .. 100000) after each batch: how much work the tensor pipe holds queued while its
+ * issuing thread does something else. FB_EINVAL / FB_ECUDA as above. */
+fb_status fb_probe_mma_gap(int gap, double* mac_per_clk);
+/* fb_probe_mufu: results per SM clock (slowest SM) of one special-function operation,
+ * op 0 = ex2.approx.ftz.f32, 1 = tanh.approx.f32, 2 = rcp.approx.ftz.f32, with 256
+ * threads per SM each running 16 independent chains. FB_EINVAL / FB_ECUDA. */
+fb_status fb_probe_mufu(int op, double* per_clk);
+/* fb_probe_tmem_load: mean SM clocks from issuing four tcgen05.ld 32x32b.x32 (128 TMEM
+ * columns of a warp's lane quarter) to the end of their wait, over 2000 repetitions by
+ * 4 warps per SM, with the tensor pipe idle (busy = 0) or running M = N = 128 MMAs into
+ * other columns (busy != 0). FB_EINVAL / FB_ECUDA. */
+fb_status fb_probe_tmem_load(int busy, double* clocks);
 fb_status fb_set_device_wait_limit(unsigned long long ns);
 fb_status fb_test_fail_alloc(long k);
 long fb_test_alloc_calls(void);

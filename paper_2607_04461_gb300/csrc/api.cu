@@ -1444,6 +1444,93 @@ fb_status fb_test_fail_alloc(long k) {
 
 long fb_test_alloc_calls(void) { return g_alloc_calls.load(); }
 
+}  // extern "C"
+
+// Shared frame of the probes below: `n` 64-bit words of output (cycles), an error word and
+// a float sink on the device, one launch on the legacy stream, a device synchronisation.
+template <typename Launch>
+static fb_status run_probe(size_t n, std::vector<unsigned long long>& h, Launch launch) {
+  unsigned long long* cyc = nullptr;
+  int* err = nullptr;
+  float* sink = nullptr;
+  if (cudaMalloc(&cyc, n * sizeof(unsigned long long)) != cudaSuccess ||
+      cudaMalloc(&err, sizeof(int)) != cudaSuccess || cudaMalloc(&sink, sizeof(float)) != cudaSuccess) {
+    cudaFree(cyc);
+    cudaFree(err);
+    cudaFree(sink);
+    cudaGetLastError();
+    return fail(FB_ENOMEM, "cudaMalloc failed");
+  }
+  h.assign(n, 0ull);
+  int herr = 0;
+  cudaError_t e = cudaMemset(err, 0, sizeof(int));
+  if (e == cudaSuccess) e = cudaMemset(cyc, 0, n * sizeof(unsigned long long));
+  fb_stream_op_not_kernel();
+  if (e == cudaSuccess) e = launch(cyc, err, sink);
+  if (e == cudaSuccess) e = cudaDeviceSynchronize();
+  if (e == cudaSuccess)
+    e = cudaMemcpy(h.data(), cyc, n * sizeof(unsigned long long), cudaMemcpyDeviceToHost);
+  if (e == cudaSuccess) e = cudaMemcpy(&herr, err, sizeof(int), cudaMemcpyDeviceToHost);
+  cudaFree(cyc);
+  cudaFree(err);
+  cudaFree(sink);
+  if (e != cudaSuccess) return fail(FB_ECUDA, "probe failed: %s", cudaGetErrorString(e));
+  if (herr != 0) return fail(FB_ECUDA, "device wait timed out");
+  return FB_OK;
+}
+
+static fb_status device_sms(int* sms) {
+  int dev = 0;
+  CK(cudaGetDevice(&dev));
+  CK(cudaDeviceGetAttribute(sms, cudaDevAttrMultiProcessorCount, dev));
+  return FB_OK;
+}
+
+extern "C" {
+
+fb_status fb_probe_mma_gap(int gap, double* mac_per_clk) {
+  if (!mac_per_clk || gap < 0 || gap > 100000)
+    return fail(FB_EINVAL, "gap 0 .. 100000 clocks, non-NULL output");
+  int sms = 0;
+  CKS(device_sms(&sms));
+  const int batches = 2048;
+  std::vector<unsigned long long> h;
+  CKS(run_probe(sms, h, [&](unsigned long long* c, int* e, float*) {
+    return mma_gap_probe(gap, batches, sms, c, e, nullptr);
+  }));
+  const unsigned long long slowest = *std::max_element(h.begin(), h.end());
+  *mac_per_clk = 128.0 * 128 * 16 * 8.0 * batches / (double)slowest;
+  return FB_OK;
+}
+
+fb_status fb_probe_mufu(int op, double* per_clk) {
+  if (!per_clk || op < 0 || op > 2) return fail(FB_EINVAL, "op 0 (ex2), 1 (tanh), 2 (rcp)");
+  int sms = 0;
+  CKS(device_sms(&sms));
+  const int reps = 4096;
+  std::vector<unsigned long long> h;
+  CKS(run_probe(sms, h, [&](unsigned long long* c, int*, float* sink) {
+    return mufu_probe(op, reps, sms, c, sink, nullptr);
+  }));
+  const unsigned long long slowest = *std::max_element(h.begin(), h.end());
+  *per_clk = 256.0 * 16.0 * reps / (double)slowest;
+  return FB_OK;
+}
+
+fb_status fb_probe_tmem_load(int busy, double* clocks) {
+  if (!clocks) return fail(FB_EINVAL, "non-NULL output");
+  int sms = 0;
+  CKS(device_sms(&sms));
+  std::vector<unsigned long long> h;
+  CKS(run_probe((size_t)sms * 4, h, [&](unsigned long long* c, int* e, float* sink) {
+    return tmem_load_probe(2000, busy ? 1 : 0, sms, c, e, sink, nullptr);
+  }));
+  double sum = 0;
+  for (unsigned long long v : h) sum += (double)v;
+  *clocks = sum / (double)h.size();
+  return FB_OK;
+}
+
 fb_status fb_probe_mma_rate(int issuers, int n, int reps, double* mac_per_clk) {
   if (!mac_per_clk || issuers < 1 || issuers > 4 || (n != 64 && n != 128 && n != 256) ||
       issuers * n > 512 || reps < 1)

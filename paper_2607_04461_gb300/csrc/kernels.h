@@ -121,5 +121,11 @@ cudaError_t f32_to_bf16(const float* x, bf16* y, size_t n, cudaStream_t st);
 // One CTA per entry of `grid`, each timing (SM clock cycles, cycles[cta]) `reps` tcgen05.mma
 // kind::f16 instructions of M = 128, K = 16 and width N (64, 128 or 256) issued by each of
 // `issuers` warps (1-4) into accumulators of their own.
+cudaError_t mma_gap_probe(int gap, int batches, int grid, unsigned long long* cycles, int* err,
+                          cudaStream_t st);
+cudaError_t mufu_probe(int op, int reps, int grid, unsigned long long* cycles, float* sink,
+                       cudaStream_t st);
+cudaError_t tmem_load_probe(int reps, int busy, int grid, unsigned long long* cycles, int* err,
+                            float* sink, cudaStream_t st);
 cudaError_t mma_rate_probe(int issuers, int N, int reps, int grid, unsigned long long* cycles,
                            int* err, cudaStream_t st);

@@ -1,7 +1,15 @@
-// Measurement probe of the tensor pipe: how many MACs per SM clock tcgen05.mma kind::f16
-// sustains when 1, 2 or 4 warps (one elected thread each) issue `reps` M = 128, K = 16
-// instructions of width N into accumulators of their own (1-SM form, operands in shared
-// memory). The attention and GEMM kernels are judged against this rate.
+// Measurement probes of the SM's pipes, against which the attention and GEMM kernels are
+// judged:
+//  * mma_rate: how many MACs per SM clock tcgen05.mma kind::f16 sustains when 1, 2 or 4
+//    warps (one elected thread each) issue `reps` M = 128, K = 16 instructions of width N
+//    into accumulators of their own (1-SM form, operands in shared memory);
+//  * mma_gap: the same rate when one thread issues batches of 8 such instructions (N =
+//    128) with a spin of `gap` clocks after each batch (how much queued work hides a gap
+//    in the issuing thread);
+//  * mufu: ex2.approx, tanh.approx or rcp.approx results per SM clock (16 independent
+//    chains per thread, 256 threads per SM);
+//  * tmem_load: clocks from four 32x32b.x32 TMEM loads (128 columns) to their wait's end,
+//    with the tensor pipe idle or running.
 #include "kernels.h"
 
 namespace {
@@ -64,7 +72,173 @@ __global__ void __launch_bounds__(PROBE_THREADS, 1)
   }
 }
 
+// ---- issue gaps: batches of 8 MMAs (M = N = 128, K = 16) with `gap` clocks between them
+__global__ void __launch_bounds__(PROBE_THREADS, 1)
+    mma_gap_kernel(int gap, int batches, unsigned long long* cycles, int* err) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* sm = reinterpret_cast<uint8_t*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  __shared__ uint64_t bar;
+  __shared__ uint32_t holder;
+  if (threadIdx.x == 0) {
+    mbar_init(&bar, 1);
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (threadIdx.x / 32 == 0) tmem_alloc(&holder, 128);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tm = holder;
+  griddep_wait();
+  if (threadIdx.x == 0) {
+    const uint64_t ad = probe_desc_sw128(smem_u32(sm)), bd = probe_desc_sw128(smem_u32(sm) + 16384);
+    const uint32_t idesc = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(128 >> 3) << 17) |
+                           ((uint32_t)(128 >> 4) << 24);
+    const long long t0 = clock64();
+    for (int b = 0; b < batches; ++b) {
+#pragma unroll
+      for (int k = 0; k < 8; ++k) tc_mma_f16(tm, ad + 2 * (k & 3), bd + 2 * (k & 3), idesc, (b | k) ? 1u : 0u);
+      const long long c0 = clock64();
+      while (clock64() - c0 < gap) {
+      }
+    }
+    tc_commit(&bar);
+    if (mbar_wait(&bar, 0, err)) cycles[blockIdx.x] = clock64() - t0;
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (threadIdx.x / 32 == 0) {
+    tc_fence_after();
+    tmem_dealloc(tm, 128);
+  }
+}
+
+// ---- MUFU rates: 16 independent chains per thread of one operation
+constexpr int PROBE_THREADS2 = 256;  // the MUFU and TMEM-load probes: 8 warps
+template <int OP>
+__global__ void __launch_bounds__(PROBE_THREADS2, 1) mufu_kernel(int reps, unsigned long long* cycles,
+                                                                float* sink) {
+  griddep_wait();
+  float a[16];
+#pragma unroll
+  for (int i = 0; i < 16; ++i) a[i] = 0.001f * (float)(threadIdx.x + i) + 0.5f;
+  const long long t0 = clock64();
+  for (int r = 0; r < reps; ++r) {
+#pragma unroll
+    for (int i = 0; i < 16; ++i) {
+      float y;
+      if (OP == 0) asm volatile("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(a[i]));
+      else if (OP == 1) asm volatile("tanh.approx.f32 %0, %1;" : "=f"(y) : "f"(a[i]));
+      else asm volatile("rcp.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(a[i]));
+      a[i] = OP == 0 ? y - 1.0f : y + 0.5f;  // bounded chains
+    }
+  }
+  const long long t1 = clock64();
+  float acc = 0.f;
+#pragma unroll
+  for (int i = 0; i < 16; ++i) acc += a[i];
+  if (acc == 12345.f) sink[0] = acc;  // keeps the chains
+  if (threadIdx.x == 0) cycles[blockIdx.x] = t1 - t0;
+}
+
+// ---- TMEM load latency: warps 4-7 time `reps` loads of 128 columns (4 x 32x32b.x32, one
+// wait) of their lane quarter; with busy != 0, thread 0 keeps the tensor pipe running
+// (M = N = 128 MMAs into other columns) meanwhile
+__global__ void __launch_bounds__(PROBE_THREADS2, 1)
+    tmem_load_kernel(int reps, int busy, unsigned long long* cycles, int* err, float* sink) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* sm = reinterpret_cast<uint8_t*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  __shared__ uint64_t bar;
+  __shared__ uint32_t holder;
+  __shared__ volatile int done;
+  const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+  if (threadIdx.x == 0) {
+    done = 0;
+    mbar_init(&bar, 1);
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 0) tmem_alloc(&holder, 512);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tm = holder;
+  griddep_wait();
+  if (threadIdx.x == 0 && busy) {
+    const uint64_t ad = probe_desc_sw128(smem_u32(sm)), bd = probe_desc_sw128(smem_u32(sm) + 16384);
+    const uint32_t idesc = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(128 >> 3) << 17) |
+                           ((uint32_t)(128 >> 4) << 24);
+    for (int i = 0; i < 200000 && done < 4; ++i)
+      tc_mma_f16(tm, ad + 2 * (i & 3), bd + 2 * (i & 3), idesc, i ? 1u : 0u);
+    tc_commit(&bar);
+    mbar_wait(&bar, 0, err);
+  }
+  if (warp >= 4 && warp < 8) {
+    const uint32_t ta = tm + ((uint32_t)((warp & 3) * 32) << 16) + 256;
+    long long tot = 0;
+    float x = 0.f;
+    for (int it = 0; it < reps; ++it) {
+      uint32_t r[128];
+      const long long c0 = clock64();
+#pragma unroll
+      for (int c = 0; c < 4; ++c) tmem_ld32(ta + c * 32, r + c * 32);
+      tmem_ld_wait();
+#pragma unroll
+      for (int c = 0; c < 4; ++c) reg_fence32(r + c * 32);
+      // the second clock read takes a loaded value as an operand, so it cannot run before
+      // the data has arrived (a wait may return before its registers are written)
+      const float y = __uint_as_float(r[0]) + __uint_as_float(r[127]);
+      long long c1;
+      asm volatile("{\n\t.reg .f32 t;\n\tmov.b32 t, %1;\n\tmov.u64 %0, %%clock64;\n\t}"
+                   : "=l"(c1) : "f"(y) : "memory");
+      tot += c1 - c0;
+      x += y;
+    }
+    if (x == 12345.f) sink[0] = x;
+    if (lane == 0) cycles[blockIdx.x * 4 + (warp & 3)] = (unsigned long long)(tot / reps);
+    __syncwarp();
+    if (lane == 0) atomicAdd((int*)&done, 1);
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 0) {
+    tc_fence_after();
+    tmem_dealloc(tm, 512);
+  }
+}
+
 }  // namespace
+
+cudaError_t mma_gap_probe(int gap, int batches, int grid, unsigned long long* cycles, int* err,
+                          cudaStream_t st) {
+  if (gap < 0 || batches < 1 || grid < 1) return cudaErrorInvalidValue;
+  cudaError_t e = cudaFuncSetAttribute(mma_gap_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       PROBE_STAGE + 1024);
+  if (e != cudaSuccess) return e;
+  e = launch_k(mma_gap_kernel, dim3(grid), dim3(PROBE_THREADS), PROBE_STAGE + 1024, st, gap,
+               batches, cycles, err);
+  return e != cudaSuccess ? e : cudaGetLastError();
+}
+
+cudaError_t mufu_probe(int op, int reps, int grid, unsigned long long* cycles, float* sink,
+                       cudaStream_t st) {
+  if (op < 0 || op > 2 || reps < 1 || grid < 1) return cudaErrorInvalidValue;
+  auto k = op == 0 ? mufu_kernel<0> : op == 1 ? mufu_kernel<1> : mufu_kernel<2>;
+  cudaError_t e = launch_k(k, dim3(grid), dim3(PROBE_THREADS2), 0, st, reps, cycles, sink);
+  return e != cudaSuccess ? e : cudaGetLastError();
+}
+
+cudaError_t tmem_load_probe(int reps, int busy, int grid, unsigned long long* cycles, int* err,
+                            float* sink, cudaStream_t st) {
+  if (reps < 1 || grid < 1) return cudaErrorInvalidValue;
+  cudaError_t e = cudaFuncSetAttribute(tmem_load_kernel,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       PROBE_STAGE + 1024);
+  if (e != cudaSuccess) return e;
+  e = launch_k(tmem_load_kernel, dim3(grid), dim3(PROBE_THREADS2), PROBE_STAGE + 1024, st, reps,
+               busy, cycles, err, sink);
+  return e != cudaSuccess ? e : cudaGetLastError();
+}
 
 cudaError_t mma_rate_probe(int issuers, int N, int reps, int grid, unsigned long long* cycles,
                            int* err, cudaStream_t st) {

@@ -56,7 +56,7 @@ EXPORTS = ["fb_weights_count", "fb_weights_entry", "fb_init_model", "fb_free", "
            "fb_state_wait", "fb_set_sm_budget", "fb_sm_split_create", "fb_sm_split_info",
            "fb_sm_split_free", "fb_pipeline_step", "fb_set_device_wait_limit",
            "fb_test_fail_alloc", "fb_test_alloc_calls", "fb_test_poison_counters",
-           "fb_probe_mma_rate"]
+           "fb_probe_mma_rate", "fb_probe_mma_gap", "fb_probe_mufu", "fb_probe_tmem_load"]
 
 PAIR_VERIFIER = ctypes.CFUNCTYPE(ctypes.c_int, ctypes.c_void_p, ctypes.c_int, ctypes.c_int,
                                  ctypes.POINTER(ctypes.c_int))
@@ -112,6 +112,9 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
         "fb_test_alloc_calls": (ctypes.c_long, []),
         "fb_test_poison_counters": (I, [P]),
         "fb_probe_mma_rate": (I, [I, I, I, ctypes.POINTER(ctypes.c_double)]),
+        "fb_probe_mma_gap": (I, [I, ctypes.POINTER(ctypes.c_double)]),
+        "fb_probe_mufu": (I, [I, ctypes.POINTER(ctypes.c_double)]),
+        "fb_probe_tmem_load": (I, [I, ctypes.POINTER(ctypes.c_double)]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(L, name)
@@ -394,6 +397,27 @@ def fb_probe_mma_rate(issuers: int, n: int, reps: int = 16384) -> float:
     """Tensor-pipe MACs per SM clock with `issuers` issuing warps and M=128 x n MMAs."""
     out = ctypes.c_double()
     _check(load_library().fb_probe_mma_rate(int(issuers), int(n), int(reps), ctypes.byref(out)))
+    return out.value
+
+
+def fb_probe_mma_gap(gap: int) -> float:
+    """Tensor-pipe MACs per SM clock with a gap of `gap` clocks after every 8 MMAs."""
+    out = ctypes.c_double()
+    _check(load_library().fb_probe_mma_gap(int(gap), ctypes.byref(out)))
+    return out.value
+
+
+def fb_probe_mufu(op: int) -> float:
+    """Results per SM clock of ex2 (0), tanh (1) or rcp (2)."""
+    out = ctypes.c_double()
+    _check(load_library().fb_probe_mufu(int(op), ctypes.byref(out)))
+    return out.value
+
+
+def fb_probe_tmem_load(busy: bool) -> float:
+    """SM clocks of a 128-column TMEM load and its wait (tensor pipe idle or running)."""
+    out = ctypes.c_double()
+    _check(load_library().fb_probe_tmem_load(1 if busy else 0, ctypes.byref(out)))
     return out.value
 
 

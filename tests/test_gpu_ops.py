@@ -294,3 +294,20 @@ def test_attention_strided_qkv(model):
         want = O.attention(r[:, :D].reshape(L, heads, dh), r[:, D:2 * D].reshape(L, heads, dh),
                            r[:, 2 * D:].reshape(L, heads, dh)).reshape(L, D)
         assert rel_max(f64(o)[b * L:(b + 1) * L], want) <= 2e-2
+
+
+def test_pipe_probes_report_plausible_rates(model):
+    """The measurement probes run and report values inside what the hardware allows: the
+    tensor pipe at most 4096 MACs per SM clock (and at least half of it with no gap, less
+    with a long gap), a special-function rate above zero and at most 64 per SM clock, and
+    a TMEM load that takes clocks."""
+    full = fb.fb_probe_mma_gap(0)
+    gapped = fb.fb_probe_mma_gap(512)
+    assert 2048 <= full <= 4096 * 1.01
+    assert 0 < gapped < full
+    for op in range(3):
+        assert 0 < fb.fb_probe_mufu(op) <= 64
+    for busy in (False, True):
+        assert 10 < fb.fb_probe_tmem_load(busy) < 100000
+    with pytest.raises(fb.FlashBonError):
+        fb.fb_probe_mufu(3)
