@@ -661,7 +661,7 @@ def run_probe(args):
         res = {"mma_gap_mac_per_clk": {str(g): round(fb.fb_probe_mma_gap(g), 1)
                                        for g in (0, 64, 128, 256, 512)},
                "mufu_per_clk": {name: round(fb.fb_probe_mufu(op), 2)
-                                for op, name in enumerate(("ex2", "tanh", "rcp"))},
+                                for op, name in enumerate(("ex2", "tanh", "rcp", "ex2_f16x2"))},
                "tmem_load_128_columns_clocks": {"tensor_idle": round(fb.fb_probe_tmem_load(False), 1),
                                                 "tensor_busy": round(fb.fb_probe_tmem_load(True), 1)}}
         print(json.dumps({"probe": "pipes", "res": res}))

@@ -398,8 +398,9 @@ fb_status fb_probe_mma_rate(int issuers, int n, int reps, double* mac_per_clk);
  * issuing thread does something else. FB_EINVAL / FB_ECUDA as above. */
 fb_status fb_probe_mma_gap(int gap, double* mac_per_clk);
 /* fb_probe_mufu: results per SM clock (slowest SM) of one special-function operation,
- * op 0 = ex2.approx.ftz.f32, 1 = tanh.approx.f32, 2 = rcp.approx.ftz.f32, with 256
- * threads per SM each running 16 independent chains. FB_EINVAL / FB_ECUDA. */
+ * op 0 = ex2.approx.ftz.f32, 1 = tanh.approx.f32, 2 = rcp.approx.ftz.f32, 3 =
+ * ex2.approx.f16x2 (two results per instruction), with 256 threads per SM each running
+ * 16 independent chains. FB_EINVAL / FB_ECUDA. */
 fb_status fb_probe_mufu(int op, double* per_clk);
 /* fb_probe_tmem_load: mean SM clocks from issuing four tcgen05.ld 32x32b.x32 (128 TMEM
  * columns of a warp's lane quarter) to the end of their wait, over 2000 repetitions by

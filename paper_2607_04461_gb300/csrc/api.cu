@@ -1504,7 +1504,8 @@ fb_status fb_probe_mma_gap(int gap, double* mac_per_clk) {
 }
 
 fb_status fb_probe_mufu(int op, double* per_clk) {
-  if (!per_clk || op < 0 || op > 2) return fail(FB_EINVAL, "op 0 (ex2), 1 (tanh), 2 (rcp)");
+  if (!per_clk || op < 0 || op > 3)
+    return fail(FB_EINVAL, "op 0 (ex2), 1 (tanh), 2 (rcp), 3 (ex2 on f16 pairs)");
   int sms = 0;
   CKS(device_sms(&sms));
   const int reps = 4096;
@@ -1513,7 +1514,7 @@ fb_status fb_probe_mufu(int op, double* per_clk) {
     return mufu_probe(op, reps, sms, c, sink, nullptr);
   }));
   const unsigned long long slowest = *std::max_element(h.begin(), h.end());
-  *per_clk = 256.0 * 16.0 * reps / (double)slowest;
+  *per_clk = 256.0 * 16.0 * reps * (op == 3 ? 2.0 : 1.0) / (double)slowest;
   return FB_OK;
 }
 

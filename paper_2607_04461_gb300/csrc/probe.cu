@@ -6,8 +6,9 @@
 //  * mma_gap: the same rate when one thread issues batches of 8 such instructions (N =
 //    128) with a spin of `gap` clocks after each batch (how much queued work hides a gap
 //    in the issuing thread);
-//  * mufu: ex2.approx, tanh.approx or rcp.approx results per SM clock (16 independent
-//    chains per thread, 256 threads per SM);
+//  * mufu: ex2.approx, tanh.approx, rcp.approx or ex2.approx.f16x2 (two results per
+//    instruction) results per SM clock (16 independent chains per thread, 256 threads
+//    per SM);
 //  * tmem_load: clocks from four 32x32b.x32 TMEM loads (128 columns) to their wait's end,
 //    with the tensor pipe idle or running.
 #include "kernels.h"
@@ -122,10 +123,19 @@ __global__ void __launch_bounds__(PROBE_THREADS2, 1) mufu_kernel(int reps, unsig
   float a[16];
 #pragma unroll
   for (int i = 0; i < 16; ++i) a[i] = 0.001f * (float)(threadIdx.x + i) + 0.5f;
+  uint32_t hv[16];  // op 3: pairs of f16
+#pragma unroll
+  for (int i = 0; i < 16; ++i) hv[i] = 0x3800b800u ^ (uint32_t)(threadIdx.x & 7);  // {-0.5, 0.5}
   const long long t0 = clock64();
   for (int r = 0; r < reps; ++r) {
 #pragma unroll
     for (int i = 0; i < 16; ++i) {
+      if (OP == 3) {
+        uint32_t y;
+        asm volatile("ex2.approx.f16x2 %0, %1;" : "=r"(y) : "r"(hv[i]));
+        hv[i] = y ^ 0x40004000u;  // keeps the pairs in range (sign and exponent bits)
+        continue;
+      }
       float y;
       if (OP == 0) asm volatile("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(a[i]));
       else if (OP == 1) asm volatile("tanh.approx.f32 %0, %1;" : "=f"(y) : "f"(a[i]));
@@ -136,7 +146,7 @@ __global__ void __launch_bounds__(PROBE_THREADS2, 1) mufu_kernel(int reps, unsig
   const long long t1 = clock64();
   float acc = 0.f;
 #pragma unroll
-  for (int i = 0; i < 16; ++i) acc += a[i];
+  for (int i = 0; i < 16; ++i) acc += a[i] + (float)(hv[i] & 1u);
   if (acc == 12345.f) sink[0] = acc;  // keeps the chains
   if (threadIdx.x == 0) cycles[blockIdx.x] = t1 - t0;
 }
@@ -222,8 +232,9 @@ cudaError_t mma_gap_probe(int gap, int batches, int grid, unsigned long long* cy
 
 cudaError_t mufu_probe(int op, int reps, int grid, unsigned long long* cycles, float* sink,
                        cudaStream_t st) {
-  if (op < 0 || op > 2 || reps < 1 || grid < 1) return cudaErrorInvalidValue;
-  auto k = op == 0 ? mufu_kernel<0> : op == 1 ? mufu_kernel<1> : mufu_kernel<2>;
+  if (op < 0 || op > 3 || reps < 1 || grid < 1) return cudaErrorInvalidValue;
+  auto k = op == 0 ? mufu_kernel<0> : op == 1 ? mufu_kernel<1> : op == 2 ? mufu_kernel<2>
+                                                                         : mufu_kernel<3>;
   cudaError_t e = launch_k(k, dim3(grid), dim3(PROBE_THREADS2), 0, st, reps, cycles, sink);
   return e != cudaSuccess ? e : cudaGetLastError();
 }

@@ -408,7 +408,7 @@ def fb_probe_mma_gap(gap: int) -> float:
 
 
 def fb_probe_mufu(op: int) -> float:
-    """Results per SM clock of ex2 (0), tanh (1) or rcp (2)."""
+    """Results per SM clock of ex2 (0), tanh (1), rcp (2) or ex2 on f16 pairs (3)."""
     out = ctypes.c_double()
     _check(load_library().fb_probe_mufu(int(op), ctypes.byref(out)))
     return out.value

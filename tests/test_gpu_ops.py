@@ -305,9 +305,9 @@ def test_pipe_probes_report_plausible_rates(model):
     gapped = fb.fb_probe_mma_gap(512)
     assert 2048 <= full <= 4096 * 1.01
     assert 0 < gapped < full
-    for op in range(3):
-        assert 0 < fb.fb_probe_mufu(op) <= 64
+    for op in range(4):
+        assert 0 < fb.fb_probe_mufu(op) <= 128
     for busy in (False, True):
         assert 10 < fb.fb_probe_tmem_load(busy) < 100000
     with pytest.raises(fb.FlashBonError):
-        fb.fb_probe_mufu(3)
+        fb.fb_probe_mufu(4)
