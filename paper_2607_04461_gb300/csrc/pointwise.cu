@@ -463,9 +463,11 @@ cudaError_t qk_norm_rope(bf16* x, int rows, int ld, int D, int nseg, int col0, c
     case 256: return QKN(64, 1);
     case 512: return QKN(128, 1);
     case 1024: return QKN(128, 2);
-    // one warp per row (96 bytes in flight per thread), two rows per block: at 49920 x
-    // 2 x 1536 this runs at 6.1 TB/s against 5.4 with one row per block
-    case 1536: return QKN(32, 12, 2);
+    // one warp per row (96 bytes in flight per thread), four rows per block: on the
+    // 16-candidate probe (24960 rows x 2 x 1536) 5.04 TB/s against 4.90 with two rows
+    // per block and 4.60 with eight (at 49920 rows two rows per block gave 6.1 TB/s, one
+    // row 5.4)
+    case 1536: return QKN(32, 12, 4);
     case 2048: return QKN(128, 4);
     case 3072: return QKN(256, 3);
     case 4096: return QKN(256, 4);
