@@ -296,6 +296,34 @@ def test_attention_strided_qkv(model):
         assert rel_max(f64(o)[b * L:(b + 1) * L], want) <= 2e-2
 
 
+@pytest.mark.parametrize("ldo_pad,o_off", [(8, 0), (0, 8), (16, 0)],
+                         ids=["row_stride_16B", "base_16B", "row_stride_32B"])
+def test_attention_persistent_output_alignment(model, ldo_pad, o_off):
+    """The persistent kernel stores O rows in 32-byte pieces only where the rows are
+    32-byte aligned; a row stride or base aligned to 16 bytes only takes the 16-byte
+    stores. Columns outside the heads' output stay untouched."""
+    batch, L, heads, dh = 2, 300, 2, 128
+    D = heads * dh
+    ldo = D + ldo_pad
+    q = randn((batch * L, D), 91)
+    k = randn((batch * L, D), 92)
+    v = randn((batch * L, D), 93)
+    buf = torch.full((batch * L * ldo + o_off + 64,), 7.0, dtype=torch.bfloat16, device="cuda")
+    o_ptr = buf.data_ptr() + 2 * o_off
+    fb.fb_op_attention(model.handle, q, D, k, D, v, D, o_ptr, ldo, batch, L, L, L, heads, dh, 4)
+    torch.cuda.synchronize()
+    rows = buf[o_off:o_off + batch * L * ldo].view(batch * L, ldo)
+    got = f64(rows[:, :D])
+    if ldo_pad:
+        assert torch.all(rows[:, D:] == 7.0)
+    qn, kn, vn = f64(q), f64(k), f64(v)
+    for b in range(batch):
+        sl = slice(b * L, (b + 1) * L)
+        want = O.attention(qn[sl].reshape(L, heads, dh), kn[sl].reshape(L, heads, dh),
+                           vn[sl].reshape(L, heads, dh)).reshape(L, D)
+        assert rel_max(got[sl], want) <= 2e-2
+
+
 def test_pipe_probes_report_plausible_rates(model):
     """The measurement probes run and report values inside what the hardware allows: the
     tensor pipe at most 4096 MACs per SM clock (and at least half of it with no gap, less
