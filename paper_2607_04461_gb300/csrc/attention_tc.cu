@@ -942,17 +942,20 @@ __global__ void __launch_bounds__(THREADS2, 1)
           if (!(ok = mbar_wait(&p_full[0], pc[0]++ & 1, err))) break;
           tc_fence_after();
           issue_pv(0, j);
+          // a group's O rows are complete with its last PV: its epilogue may start while
+          // the other group's last PV runs
+          if (!more) tc_commit(&o_done[0]);
           if (ng == 1) tc_commit(&v_empty[vt & 1]);
           if (more) issue_s(0, j + 1, ng);
           if (ng == 1) continue;
           if (!(ok = mbar_wait(&p_full[1], pc[1]++ & 1, err))) break;
           tc_fence_after();
           issue_pv(1, j);
+          if (!more) tc_commit(&o_done[1]);
           tc_commit(&v_empty[vt & 1]);
           if (more) issue_s(1, j + 1, ng);
         }
         if (!ok) break;
-        for (int g = 0; g < ng; ++g) tc_commit(&o_done[g]);
         kb += n_kv;
         vb += n_kv;
       }
