@@ -663,7 +663,15 @@ def run_probe(args):
                "mufu_per_clk": {name: round(fb.fb_probe_mufu(op), 2)
                                 for op, name in enumerate(("ex2", "tanh", "rcp", "ex2_f16x2"))},
                "tmem_load_128_columns_clocks": {"tensor_idle": round(fb.fb_probe_tmem_load(False), 1),
-                                                "tensor_busy": round(fb.fb_probe_tmem_load(True), 1)}}
+                                                "tensor_busy": round(fb.fb_probe_tmem_load(True), 1)},
+               "mma_mix_mac_per_clk": {f"{fname}/loaders{ld}/gap{gp}": round(fb.fb_probe_mma_mix(f, ld, gp), 1)
+                                       for f, fname in enumerate(("ss", "ss_mn", "ts_mn", "attn_step",
+                                                                  "attn_step_commits"))
+                                       for ld, gp in ((0, 0), (7, 800), (7, 0))},
+               "mma_mix_softmax_loaders_mac_per_clk": {
+                   f"{fname}/loaders{ld}/gap{gp}": round(fb.fb_probe_mma_mix(5 + f, ld, gp), 1)
+                   for f, fname in enumerate(("ss", "ss_mn", "ts_mn", "attn_step", "attn_step_commits"))
+                   for ld, gp in ((3, 0), (7, 0), (7, 400))}}
         print(json.dumps({"probe": "pipes", "res": res}))
         m.close()
         return 0

@@ -407,6 +407,19 @@ fb_status fb_probe_mufu(int op, double* per_clk);
  * 4 warps per SM, with the tensor pipe idle (busy = 0) or running M = N = 128 MMAs into
  * other columns (busy != 0). FB_EINVAL / FB_ECUDA. */
 fb_status fb_probe_tmem_load(int busy, double* clocks);
+/* fb_probe_mma_mix: MACs per SM clock (slowest SM) of 1024 batches shaped like one
+ * attention step of one 128-query tile, issued by one thread per SM: 8 instructions
+ * (M = N = 128, K = 16) into one accumulator, in form 0 (A and B K-major in shared
+ * memory), 1 (B MN-major in shared memory, as V is read) or 2 (B MN-major, A read from
+ * TMEM, as P is read), then 8 K-major shared-memory instructions into another. Warps
+ * 1..loaders (0-7) meanwhile load 128 TMEM columns of their lane quarter, store 64 and
+ * spin loader_gap clocks (0 .. 100000), as softmax warps do. Forms 3 and 4 issue one whole
+ * attention step per batch instead (32 instructions: PV and S of two query tiles over
+ * distinct operand slices), form 4 with the attention's tcgen05.commit instructions.
+ * Forms 5-9 are forms 0-4 with the loaders also doing a softmax row's arithmetic
+ * (maximum, 128 exponentials, sum, bf16 packing) between load and store.
+ * FB_EINVAL / FB_ECUDA. */
+fb_status fb_probe_mma_mix(int form, int loaders, int loader_gap, double* mac_per_clk);
 fb_status fb_set_device_wait_limit(unsigned long long ns);
 fb_status fb_test_fail_alloc(long k);
 long fb_test_alloc_calls(void);

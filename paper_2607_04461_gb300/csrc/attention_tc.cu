@@ -67,6 +67,43 @@ __device__ __forceinline__ uint64_t desc_mn_sw128(uint32_t saddr, uint32_t lbo) 
   return d;
 }
 
+// The same descriptors split into their two 32-bit words. The upper word (stride byte
+// offset 1024 B, version bit, 128-byte swizzle) is one constant; the lower word holds the
+// start address >> 4 (bits 0-13) and the leading byte offset >> 4 (bits 16-29), so the
+// descriptor of an operand slice `off` bytes further on is lower word + (off >> 4) (shared
+// addresses stay below 256 KB: the start field cannot carry into the offset field).
+constexpr uint32_t DESC_HI = (1024u >> 4) | (1u << 14) | (2u << 29);
+__device__ __forceinline__ uint32_t desc_lo_k(uint32_t saddr) {
+  return ((saddr & 0x3FFFFu) >> 4) | (1u << 16);
+}
+__device__ __forceinline__ uint32_t desc_lo_mn(uint32_t saddr, uint32_t lbo) {
+  return ((saddr & 0x3FFFFu) >> 4) | (((lbo >> 4) & 0x3FFFu) << 16);
+}
+// tcgen05.mma kind::f16 from the descriptors' lower words (A and B in shared memory, or A
+// in TMEM): the issuing thread spends one add per operand and instruction, which keeps it
+// ahead of the tensor pipe while softmax warps share its SM sub-partition
+__device__ __forceinline__ void tc_mma_ss_lo(uint32_t d_tmem, uint32_t alo, uint32_t blo,
+                                             uint32_t hi, uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t.reg .b64 da, db;\n\t"
+      "setp.ne.b32 p, %5, 0;\n\t"
+      "mov.b64 da, {%1, %3};\n\t"
+      "mov.b64 db, {%2, %3};\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], da, db, %4, p;\n\t}" ::"r"(d_tmem),
+      "r"(alo), "r"(blo), "r"(hi), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+__device__ __forceinline__ void tc_mma_ts_lo(uint32_t d_tmem, uint32_t a_tmem, uint32_t blo,
+                                             uint32_t hi, uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t.reg .b64 db;\n\t"
+      "setp.ne.b32 p, %5, 0;\n\t"
+      "mov.b64 db, {%2, %3};\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], db, %4, p;\n\t}" ::"r"(d_tmem),
+      "r"(a_tmem), "r"(blo), "r"(hi), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
 // instruction descriptor of the S MMA with N = 32 * nch keys (N field: N >> 3 at bit 17)
 __device__ __forceinline__ uint32_t idesc_keys(uint32_t idesc128, int nch) {
   return (idesc128 & ~(0x3Fu << 17)) | ((uint32_t)(4 * nch) << 17);
@@ -873,8 +910,12 @@ __global__ void __launch_bounds__(THREADS2, 1)
       const uint32_t idesc_s = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(TB >> 3) << 17) |
                                ((uint32_t)(TB >> 4) << 24);
       const uint32_t idesc_pv = idesc_s | (1u << 16);
-      const uint32_t qa = smem_u32(Qs);
       const int last_nch = (p.Lkv - (n_kv - 1) * TB + 31) >> 5;
+      // descriptor lower words of the Q buffers, K slot 0 and V slot 0 (the other slots lie
+      // K_BYTES / V_BYTES further on)
+      const uint32_t dhi = DESC_HI;
+      const uint32_t q_lo[2] = {desc_lo_k(smem_u32(Qs)), desc_lo_k(smem_u32(Qs + Q_BYTES))};
+      const uint32_t k_lo = desc_lo_k(smem_u32(Ks)), v_lo = desc_lo_mn(smem_u32(Vs), SUB);
       uint32_t kb = 0, vb = 0, pc[2] = {0u, 0u};  // K, V tiles and P tiles (per group) consumed
       bool ok = true;
       int it = 0;
@@ -882,22 +923,20 @@ __global__ void __launch_bounds__(THREADS2, 1)
       // its K slot, and of the last tile also the Q buffer
       auto issue_s = [&](int g, int j, int ng) {
         const uint32_t kt = kb + j;
-        const uint32_t ka = smem_u32(Ks + (kt % KS) * K_BYTES);
-        const uint32_t qg = qa + g * Q_BYTES;
+        const uint32_t ka = k_lo + (kt % KS) * (K_BYTES >> 4);
+        const uint32_t qg = q_lo[g];
         if (j + 1 < n_kv || last_nch == 4) {
 #pragma unroll
           for (int kk = 0; kk < 8; ++kk) {
-            const uint32_t off = (kk >> 2) * SUB + (kk & 3) * 32;
-            tc_mma_f16(tmem + g * TB, desc_k_sw128(qg + off), desc_k_sw128(ka + off), idesc_s,
-                       kk ? 1u : 0u);
+            const uint32_t off = ((kk >> 2) * SUB + (kk & 3) * 32) >> 4;
+            tc_mma_ss_lo(tmem + g * TB, qg + off, ka + off, dhi, idesc_s, kk ? 1u : 0u);
           }
         } else {
           const uint32_t idesc = idesc_keys(idesc_s, last_nch);
 #pragma unroll 1
           for (int kk = 0; kk < 8; ++kk) {
-            const uint32_t off = (kk >> 2) * SUB + (kk & 3) * 32;
-            tc_mma_f16(tmem + g * TB, desc_k_sw128(qg + off), desc_k_sw128(ka + off), idesc,
-                       kk ? 1u : 0u);
+            const uint32_t off = ((kk >> 2) * SUB + (kk & 3) * 32) >> 4;
+            tc_mma_ss_lo(tmem + g * TB, qg + off, ka + off, dhi, idesc, kk ? 1u : 0u);
           }
         }
         tc_commit(&s_full[g]);
@@ -907,17 +946,17 @@ __global__ void __launch_bounds__(THREADS2, 1)
         }
       };
       auto issue_pv = [&](int g, int j) {
-        const uint32_t va = smem_u32(Vs + ((vb + j) & 1) * V_BYTES);
+        const uint32_t va = v_lo + ((vb + j) & 1) * (V_BYTES >> 4);
         if (j + 1 < n_kv || last_nch == 4) {
 #pragma unroll
           for (int kk = 0; kk < 8; ++kk)
-            tc_mma_f16_ts(tmem + O_COL + g * TB, tmem + g * TB + kk * 8,
-                          desc_mn_sw128(va + kk * 2048, SUB), idesc_pv, (j | kk) ? 1u : 0u);
+            tc_mma_ts_lo(tmem + O_COL + g * TB, tmem + g * TB + kk * 8, va + kk * (2048 >> 4),
+                         dhi, idesc_pv, (j | kk) ? 1u : 0u);
         } else {
 #pragma unroll 1
           for (int kk = 0; kk < 2 * last_nch; ++kk)
-            tc_mma_f16_ts(tmem + O_COL + g * TB, tmem + g * TB + kk * 8,
-                          desc_mn_sw128(va + kk * 2048, SUB), idesc_pv, (j | kk) ? 1u : 0u);
+            tc_mma_ts_lo(tmem + O_COL + g * TB, tmem + g * TB + kk * 8, va + kk * (2048 >> 4),
+                         dhi, idesc_pv, (j | kk) ? 1u : 0u);
         }
       };
       for (int item = blockIdx.x; item < n_items && ok; item += gridDim.x, ++it) {

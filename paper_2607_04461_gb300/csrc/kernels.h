@@ -127,5 +127,7 @@ cudaError_t mufu_probe(int op, int reps, int grid, unsigned long long* cycles, f
                        cudaStream_t st);
 cudaError_t tmem_load_probe(int reps, int busy, int grid, unsigned long long* cycles, int* err,
                             float* sink, cudaStream_t st);
+cudaError_t mma_mix_probe(int form, int loaders, int loader_gap, int batches, int grid,
+                          unsigned long long* cycles, int* err, float* sink, cudaStream_t st);
 cudaError_t mma_rate_probe(int issuers, int N, int reps, int grid, unsigned long long* cycles,
                            int* err, cudaStream_t st);

@@ -56,7 +56,8 @@ EXPORTS = ["fb_weights_count", "fb_weights_entry", "fb_init_model", "fb_free", "
            "fb_state_wait", "fb_set_sm_budget", "fb_sm_split_create", "fb_sm_split_info",
            "fb_sm_split_free", "fb_pipeline_step", "fb_set_device_wait_limit",
            "fb_test_fail_alloc", "fb_test_alloc_calls", "fb_test_poison_counters",
-           "fb_probe_mma_rate", "fb_probe_mma_gap", "fb_probe_mufu", "fb_probe_tmem_load"]
+           "fb_probe_mma_rate", "fb_probe_mma_gap", "fb_probe_mufu", "fb_probe_tmem_load",
+           "fb_probe_mma_mix"]
 
 PAIR_VERIFIER = ctypes.CFUNCTYPE(ctypes.c_int, ctypes.c_void_p, ctypes.c_int, ctypes.c_int,
                                  ctypes.POINTER(ctypes.c_int))
@@ -115,6 +116,7 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
         "fb_probe_mma_gap": (I, [I, ctypes.POINTER(ctypes.c_double)]),
         "fb_probe_mufu": (I, [I, ctypes.POINTER(ctypes.c_double)]),
         "fb_probe_tmem_load": (I, [I, ctypes.POINTER(ctypes.c_double)]),
+        "fb_probe_mma_mix": (I, [I, I, I, ctypes.POINTER(ctypes.c_double)]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(L, name)
@@ -418,6 +420,17 @@ def fb_probe_tmem_load(busy: bool) -> float:
     """SM clocks of a 128-column TMEM load and its wait (tensor pipe idle or running)."""
     out = ctypes.c_double()
     _check(load_library().fb_probe_tmem_load(1 if busy else 0, ctypes.byref(out)))
+    return out.value
+
+
+def fb_probe_mma_mix(form: int, loaders: int = 0, loader_gap: int = 0) -> float:
+    """Tensor-pipe MACs per SM clock of attention-step-shaped MMA batches (form 0: both
+    operands K-major in shared memory, 1: B MN-major, 2: B MN-major and A from TMEM, 3: a
+    whole attention step, 4: the same with its commits; 5-9: forms 0-4 with softmax
+    arithmetic in the loaders) with `loaders` warps reading and writing TMEM meanwhile."""
+    out = ctypes.c_double()
+    _check(load_library().fb_probe_mma_mix(int(form), int(loaders), int(loader_gap),
+                                           ctypes.byref(out)))
     return out.value
 
 
