@@ -48,61 +48,9 @@ struct Params {
   int batch, heads;  // the persistent kernel's item count
 };
 
-__device__ __forceinline__ uint64_t desc_k_sw128(uint32_t saddr) {
-  uint64_t d = (uint64_t)((saddr & 0x3FFFFu) >> 4);
-  d |= (uint64_t)1 << 16;               // leading byte offset (unused, K-major swizzled)
-  d |= (uint64_t)(1024 >> 4) << 32;     // 8-row groups 1024 B apart
-  d |= (uint64_t)1 << 46;
-  d |= (uint64_t)2 << 61;               // 128-byte swizzle
-  return d;
-}
-// MN-major, 128-byte swizzle: 64 consecutive N elements per 128-byte row, one row per K;
-// 8-row (K) groups 1024 B apart (stride byte offset), the next 64 N elements lbo bytes on.
-__device__ __forceinline__ uint64_t desc_mn_sw128(uint32_t saddr, uint32_t lbo) {
-  uint64_t d = (uint64_t)((saddr & 0x3FFFFu) >> 4);
-  d |= (uint64_t)((lbo >> 4) & 0x3FFFu) << 16;
-  d |= (uint64_t)(1024 >> 4) << 32;
-  d |= (uint64_t)1 << 46;
-  d |= (uint64_t)2 << 61;
-  return d;
-}
-
-// The same descriptors split into their two 32-bit words. The upper word (stride byte
-// offset 1024 B, version bit, 128-byte swizzle) is one constant; the lower word holds the
-// start address >> 4 (bits 0-13) and the leading byte offset >> 4 (bits 16-29), so the
-// descriptor of an operand slice `off` bytes further on is lower word + (off >> 4) (shared
-// addresses stay below 256 KB: the start field cannot carry into the offset field).
-constexpr uint32_t DESC_HI = (1024u >> 4) | (1u << 14) | (2u << 29);
-__device__ __forceinline__ uint32_t desc_lo_k(uint32_t saddr) {
-  return ((saddr & 0x3FFFFu) >> 4) | (1u << 16);
-}
-__device__ __forceinline__ uint32_t desc_lo_mn(uint32_t saddr, uint32_t lbo) {
-  return ((saddr & 0x3FFFFu) >> 4) | (((lbo >> 4) & 0x3FFFu) << 16);
-}
-// tcgen05.mma kind::f16 from the descriptors' lower words (A and B in shared memory, or A
-// in TMEM): the issuing thread spends one add per operand and instruction, which keeps it
-// ahead of the tensor pipe while softmax warps share its SM sub-partition
-__device__ __forceinline__ void tc_mma_ss_lo(uint32_t d_tmem, uint32_t alo, uint32_t blo,
-                                             uint32_t hi, uint32_t idesc, uint32_t accumulate) {
-  asm volatile(
-      "{\n\t.reg .pred p;\n\t.reg .b64 da, db;\n\t"
-      "setp.ne.b32 p, %5, 0;\n\t"
-      "mov.b64 da, {%1, %3};\n\t"
-      "mov.b64 db, {%2, %3};\n\t"
-      "tcgen05.mma.cta_group::1.kind::f16 [%0], da, db, %4, p;\n\t}" ::"r"(d_tmem),
-      "r"(alo), "r"(blo), "r"(hi), "r"(idesc), "r"(accumulate)
-      : "memory");
-}
-__device__ __forceinline__ void tc_mma_ts_lo(uint32_t d_tmem, uint32_t a_tmem, uint32_t blo,
-                                             uint32_t hi, uint32_t idesc, uint32_t accumulate) {
-  asm volatile(
-      "{\n\t.reg .pred p;\n\t.reg .b64 db;\n\t"
-      "setp.ne.b32 p, %5, 0;\n\t"
-      "mov.b64 db, {%2, %3};\n\t"
-      "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], db, %4, p;\n\t}" ::"r"(d_tmem),
-      "r"(a_tmem), "r"(blo), "r"(hi), "r"(idesc), "r"(accumulate)
-      : "memory");
-}
+// Operand layouts (descriptors from desc_lo_k / desc_lo_mn): Q, K and P are K-major with
+// 128-byte swizzle, 8-row groups 1024 B apart; V is MN-major with 128-byte swizzle, 64
+// consecutive head dims per 128-byte row (one row per key), the next 64 dims SUB bytes on.
 
 // instruction descriptor of the S MMA with N = 32 * nch keys (N field: N >> 3 at bit 17)
 __device__ __forceinline__ uint32_t idesc_keys(uint32_t idesc128, int nch) {
@@ -300,23 +248,23 @@ __global__ void __launch_bounds__(THREADS, 1)
       const uint32_t idesc_s = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(TB >> 3) << 17) |
                                ((uint32_t)(TB >> 4) << 24);
       const uint32_t idesc_pv = idesc_s | (1u << 16);  // B (V) is MN-major
-      const uint32_t qa = smem_u32(Qs), pa = smem_u32(Ps);
+      const uint32_t dhi = DESC_HI;
+      const uint32_t q_lo = desc_lo_k(smem_u32(Qs)), p_lo = desc_lo_k(smem_u32(Ps));
+      const uint32_t k_lo = desc_lo_k(smem_u32(Ks)), v_lo = desc_lo_mn(smem_u32(Vs), SUB);
       auto issue_s = [&](int j) {
-        const uint32_t ka = smem_u32(Ks + (j % KSLOT) * K_BYTES);
+        const uint32_t ka = k_lo + (j % KSLOT) * (K_BYTES >> 4);
         if (j + 1 < n_kv || last_nch == 4) {
 #pragma unroll
           for (int kk = 0; kk < 8; ++kk) {
-            const uint32_t off = (kk >> 2) * SUB + (kk & 3) * 32;
-            tc_mma_f16(tmem + (j & 1) * TB, desc_k_sw128(qa + off), desc_k_sw128(ka + off),
-                       idesc_s, kk ? 1u : 0u);
+            const uint32_t off = ((kk >> 2) * SUB + (kk & 3) * 32) >> 4;
+            tc_mma_ss_lo(tmem + (j & 1) * TB, q_lo + off, ka + off, dhi, idesc_s, kk ? 1u : 0u);
           }
         } else {
           const uint32_t idesc = idesc_keys(idesc_s, last_nch);
 #pragma unroll 1
           for (int kk = 0; kk < 8; ++kk) {
-            const uint32_t off = (kk >> 2) * SUB + (kk & 3) * 32;
-            tc_mma_f16(tmem + (j & 1) * TB, desc_k_sw128(qa + off), desc_k_sw128(ka + off),
-                       idesc, kk ? 1u : 0u);
+            const uint32_t off = ((kk >> 2) * SUB + (kk & 3) * 32) >> 4;
+            tc_mma_ss_lo(tmem + (j & 1) * TB, q_lo + off, ka + off, dhi, idesc, kk ? 1u : 0u);
           }
         }
         tc_commit(&s_full[j & 1]);
@@ -334,20 +282,20 @@ __global__ void __launch_bounds__(THREADS, 1)
           if (!mbar_wait(p_full, j & 1, err)) { failed = true; break; }
           if (!mbar_wait(&v_full[j & 1], (j >> 1) & 1, err)) { failed = true; break; }
           tc_fence_after();
-          const uint32_t va = smem_u32(Vs + (j & 1) * V_BYTES);
+          const uint32_t va = v_lo + (j & 1) * (V_BYTES >> 4);
           if (j + 1 < n_kv || last_nch == 4) {
 #pragma unroll
             for (int kk = 0; kk < 8; ++kk) {
-              const uint32_t off = (kk >> 2) * SUB + (kk & 3) * 32;
-              tc_mma_f16(tmem + O_COL, desc_k_sw128(pa + off), desc_mn_sw128(va + kk * 2048, SUB),
-                         idesc_pv, (j | kk) ? 1u : 0u);
+              const uint32_t off = ((kk >> 2) * SUB + (kk & 3) * 32) >> 4;
+              tc_mma_ss_lo(tmem + O_COL, p_lo + off, va + kk * (2048 >> 4), dhi, idesc_pv,
+                           (j | kk) ? 1u : 0u);
             }
           } else {
 #pragma unroll 1
             for (int kk = 0; kk < 2 * last_nch; ++kk) {  // 16 keys per step
-              const uint32_t off = (kk >> 2) * SUB + (kk & 3) * 32;
-              tc_mma_f16(tmem + O_COL, desc_k_sw128(pa + off), desc_mn_sw128(va + kk * 2048, SUB),
-                         idesc_pv, (j | kk) ? 1u : 0u);
+              const uint32_t off = ((kk >> 2) * SUB + (kk & 3) * 32) >> 4;
+              tc_mma_ss_lo(tmem + O_COL, p_lo + off, va + kk * (2048 >> 4), dhi, idesc_pv,
+                           (j | kk) ? 1u : 0u);
             }
           }
           tc_commit(&v_empty[j & 1]);
@@ -481,15 +429,6 @@ __global__ void __launch_bounds__(THREADS, 1)
 constexpr int THREADS2 = 320;
 constexpr int SMEM2_BYTES = 2 * Q_BYTES + KSLOT * K_BYTES + VSLOT * V_BYTES + 1024 + 256;
 
-__device__ __forceinline__ void tc_mma_f16_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t bdesc,
-                                              uint32_t idesc, uint32_t accumulate) {
-  asm volatile(
-      "{\n\t.reg .pred p;\n\t"
-      "setp.ne.b32 p, %4, 0;\n\t"
-      "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}" ::"r"(d_tmem),
-      "r"(a_tmem), "l"(bdesc), "r"(idesc), "r"(accumulate)
-      : "memory");
-}
 
 __global__ void __launch_bounds__(THREADS2, 1)
     attn_tc2_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
@@ -582,7 +521,9 @@ __global__ void __launch_bounds__(THREADS2, 1)
       const uint32_t idesc_s = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(TB >> 3) << 17) |
                                ((uint32_t)(TB >> 4) << 24);
       const uint32_t idesc_pv = idesc_s | (1u << 16);
-      const uint32_t qa = smem_u32(Qs);
+      const uint32_t dhi = DESC_HI;
+      const uint32_t q_lo[2] = {desc_lo_k(smem_u32(Qs)), desc_lo_k(smem_u32(Qs + Q_BYTES))};
+      const uint32_t k_lo = desc_lo_k(smem_u32(Ks)), v_lo = desc_lo_mn(smem_u32(Vs), SUB);
       const int two = qb * 2 * TB + TB < p.Lq;  // both tiles hold queries (as for the Q load)
       // real keys of the last key tile, in 32-key chunks (see attn_tc_kernel)
       const int last_nch = (p.Lkv - (n_kv - 1) * TB + 31) >> 5;
@@ -590,39 +531,37 @@ __global__ void __launch_bounds__(THREADS2, 1)
       // (last_nch < 4 chunks of 32 keys) issues S with N = 32 * last_nch and PV over those
       // keys only
       auto issue_s = [&](int g, int j) {
-        const uint32_t ka = smem_u32(Ks + (j % KSLOT) * K_BYTES);
-        const uint32_t qg = qa + g * Q_BYTES;
+        const uint32_t ka = k_lo + (j % KSLOT) * (K_BYTES >> 4);
+        const uint32_t qg = q_lo[g];
         if (j + 1 < n_kv || last_nch == 4) {
 #pragma unroll
           for (int kk = 0; kk < 8; ++kk) {
-            const uint32_t off = (kk >> 2) * SUB + (kk & 3) * 32;
-            tc_mma_f16(tmem + g * TB, desc_k_sw128(qg + off), desc_k_sw128(ka + off), idesc_s,
-                       kk ? 1u : 0u);
+            const uint32_t off = ((kk >> 2) * SUB + (kk & 3) * 32) >> 4;
+            tc_mma_ss_lo(tmem + g * TB, qg + off, ka + off, dhi, idesc_s, kk ? 1u : 0u);
           }
         } else {
           const uint32_t idesc = idesc_keys(idesc_s, last_nch);
 #pragma unroll 1
           for (int kk = 0; kk < 8; ++kk) {
-            const uint32_t off = (kk >> 2) * SUB + (kk & 3) * 32;
-            tc_mma_f16(tmem + g * TB, desc_k_sw128(qg + off), desc_k_sw128(ka + off), idesc,
-                       kk ? 1u : 0u);
+            const uint32_t off = ((kk >> 2) * SUB + (kk & 3) * 32) >> 4;
+            tc_mma_ss_lo(tmem + g * TB, qg + off, ka + off, dhi, idesc, kk ? 1u : 0u);
           }
         }
         tc_commit(&s_full[g]);
         if (g == 1 || two == 0) tc_commit(&k_empty[j % KSLOT]);  // every tile's S_j done
       };
       auto issue_pv = [&](int g, int j) {
-        const uint32_t va = smem_u32(Vs + (j & 1) * V_BYTES);
+        const uint32_t va = v_lo + (j & 1) * (V_BYTES >> 4);
         if (j + 1 < n_kv || last_nch == 4) {
 #pragma unroll
           for (int kk = 0; kk < 8; ++kk)
-            tc_mma_f16_ts(tmem + O_COL + g * TB, tmem + g * TB + kk * 8,
-                          desc_mn_sw128(va + kk * 2048, SUB), idesc_pv, (j | kk) ? 1u : 0u);
+            tc_mma_ts_lo(tmem + O_COL + g * TB, tmem + g * TB + kk * 8, va + kk * (2048 >> 4),
+                         dhi, idesc_pv, (j | kk) ? 1u : 0u);
         } else {
 #pragma unroll 1
           for (int kk = 0; kk < 2 * last_nch; ++kk)  // 16 keys per step
-            tc_mma_f16_ts(tmem + O_COL + g * TB, tmem + g * TB + kk * 8,
-                          desc_mn_sw128(va + kk * 2048, SUB), idesc_pv, (j | kk) ? 1u : 0u);
+            tc_mma_ts_lo(tmem + O_COL + g * TB, tmem + g * TB + kk * 8, va + kk * (2048 >> 4),
+                         dhi, idesc_pv, (j | kk) ? 1u : 0u);
         }
       };
       bool ok = mbar_wait(q_full, 0, err) && mbar_wait(&k_full[0], 0, err);

@@ -323,6 +323,44 @@ __device__ __forceinline__ void reg_fence32(uint32_t* r) {
                  "+r"(r[30]), "+r"(r[31]));
 }
 
+// Shared-memory matrix descriptors with 128-byte swizzle, split into their two 32-bit
+// words. The upper word (stride byte offset 1024 B, version bit, 128-byte swizzle) is one
+// constant; the lower word holds the start address >> 4 (bits 0-13) and the leading byte
+// offset >> 4 (bits 16-29), so the
+// descriptor of an operand slice `off` bytes further on is lower word + (off >> 4) (shared
+// addresses stay below 256 KB: the start field cannot carry into the offset field).
+constexpr uint32_t DESC_HI = (1024u >> 4) | (1u << 14) | (2u << 29);
+__device__ __forceinline__ uint32_t desc_lo_k(uint32_t saddr) {
+  return ((saddr & 0x3FFFFu) >> 4) | (1u << 16);
+}
+__device__ __forceinline__ uint32_t desc_lo_mn(uint32_t saddr, uint32_t lbo) {
+  return ((saddr & 0x3FFFFu) >> 4) | (((lbo >> 4) & 0x3FFFu) << 16);
+}
+// tcgen05.mma kind::f16 from the descriptors' lower words (A and B in shared memory, or A
+// in TMEM): the issuing thread spends one add per operand and instruction, which keeps it
+// ahead of the tensor pipe while softmax warps share its SM sub-partition
+__device__ __forceinline__ void tc_mma_ss_lo(uint32_t d_tmem, uint32_t alo, uint32_t blo,
+                                             uint32_t hi, uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t.reg .b64 da, db;\n\t"
+      "setp.ne.b32 p, %5, 0;\n\t"
+      "mov.b64 da, {%1, %3};\n\t"
+      "mov.b64 db, {%2, %3};\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], da, db, %4, p;\n\t}" ::"r"(d_tmem),
+      "r"(alo), "r"(blo), "r"(hi), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+__device__ __forceinline__ void tc_mma_ts_lo(uint32_t d_tmem, uint32_t a_tmem, uint32_t blo,
+                                             uint32_t hi, uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t.reg .b64 db;\n\t"
+      "setp.ne.b32 p, %5, 0;\n\t"
+      "mov.b64 db, {%2, %3};\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], db, %4, p;\n\t}" ::"r"(d_tmem),
+      "r"(a_tmem), "r"(blo), "r"(hi), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
 // ---- clusters and the 2-SM (cta_group::2) forms -----------------------------------
 __device__ __forceinline__ uint32_t cluster_ctarank() {
   uint32_t r;
