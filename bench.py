@@ -658,6 +658,8 @@ def run_probe(args):
         m.close()
         return 0
     if args.probe == "pipes":
+        MIX_FORMS = ("ss", "ss_mn", "ts_mn", "attn_step", "attn_step_commits",
+                     "attn_step_hoisted", "attn_step_hoisted_commits")
         res = {"mma_gap_mac_per_clk": {str(g): round(fb.fb_probe_mma_gap(g), 1)
                                        for g in (0, 64, 128, 256, 512)},
                "mufu_per_clk": {name: round(fb.fb_probe_mufu(op), 2)
@@ -665,12 +667,11 @@ def run_probe(args):
                "tmem_load_128_columns_clocks": {"tensor_idle": round(fb.fb_probe_tmem_load(False), 1),
                                                 "tensor_busy": round(fb.fb_probe_tmem_load(True), 1)},
                "mma_mix_mac_per_clk": {f"{fname}/loaders{ld}/gap{gp}": round(fb.fb_probe_mma_mix(f, ld, gp), 1)
-                                       for f, fname in enumerate(("ss", "ss_mn", "ts_mn", "attn_step",
-                                                                  "attn_step_commits"))
+                                       for f, fname in enumerate(MIX_FORMS)
                                        for ld, gp in ((0, 0), (7, 800), (7, 0))},
                "mma_mix_softmax_loaders_mac_per_clk": {
-                   f"{fname}/loaders{ld}/gap{gp}": round(fb.fb_probe_mma_mix(5 + f, ld, gp), 1)
-                   for f, fname in enumerate(("ss", "ss_mn", "ts_mn", "attn_step", "attn_step_commits"))
+                   f"{fname}/loaders{ld}/gap{gp}": round(fb.fb_probe_mma_mix(7 + f, ld, gp), 1)
+                   for f, fname in enumerate(MIX_FORMS)
                    for ld, gp in ((3, 0), (7, 0), (7, 400))}}
         print(json.dumps({"probe": "pipes", "res": res}))
         m.close()

@@ -415,10 +415,11 @@ fb_status fb_probe_tmem_load(int busy, double* clocks);
  * 1..loaders (0-7) meanwhile load 128 TMEM columns of their lane quarter, store 64 and
  * spin loader_gap clocks (0 .. 100000), as softmax warps do. Forms 3 and 4 issue one whole
  * attention step per batch instead (32 instructions: PV and S of two query tiles over
- * distinct operand slices), form 4 with the attention's tcgen05.commit instructions.
- * Forms 5-9 are forms 0-4 with the loaders also doing a softmax row's arithmetic
- * (maximum, 128 exponentials, sum, bf16 packing) between load and store.
- * FB_EINVAL / FB_ECUDA. */
+ * distinct operand slices, each descriptor built from its address), form 4 with the
+ * attention's tcgen05.commit instructions; forms 5 and 6 are forms 3 and 4 with the
+ * descriptors' lower words hoisted (one add per operand and instruction). Forms 7-13 are
+ * forms 0-6 with the loaders also doing a softmax row's arithmetic (maximum, 128
+ * exponentials, sum, bf16 packing) between load and store. FB_EINVAL / FB_ECUDA. */
 fb_status fb_probe_mma_mix(int form, int loaders, int loader_gap, double* mac_per_clk);
 fb_status fb_set_device_wait_limit(unsigned long long ns);
 fb_status fb_test_fail_alloc(long k);

@@ -1519,9 +1519,9 @@ fb_status fb_probe_mufu(int op, double* per_clk) {
 }
 
 fb_status fb_probe_mma_mix(int form, int loaders, int loader_gap, double* mac_per_clk) {
-  if (!mac_per_clk || form < 0 || form > 9 || loaders < 0 || loaders > 7 || loader_gap < 0 ||
+  if (!mac_per_clk || form < 0 || form > 13 || loaders < 0 || loaders > 7 || loader_gap < 0 ||
       loader_gap > 100000)
-    return fail(FB_EINVAL, "form 0..9, loaders 0..7, loader_gap 0..100000, non-NULL output");
+    return fail(FB_EINVAL, "form 0..13, loaders 0..7, loader_gap 0..100000, non-NULL output");
   int sms = 0;
   CKS(device_sms(&sms));
   const int batches = 1024;
@@ -1530,7 +1530,7 @@ fb_status fb_probe_mma_mix(int form, int loaders, int loader_gap, double* mac_pe
     return mma_mix_probe(form, loaders, loader_gap, batches, sms, c, e, sink, nullptr);
   }));
   const unsigned long long slowest = *std::max_element(h.begin(), h.end());
-  const double per_batch = form % 5 >= 3 ? 32.0 : 16.0;
+  const double per_batch = form % 7 >= 3 ? 32.0 : 16.0;
   *mac_per_clk = 128.0 * 128 * 16 * per_batch * batches / (double)slowest;
   return FB_OK;
 }

@@ -763,7 +763,7 @@ __global__ void __launch_bounds__(THREADS2, 1)
   uint64_t* k_full = bars + 2;         // [KS]
   uint64_t* k_empty = bars + 5;        // [KS]
   uint64_t* v_full = bars + 8;         // [2]
-  uint64_t* v_empty = bars + 10;       // [2]
+  // bars + 10, + 11: unused (a V slot is released by the K slot release of the next tile)
   uint64_t* s_full = bars + 12;        // [2 groups]
   uint64_t* p_full = bars + 14;        // [2 groups]
   uint64_t* o_done = bars + 16;        // [2 groups]
@@ -785,7 +785,6 @@ __global__ void __launch_bounds__(THREADS2, 1)
     }
     for (int s = 0; s < 2; ++s) {
       mbar_init(&v_full[s], 1);
-      mbar_init(&v_empty[s], 1);
       mbar_init(&s_full[s], 1);
       mbar_init(&p_full[s], 4);
       mbar_init(&o_done[s], 1);
@@ -835,7 +834,13 @@ __global__ void __launch_bounds__(THREADS2, 1)
         const int xq = h * 128, kv_row0 = b * p.kv_batch_rows;
         for (int j = 0; j < n_kv; ++j, ++vt) {
           const int s = vt & 1;
-          if (!mbar_wait(&v_empty[s], ((vt >> 1) & 1) ^ 1u, err)) { failed = true; break; }
+          // slot s last held tile vt - 2; its PV MMAs are done once the S MMAs of tile
+          // vt - 1 are (the issuer issues those after them): the K slot release of tile
+          // vt - 1 (K and V tiles are counted alike)
+          if (vt >= 2) {
+            const uint32_t t = vt - 1;
+            if (!mbar_wait(&k_empty[t % KS], (t / KS) & 1, err)) { failed = true; break; }
+          }
           uint8_t* st = Vs + s * V_BYTES;
           const int y = kv_row0 + j * TB;
           mbar_expect_tx(&v_full[s], V_BYTES);
@@ -923,14 +928,12 @@ __global__ void __launch_bounds__(THREADS2, 1)
           // a group's O rows are complete with its last PV: its epilogue may start while
           // the other group's last PV runs
           if (!more) tc_commit(&o_done[0]);
-          if (ng == 1) tc_commit(&v_empty[vt & 1]);
           if (more) issue_s(0, j + 1, ng);
           if (ng == 1) continue;
           if (!(ok = mbar_wait(&p_full[1], pc[1]++ & 1, err))) break;
           tc_fence_after();
           issue_pv(1, j);
           if (!more) tc_commit(&o_done[1]);
-          tc_commit(&v_empty[vt & 1]);
           if (more) issue_s(1, j + 1, ng);
         }
         if (!ok) break;

@@ -227,7 +227,9 @@ __global__ void __launch_bounds__(PROBE_THREADS2, 1)
 // 256-319, as PV reads P), then 8 K-major instructions into D1 (columns 128-255, as S).
 // Forms 3 and 4 issue the attention kernel's whole step instead (32 instructions per
 // batch: PV_A, S_A, PV_B, S_B over its shared-memory rings and TMEM map, every operand
-// slice distinct), form 4 with its tcgen05.commit after S_A, PV_B and S_B (two).
+// slice distinct), form 4 with its tcgen05.commit after S_A, PV_B and S_B (two). Forms 3
+// and 4 build each descriptor from its address per instruction; forms 5 and 6 are forms
+// 3 and 4 with the descriptors' lower words hoisted (one add per operand).
 // Warps 1..loaders meanwhile each load columns 128-255 of their lane quarter (4 x
 // 32x32b.x32, one wait), store 64 columns (2 x 32x32b.x32 into columns 384-447) and spin
 // `loader_gap` clocks, until thread 0 is done (at most 1 << 20 rounds). With SOFTMAX the
@@ -293,7 +295,29 @@ __global__ void __launch_bounds__(PROBE_THREADS2, 1)
                            ((uint32_t)(128 >> 4) << 24);
     const uint32_t idesc_mn = idesc | (1u << 16);
     const long long t0 = clock64();
-    for (int b = 0; b < batches && FORM >= 3; ++b) {
+    // forms 5 and 6: the same step from descriptor lower words hoisted out of the loop
+    const uint32_t dhi = DESC_HI, q_lo = desc_lo_k(base), k_lo = desc_lo_k(base + 65536);
+    const uint32_t v_lo = desc_lo_mn(base + 163840, 16384);
+    for (int b = 0; b < batches && FORM >= 5; ++b) {
+      const uint32_t ka = k_lo + (uint32_t)(b % 3) * 2048, va = v_lo + (uint32_t)(b & 1) * 2048;
+#pragma unroll
+      for (int g = 0; g < 2; ++g) {
+#pragma unroll
+        for (int k = 0; k < 8; ++k)
+          tc_mma_ts_lo(tm + 256 + 128 * g, tm + 128 * g + 8 * k, va + k * 128, dhi, idesc_mn,
+                       (b | k) ? 1u : 0u);
+        if (FORM == 6 && g == 1) tc_commit(&bar2[1]);
+        const uint32_t qa = q_lo + (uint32_t)g * 2048;
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+          const uint32_t off = ((k >> 2) * 16384 + (k & 3) * 32) >> 4;
+          tc_mma_ss_lo(tm + 128 * g, qa + off, ka + off, dhi, idesc, k ? 1u : 0u);
+        }
+        if (FORM == 6) tc_commit(&bar2[0]);
+        if (FORM == 6 && g == 1) tc_commit(&bar2[2]);
+      }
+    }
+    for (int b = 0; b < batches && FORM >= 3 && FORM < 5; ++b) {
       // one attention step: Q tiles at 0 and 32 KB, K ring (3 x 32 KB) from 64 KB, V ring
       // (2 x 32 KB) from 160 KB; TMEM S_A|P_A, S_B|P_B, O_A, O_B at columns 0/128/256/384
       const uint32_t ka = base + 65536 + (uint32_t)(b % 3) * 32768;
@@ -389,16 +413,18 @@ __global__ void __launch_bounds__(PROBE_THREADS2, 1)
 
 cudaError_t mma_mix_probe(int form, int loaders, int loader_gap, int batches, int grid,
                           unsigned long long* cycles, int* err, float* sink, cudaStream_t st) {
-  if (form < 0 || form > 9 || loaders < 0 || loaders > 7 || loader_gap < 0 || batches < 1 ||
+  if (form < 0 || form > 13 || loaders < 0 || loaders > 7 || loader_gap < 0 || batches < 1 ||
       grid < 1)
     return cudaErrorInvalidValue;
   using K = void (*)(int, int, int, unsigned long long*, int*, float*);
-  const K ks[10] = {mma_mix_kernel<0, false>, mma_mix_kernel<1, false>, mma_mix_kernel<2, false>,
-                    mma_mix_kernel<3, false>, mma_mix_kernel<4, false>,
+  const K ks[14] = {mma_mix_kernel<0, false>, mma_mix_kernel<1, false>, mma_mix_kernel<2, false>,
+                    mma_mix_kernel<3, false>, mma_mix_kernel<4, false>, mma_mix_kernel<5, false>,
+                    mma_mix_kernel<6, false>,
                     mma_mix_kernel<0, true>,  mma_mix_kernel<1, true>,  mma_mix_kernel<2, true>,
-                    mma_mix_kernel<3, true>,  mma_mix_kernel<4, true>};
+                    mma_mix_kernel<3, true>,  mma_mix_kernel<4, true>,  mma_mix_kernel<5, true>,
+                    mma_mix_kernel<6, true>};
   const K k = ks[form];
-  const int smem = (form % 5 >= 3 ? 7 * 32768 : PROBE_STAGE) + 1024;
+  const int smem = (form % 7 >= 3 ? 7 * 32768 : PROBE_STAGE) + 1024;
   cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
   e = launch_k(k, dim3(grid), dim3(PROBE_THREADS2), smem, st, loaders, loader_gap, batches,

@@ -426,8 +426,9 @@ def fb_probe_tmem_load(busy: bool) -> float:
 def fb_probe_mma_mix(form: int, loaders: int = 0, loader_gap: int = 0) -> float:
     """Tensor-pipe MACs per SM clock of attention-step-shaped MMA batches (form 0: both
     operands K-major in shared memory, 1: B MN-major, 2: B MN-major and A from TMEM, 3: a
-    whole attention step, 4: the same with its commits; 5-9: forms 0-4 with softmax
-    arithmetic in the loaders) with `loaders` warps reading and writing TMEM meanwhile."""
+    whole attention step, 4: the same with its commits, 5 and 6: forms 3 and 4 with hoisted
+    descriptor words; 7-13: forms 0-6 with softmax arithmetic in the loaders) with `loaders`
+    warps reading and writing TMEM meanwhile."""
     out = ctypes.c_double()
     _check(load_library().fb_probe_mma_mix(int(form), int(loaders), int(loader_gap),
                                            ctypes.byref(out)))

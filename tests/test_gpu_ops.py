@@ -337,10 +337,10 @@ def test_pipe_probes_report_plausible_rates(model):
         assert 0 < fb.fb_probe_mufu(op) <= 128
     for busy in (False, True):
         assert 10 < fb.fb_probe_tmem_load(busy) < 100000
-    for form in range(10):
+    for form in range(14):
         for loaders, gap in ((0, 0), (7, 0)):
             assert 500 < fb.fb_probe_mma_mix(form, loaders, gap) < 4200
     with pytest.raises(fb.FlashBonError):
-        fb.fb_probe_mma_mix(10)
+        fb.fb_probe_mma_mix(14)
     with pytest.raises(fb.FlashBonError):
         fb.fb_probe_mufu(4)
