@@ -738,7 +738,10 @@ __global__ void __launch_bounds__(THREADS2, 1)
 // time share their K/V tiles in L2. Per CTA the work of consecutive items overlaps:
 //  * the producer loads the next item's Q as soon as the current item's last S MMAs are
 //    done (q_empty) and carries on through the K/V rings, whose slots and phases count
-//    across items;
+//    across items; the slots are released by a softmax thread that has seen a tile's last
+//    S MMAs done, so the MMA issuer commits only what the softmax groups wait for (each
+//    tcgen05.commit holds up the issuing thread while softmax warps share its SM
+//    sub-partition);
 //  * the MMA issuer starts the next item's S MMAs right after the current item's last PV
 //    (the tensor pipe runs in order, so S_g overwrites P_g only after PV_g has read it);
 //  * each softmax group stores its O rows (o_done, one phase per item of the group) while
@@ -884,10 +887,6 @@ __global__ void __launch_bounds__(THREADS2, 1)
           }
         }
         tc_commit(&s_full[g]);
-        if (g == ng - 1) {
-          tc_commit(&k_empty[kt % KS]);
-          if (j == n_kv - 1) tc_commit(q_empty);
-        }
       };
       auto issue_pv = [&](int g, int j) {
         const uint32_t va = v_lo + ((vb + j) & 1) * (V_BYTES >> 4);
@@ -949,14 +948,25 @@ __global__ void __launch_bounds__(THREADS2, 1)
     const int r = quarter * 32 + lane;
     const uint32_t lane_base = tmem + ((uint32_t)(quarter * 32) << 16);
     const uint32_t s_col = g * TB, o_col = O_COL + g * TB;
-    uint32_t cnt = 0;  // items this group has worked on
-    for (int item = blockIdx.x; item < n_items && !failed; item += gridDim.x) {
+    uint32_t cnt = 0;   // items this group has worked on
+    uint32_t kbase = 0;  // K tiles of the CTA's earlier items (numbered as the producer does)
+    // the group whose S MMAs come last in a key tile (B, or A where B has no work) releases
+    // the tile's K slot, and at the item's last tile the Q buffer, once its S is done: the
+    // issuer's S MMAs of a tile follow its PV MMAs of the tile before, so this also frees
+    // that tile's V slot
+    const bool lead = (warp & 3) == 2 && lane == 0;  // one thread per group
+    for (int item = blockIdx.x; item < n_items && !failed; item += gridDim.x, kbase += n_kv) {
       const int qb = item % nqb;
       if (qb * 2 * TB + g * TB >= p.Lq) continue;  // this tile lies past Lq: no work
+      const bool last_group = g == 1 || qb * 2 * TB + TB >= p.Lq;
       float m_used = -INFINITY, l = 0.f;
       for (int j = 0; j < n_kv; ++j) {
         const bool ok = mbar_wait(&s_full[g], (cnt * (uint32_t)n_kv + j) & 1, err);
         if (!__all_sync(0xffffffffu, ok)) { failed = true; break; }
+        if (lead && last_group) {
+          mbar_arrive(&k_empty[(kbase + j) % KS]);
+          if (j == n_kv - 1) mbar_arrive(q_empty);
+        }
         tc_fence_after();
         float s[128];
         {
