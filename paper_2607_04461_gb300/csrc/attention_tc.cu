@@ -268,7 +268,6 @@ __global__ void __launch_bounds__(THREADS, 1)
           }
         }
         tc_commit(&s_full[j & 1]);
-        tc_commit(&k_empty[j % KSLOT]);  // K_j is no longer needed once S_j is done
       };
       if (mbar_wait(q_full, 0, err) && mbar_wait(&k_full[0], 0, err)) {
         tc_fence_after();
@@ -298,7 +297,6 @@ __global__ void __launch_bounds__(THREADS, 1)
                            (j | kk) ? 1u : 0u);
             }
           }
-          tc_commit(&v_empty[j & 1]);
           tc_commit(o_done);
         }
       } else {
@@ -312,9 +310,14 @@ __global__ void __launch_bounds__(THREADS, 1)
     const uint32_t lane_base = tmem + ((uint32_t)(quarter * 32) << 16);
     float m_used = -INFINITY, l = 0.f;
     uint8_t* prow = Ps + r * 128;  // this row inside each 64-key sub-tile
+    // one softmax thread releases K_j once S_j is done and V_{j-1} once PV_{j-1} is, so
+    // the MMA issuer commits only what the softmax waits for (each tcgen05.commit holds up
+    // the issuing thread while softmax warps share its SM sub-partition)
+    const bool lead = warp == 2 && lane == 0;
     for (int j = 0; j < n_kv && !failed; ++j) {
       const bool ok = mbar_wait(&s_full[j & 1], (j >> 1) & 1, err);
       if (!__all_sync(0xffffffffu, ok)) { failed = true; break; }
+      if (lead) mbar_arrive(&k_empty[j % KSLOT]);
       tc_fence_after();
       float s[128];
       {
@@ -340,6 +343,7 @@ __global__ void __launch_bounds__(THREADS, 1)
         // PV_{j-1} must be done before P is overwritten and before O is touched
         const bool ok2 = mbar_wait(o_done, (j - 1) & 1, err);
         if (!__all_sync(0xffffffffu, ok2)) { failed = true; break; }
+        if (lead) mbar_arrive(&v_empty[(j - 1) & 1]);
         tc_fence_after();
       }
       if (j == 0) {
