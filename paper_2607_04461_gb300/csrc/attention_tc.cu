@@ -1191,16 +1191,17 @@ cudaError_t attention_tc(const AttnArgs& a, int* err, cudaStream_t st) {
   p.err = err;
   p.batch = a.batch;
   p.heads = a.heads;
-  // 256-query CTAs share each K/V tile between two query tiles and overlap one tile's
-  // softmax with the other's MMAs; one costs about 1.4 times a 128-query CTA (measured:
-  // 4 x 1560 queries x 12 heads, 5 waves of 128-query CTAs 93.8 us, 3 waves of 256-query
-  // CTAs 79.8 us). The choice compares waves (for the persistent kernel, items per CTA):
-  // on 152 SMs, 1 x 1560 queries x 12 heads is 2 waves of 128-query CTAs (156) or 1 of
-  // 256-query CTAs (84); on a 40-SM partition it is 4 waves against 3 (1.4 x 3 > 4).
+  // 256-query items share each K/V tile between two query tiles and overlap one tile's
+  // softmax with the other's MMAs; in the persistent kernel one costs about 1.25 times a
+  // 128-query CTA (measured on a 40-SM partition, 1 x 1560 queries x 12 heads: 4 waves of
+  // 128-query CTAs 68.3 us self / 30.9 us cross, 3 items per CTA 64.7 / 25.6 us). The
+  // choice compares waves (for the persistent kernel, items per CTA): on 152 SMs that
+  // shape is 2 waves of 128-query CTAs (156) or 1 item per CTA (84), on 40 SMs 4 against
+  // 3; only where both fit one wave do the shorter 128-query CTAs win.
   const long ctas1 = (long)((a.Lq + TB - 1) / TB) * a.heads * a.batch;
   const long ctas2 = (long)((a.Lq + 2 * TB - 1) / (2 * TB)) * a.heads * a.batch;
   const long w1 = (ctas1 + sms - 1) / sms, w2 = (ctas2 + sms - 1) / sms;
-  const bool two = a.tc_variant >= 2 || (a.tc_variant == 0 && 10 * w1 >= 14 * w2);
+  const bool two = a.tc_variant >= 2 || (a.tc_variant == 0 && 4 * w1 >= 5 * w2);
   // 256-query items run in the persistent kernel (one CTA per SM looping over them, or one
   // item per CTA when they fit one wave: its MMA issue and slot releases are the leaner
   // ones, 1 x 1560 queries x 12 heads 25.8 -> 24.5 us); tc_variant 2 keeps the one-item
