@@ -215,7 +215,8 @@ ATTN_CASES = [
     (2, 1560, 1560, 2, 128, False),   # Wan2.1 self-attention length, ragged last tile
     (3, 256, 128, 1, 128, False),     # exact tile multiples
     (2, 129, 257, 2, 128, True),      # one row / one key past a tile
-    # grids of more than one wave of 128-query CTAs take the 256-query kernel (P in TMEM)
+    # grids of more than one wave of 128-query CTAs take the persistent 256-query kernel
+    # (P in TMEM)
     (4, 1560, 1560, 12, 128, False),
     (9, 600, 512, 12, 128, True),     # last CTA: tile A partly valid, tile B past Lq
     # the last key tile's MMAs cover only its 32-key chunks of real keys
