@@ -388,9 +388,8 @@ def test_wide_two_step_draft(wide):
 def test_wan13_refine_on_a_partition_matches_the_whole_gpu(wan13_pool):
     """The refine as the bench runs it: one candidate on a 40-SM partition, where the FFN
     down-projection takes the stream-K split and attention three 256-query items per
-    persistent CTA. Against
-    the same refine on the whole GPU (whose draft path the oracle checks above) only fp32
-    summation orders differ."""
+    persistent CTA. Against the same refine on the whole GPU (whose draft path the oracle
+    checks above) only fp32 summation orders differ."""
     cfg, w, m = wan13_pool
     z = synth.make_latents(cfg, 1)[0]
     ctx = synth.make_text(cfg)
