@@ -136,6 +136,23 @@ def test_null_model_is_rejected(lib):
     lib.fb_free(None)
 
 
+@pytest.mark.parametrize("call", [
+    lambda lib, out: lib.fb_probe_mma_gap(-1, out),
+    lambda lib, out: lib.fb_probe_mma_gap(100001, out),
+    lambda lib, out: lib.fb_probe_mufu(4, out),
+    lambda lib, out: lib.fb_probe_mma_rate(3, 256, 16, out),   # 3 x 256 > 512 TMEM columns
+    lambda lib, out: lib.fb_probe_mma_rate(1, 96, 16, out),
+    lambda lib, out: lib.fb_probe_mma_mix(14, 0, 0, out),
+    lambda lib, out: lib.fb_probe_mma_mix(0, 8, 0, out),
+    lambda lib, out: lib.fb_probe_mma_mix(0, 7, 100001, out),
+    lambda lib, out: lib.fb_probe_tmem_load(0, None),
+])
+def test_probes_reject_bad_arguments_before_touching_the_device(lib, call):
+    out = ctypes.c_double()
+    assert call(lib, ctypes.byref(out)) == fb.FB_EINVAL
+    assert lib.fb_last_error()
+
+
 # ---- Stage 2 selection (host logic) ---------------------------------------------------
 
 @pytest.mark.parametrize("seed", range(12))
