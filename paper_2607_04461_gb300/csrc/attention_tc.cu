@@ -1197,7 +1197,8 @@ cudaError_t attention_tc(const AttnArgs& a, int* err, cudaStream_t st) {
   // 128-query CTAs 68.3 us self / 30.9 us cross, 3 items per CTA 64.7 / 25.6 us). The
   // choice compares waves (for the persistent kernel, items per CTA): on 152 SMs that
   // shape is 2 waves of 128-query CTAs (156) or 1 item per CTA (84), on 40 SMs 4 against
-  // 3; only where both fit one wave do the shorter 128-query CTAs win.
+  // 3. The shorter 128-query CTAs remain only where the 256-query form saves no waves
+  // (both fit one wave, or Lq <= 128).
   const long ctas1 = (long)((a.Lq + TB - 1) / TB) * a.heads * a.batch;
   const long ctas2 = (long)((a.Lq + 2 * TB - 1) / (2 * TB)) * a.heads * a.batch;
   const long w1 = (ctas1 + sms - 1) / sms, w2 = (ctas2 + sms - 1) / sms;
