@@ -328,8 +328,8 @@ fb_status fb_op_gemm(fb_model* m, int M, int N, int K, const void* A, const void
  * (the tcgen05 kernel for head_dim 128, the mma.sync kernel for 64), 1 = force the
  * mma.sync kernel, 2 / 3 = force the tcgen05 kernel with 128- / 256-query CTAs, 4 = force
  * the persistent 256-query kernel (at most one CTA per SM looping over the (batch, head,
- * query-tile pair) items; the automatic choice unless the 128- and 256-query forms
- * both fit one wave)
+ * query-tile pair) items; the automatic choice unless the 256-query form saves no
+ * waves: both forms fit one wave, or Lq <= 128)
  * (2-4: head_dim 128 only, else FB_EINVAL). */
 fb_status fb_op_attention(fb_model* m, const void* Q, int ldq, const void* K, int ldk,
                           const void* V, int ldv, void* O, int ldo, int batch, int Lq,
